@@ -1,0 +1,443 @@
+"""Pins of the fp64 oracle against what the paper and the mathematics fix.
+
+Each test checks the oracle against something other than itself: a value
+worked by hand from the paper's equations (tests/golden/), a closed form, an
+invariant, a special case that reduces to a library routine, or brute force.
+"""
+import itertools
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import mpcache_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _golden(name):
+    out = {}
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            key, *vals = line.split()
+            out.setdefault(key, []).append([float(v) for v in vals])
+    return out
+
+
+# --------------------------------------------------------- worked examples --
+
+def test_similarity_worked_example():
+    g = _golden("eq1_eq2_eq3_cluster_similarity.txt")
+    q = np.array(g["q"][0])
+    keys = np.array(g["k"])
+    lev = O.cluster_pyramid(keys, 3, (), 0.6)[0]
+    assert np.array_equal(lev.r_max[0], g["r_max"][0])
+    assert np.array_equal(lev.r_min[0], g["r_min"][0])
+    assert np.allclose(lev.rep[0], g["rep_alpha_0.6"][0], atol=1e-15)
+    assert O.sim_max_dot(q, keys) == g["max_dot"][0][0]
+    assert O.sim_bound(q, lev.r_max[0], lev.r_min[0]) == g["bound"][0][0]
+    for a in ("0.6", "1.0", "0.0"):
+        want = g["linear_alpha_" + a][0][0]
+        assert abs(O.sim_linear(q, lev.r_max[0], lev.r_min[0], float(a)) - want) < 1e-14
+    assert abs(O.sim_average(q, keys) - g["average"][0][0]) < 1e-15
+
+
+def test_static_window_worked_example():
+    g = _golden("static_window_scores.txt")
+    k = np.array(g["keys"][0])[:, None]
+    qw = np.array(g["queries"][0])[None, :, None]          # [G=1][w=2][d=1]
+    score = O.accumulated_attention(qw, k, scale=1.0)
+    assert np.allclose(score, g["score"][0], atol=1e-12)
+    assert list(O.static_evict(score, 2)) == [int(x) for x in g["keep2"][0]]
+    assert list(O.static_evict(score, 1)) == [int(x) for x in g["keep1"][0]]
+    assert O.window_length(3, window_ppm=600_000) == 2   # ceil(1.8)
+
+
+def test_hierarchical_worked_example():
+    g = _golden("hierarchical_selection.txt")
+    keys = np.array(g["keys"][0])[:, None]
+    levels = O.cluster_pyramid(keys, 1, (2,), 0.6)
+    assert np.allclose(levels[1].rep[:, 0], g["parent_rep"][0], atol=1e-15)
+    q = np.ones((1, 1))
+    hier = O.hierarchical_select(q, levels, (2,), (250_000, 500_000))
+    assert list(hier) == [int(x) for x in g["hierarchical"][0]]
+    flat = O.hierarchical_select(q, levels[:1], (), (250_000,))
+    assert list(flat) == [int(x) for x in g["flat"][0]]
+
+
+def test_table5_ratio_semantics():
+    """Table 5: coarse x fine ratio = 0.2.  With the fine ratio read as a share
+    of the coarse level's survivors, the oracle keeps ~20% of the finest
+    clusters overall and ~fine_ratio of the candidates."""
+    rng = np.random.default_rng(5)
+    with open(os.path.join(GOLDEN, "table5_hierarchy_ratios.txt")) as f:
+        rows = [list(map(float, l.split())) for l in f if l.strip() and not l.startswith("#")]
+    assert len(rows) == 8
+    for cs, rc, fs, rf in rows:
+        assert abs(rc * rf - 0.2) < 0.01
+        f = int(cs // fs)
+        n_fine = 256
+        keys = rng.standard_normal((n_fine * int(fs), 8))
+        levels = O.cluster_pyramid(keys, int(fs), (f,), 0.6)
+        q = rng.standard_normal((1, 8))
+        keep = (round(rc * rf * 1e6), round(rc * 1e6))
+        sel = O.hierarchical_select(q, levels, (f,), keep)
+        n_cand = f * O.selected_count(len(levels[1].rep), keep[1], len(levels[1].rep))
+        # the printed fine ratio is 0.2 / coarse ratio to two digits
+        assert abs(rf - 0.2 / rc) < 0.006
+        assert abs(len(sel) / n_fine - 0.2) < 0.01
+        # both counts are ceilings: up to one parent (f candidates) and one
+        # cluster of rounding
+        assert abs(len(sel) / n_cand - 0.2 / rc) < (f + 1.0) / n_cand
+
+
+# ------------------------------------------------------------ counts -------
+
+def test_counts_and_rules():
+    assert O.window_length(512) == 103            # ceil(0.2 * 512)
+    assert O.window_length(2048) == 410
+    assert O.window_length(8192) == 1639
+    assert O.window_length(24_576) == 4916        # 24k is not "longer than 24k"
+    assert O.window_length(32_768) == 3277        # 10% above 24k tokens
+    assert O.window_length(1000) == 200           # exact integer arithmetic
+    assert O.kept_count(2048, 500_000) == 1024
+    assert O.kept_count(32_768, 250_000) == 8192
+    assert O.kept_count(5, 1) == 1
+    assert O.kept_count(7, 1_000_000) == 7
+    assert O.selected_count(512, 50_000, 128) == 26
+    assert O.selected_count(64, 250_000, 32) == 16
+    assert O.selected_count(8, 500_000, 8) == 4
+    assert O.selected_count(0, 500_000, 0) == 0
+    assert O.selected_count(10, 900_000, 3) == 3  # clamped to candidates
+    assert O.level_keep_fractions(50_000, 3) == [50_000, 250_000, 500_000]
+    assert O.level_keep_fractions(125_000, 2) == [125_000, 500_000]
+    assert O.level_keep_fractions(1_000_000, 2) == [1_000_000, 1_000_000]
+    assert O.level_keep_fractions(250_000, 1) == [250_000]
+    # sharing: first two layers lead themselves; groups of m after them
+    assert [O.leader_of(l, 2) for l in range(8)] == [0, 1, 2, 2, 4, 4, 6, 6]
+    assert [O.leader_of(l, 4) for l in range(11)] == [0, 1, 2, 2, 2, 2, 6, 6, 6, 6, 10]
+    assert len({O.leader_of(l, 2) for l in range(32)}) == 17
+    assert len({O.leader_of(l, 4) for l in range(32)}) == 10
+    assert [O.leader_of(l, 1) for l in range(4)] == [0, 1, 2, 3]
+
+
+# ---------------------------------------------------------------- P1 -------
+
+def _dense_decode(q, K, V, scale):
+    """Dense decode attention through torch's SDPA in float64."""
+    qt = torch.from_numpy(q)[None, None, None]            # [1,1,1,d]
+    kt = torch.from_numpy(K)[None, None]
+    vt = torch.from_numpy(V)[None, None]
+    return torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, scale=scale)[0, 0, 0].numpy()
+
+
+@pytest.mark.parametrize("G", [1, 2])
+def test_p1_keep_all_equals_dense(G):
+    rng = np.random.default_rng(11 + G)
+    Hkv, d, T, E, s = 2, 16, 37, 5, 4
+    Hq = Hkv * G
+    K = rng.standard_normal((Hkv, T, d)); V = rng.standard_normal((Hkv, T, d))
+    R = T
+    Qw = rng.standard_normal((Hq, R, d))
+    q = rng.standard_normal((E, Hq, d)); kn = rng.standard_normal((E, Hkv, d))
+    vn = rng.standard_normal((E, Hkv, d))
+    p = O.Params(keep_ppm=O.PPM, cluster_size=s, fanouts=(2,), level_keep_ppm=(O.PPM, O.PPM),
+                 share_every=1)
+    res = O.run(lambda l, b: K, lambda l, b: V, lambda l, b: Qw, lambda e, l, b: q[e],
+                lambda e, l, b: kn[e], lambda e, l, b: vn[e], [T], p, steps=E, layers=[0])
+    scale = 1 / math.sqrt(d)
+    for e in range(E):
+        for h in range(Hkv):
+            Kf = np.vstack([K[h], kn[:e + 1, h]])
+            Vf = np.vstack([V[h], vn[:e + 1, h]])
+            for g in range(G):
+                want = _dense_decode(q[e, h * G + g], Kf, Vf, scale)
+                assert np.abs(res.out[(e, 0, 0)][h * G + g] - want).max() < 1e-12
+
+
+# ---------------------------------------------------------------- P2 -------
+
+@pytest.mark.parametrize("T,w,G", [(50, 10, 1), (130, 26, 4), (9, 9, 2)])
+def test_p2_window_mass(T, w, G):
+    rng = np.random.default_rng(T)
+    d = 8
+    qw = rng.standard_normal((G, w, d)) * 2
+    k = rng.standard_normal((T, d)) * 2
+    score = O.accumulated_attention(qw, k, 1 / math.sqrt(d))
+    assert abs(score.sum() - w * G) < 1e-9 * w * G
+    assert (score >= 0).all()
+    # a key after every window row's position is never attended: only the
+    # last row sees key T-1, only rows >= i see key T-w+i
+    assert score[T - 1] <= G + 1e-12
+
+
+def test_p2_causal_mask_brute_force():
+    """Each window row's softmax, taken over exactly the causal prefix by a
+    per-row python loop, summed per column."""
+    rng = np.random.default_rng(3)
+    T, w, d = 12, 5, 4
+    qw = rng.standard_normal((1, w, d)); k = rng.standard_normal((T, d))
+    want = np.zeros(T)
+    for i in range(w):
+        pos = T - w + i
+        logits = [float(np.dot(qw[0, i], k[j])) / 2.0 for j in range(pos + 1)]
+        mx = max(logits)
+        ex = [math.exp(x - mx) for x in logits]
+        z = sum(ex)
+        for j in range(pos + 1):
+            want[j] += ex[j] / z
+    assert np.allclose(O.accumulated_attention(qw, k, 0.5), want, atol=1e-13)
+
+
+# ---------------------------------------------------------------- P3 -------
+
+@pytest.mark.parametrize("N,s,fan", [(64, 16, (4,)), (70, 16, (4,)), (200, 4, (3, 2)), (15, 16, (4,)),
+                                     (512, 16, (8, 8))])
+def test_p3_partition(N, s, fan):
+    rng = np.random.default_rng(N)
+    keys = rng.standard_normal((N, 6))
+    levels = O.cluster_pyramid(keys, s, fan, 0.6)
+    n_full = N // s
+    covered = np.arange(n_full * s)
+    for lvl, lev in enumerate(levels):
+        allm = np.concatenate(lev.members) if lev.members else np.zeros(0, int)
+        assert np.array_equal(np.sort(allm), covered)          # disjoint + covering
+        if lvl == 0:
+            assert all(len(m) == s for m in lev.members)
+        if lvl > 0:
+            f = fan[lvl - 1]
+            assert len(lev.members) == -(-len(levels[lvl - 1].members) // f)
+        for c, m in enumerate(lev.members):
+            assert np.array_equal(lev.r_max[c], keys[m].max(0))
+            assert np.array_equal(lev.r_min[c], keys[m].min(0))
+        # coarse summaries equal the element-wise max/min of their children
+        if lvl > 0:
+            f = fan[lvl - 1]
+            ch = levels[lvl - 1]
+            for p in range(len(lev.members)):
+                kids = range(p * f, min((p + 1) * f, len(ch.members)))
+                assert np.array_equal(lev.r_max[p], np.max([ch.r_max[c] for c in kids], 0))
+                assert np.array_equal(lev.r_min[p], np.min([ch.r_min[c] for c in kids], 0))
+    # attended set = selected clusters + tail, disjoint
+    sel = np.array([0, 2]) if n_full >= 3 else np.arange(n_full)
+    toks = O.attended_tokens(N, s, sel)
+    assert len(set(toks.tolist())) == len(toks)
+    assert toks.max() == N   # the token appended at this step
+
+
+# ---------------------------------------------------------------- P4 -------
+
+@pytest.mark.parametrize("G,k_ppm", [(1, 250_000), (4, 100_000), (2, 1_000_000)])
+def test_p4_token_wise_equals_topk(G, k_ppm):
+    """s = 1 (one token per cluster, no hierarchy): rep = k, so selection is
+    the exact token top-k of (sum_g q_g) . k, computed here by torch.topk."""
+    rng = np.random.default_rng(G)
+    N, d = 97, 16
+    keys = rng.standard_normal((N, d))
+    qg = rng.standard_normal((G, d))
+    levels = O.cluster_pyramid(keys, 1, (), 0.6)
+    assert np.allclose(levels[0].rep, keys, rtol=1e-15, atol=0)   # 0.6 k + 0.4 k
+    sel = O.hierarchical_select(qg, levels, (), (k_ppm,))
+    k = O.selected_count(N, k_ppm, N)
+    scores = torch.from_numpy(keys) @ torch.from_numpy(qg).sum(0)
+    want = np.sort(torch.topk(scores, k).indices.numpy())
+    assert np.array_equal(sel, want)
+
+
+# ---------------------------------------------------------------- P5 / P6 --
+
+def test_p5_identical_tokens():
+    rng = np.random.default_rng(5)
+    key = rng.standard_normal(32)
+    keys = np.tile(key, (16, 1))
+    q = rng.standard_normal(32)
+    lev = O.cluster_pyramid(keys, 16, (), 0.6)[0]
+    assert np.array_equal(lev.r_max[0], lev.r_min[0])
+    assert abs(float(lev.rep[0] @ q) - float(key @ q)) < 1e-12
+    assert abs(O.sim_bound(q, lev.r_max[0], lev.r_min[0]) - O.sim_max_dot(q, keys)) < 1e-12
+
+
+def test_p6_bound_and_linearisation():
+    rng = np.random.default_rng(6)
+    for _ in range(200):
+        s, d = rng.integers(1, 20), rng.integers(1, 40)
+        keys = rng.standard_normal((s, d)) * rng.uniform(0.1, 5)
+        q = rng.standard_normal(d)
+        lev = O.cluster_pyramid(keys, s, (), 0.6)[0]
+        rmax, rmin = lev.r_max[0], lev.r_min[0]
+        bound = O.sim_bound(q, rmax, rmin)
+        assert bound >= O.sim_max_dot(q, keys) - 1e-9          # Eq. 1 <= Eq. 2
+        # Eq. 3 reordering: linearised sum == q . rep
+        for a in (0.0, 0.3, 0.6, 1.0):
+            rep = a * rmax + (1 - a) * rmin
+            assert abs(O.sim_linear(q, rmax, rmin, a) - float(q @ rep)) < 1e-9
+        # alpha = 1 with q >= 0 reaches the bound exactly
+        qp = np.abs(q)
+        assert abs(O.sim_linear(qp, rmax, rmin, 1.0) - O.sim_bound(qp, rmax, rmin)) < 1e-9
+        # the linearised value never exceeds the bound
+        assert O.sim_linear(q, rmax, rmin, 0.6) <= bound + 1e-9
+
+
+# ---------------------------------------------------------------- P7 -------
+
+def _brute_select(qsum, keys, s, fanouts, level_keep):
+    """Coarse-to-fine selection by exhaustive search: at every level, try every
+    subset of the candidates of the required size and keep the one with the
+    largest total similarity (ties: the lexicographically smallest id list).
+    Summaries are recomputed from the member tokens with explicit loops."""
+    N, d = keys.shape
+    n_full = N // s
+    sizes = [s]
+    for f in fanouts:
+        sizes.append(sizes[-1] * f)
+
+    def members(lvl, c):
+        lo = c * sizes[lvl]
+        return list(range(lo, min(lo + sizes[lvl], n_full * s)))
+
+    def sim(lvl, c):
+        toks = members(lvl, c)
+        total = 0.0
+        for i in range(d):
+            mx = max(keys[t][i] for t in toks)
+            mn = min(keys[t][i] for t in toks)
+            total += qsum[i] * (0.6 * mx + 0.4 * mn)
+        return total
+
+    n_level = [n_full]
+    for f in fanouts:
+        n_level.append(-(-n_level[-1] // f))
+    cand = list(range(n_level[-1]))
+    chosen = []
+    for lvl in range(len(sizes) - 1, -1, -1):
+        k = O.selected_count(n_level[lvl], level_keep[lvl], len(cand))
+        best, best_val = None, None
+        for sub in itertools.combinations(cand, k):
+            val = sum(sim(lvl, c) for c in sub)
+            if best is None or val > best_val + 1e-12:
+                best, best_val = list(sub), val
+        chosen = best
+        if lvl > 0:
+            f = fanouts[lvl - 1]
+            cand = [c for p in chosen for c in range(p * f, min((p + 1) * f, n_level[lvl - 1]))]
+    return chosen
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_p7_brute_force_tiny(seed):
+    rng = np.random.default_rng(100 + seed)
+    s = int(rng.choice([2, 4]))
+    fan = [(), (2,), (3,), (2, 2)][seed % 4]
+    N = int(rng.integers(s * 3, 64))
+    d, G = 5, int(rng.choice([1, 3]))
+    keys = rng.standard_normal((N, d))
+    qg = rng.standard_normal((G, d))
+    keep = O.level_keep_fractions(int(rng.choice([250_000, 400_000])), 1 + len(fan))
+    levels = O.cluster_pyramid(keys, s, fan, 0.6)
+    got = O.hierarchical_select(qg, levels, fan, keep)
+    want = _brute_select(qg.sum(0), keys, s, fan, keep)
+    assert list(got) == sorted(want)
+
+
+# ---------------------------------------------------------------- P8 -------
+
+def test_p8_coarse_keep_all_equals_flat():
+    rng = np.random.default_rng(8)
+    keys = rng.standard_normal((16 * 40, 12))
+    qg = rng.standard_normal((2, 12))
+    flat = O.hierarchical_select(qg, O.cluster_pyramid(keys, 16, (), 0.6), (), (150_000,))
+    for fan in ((4,), (3, 2), (8,)):
+        lev = O.cluster_pyramid(keys, 16, fan, 0.6)
+        keep = [150_000] + [O.PPM] * len(fan)
+        assert np.array_equal(O.hierarchical_select(qg, lev, fan, keep), flat)
+
+
+# ---------------------------------------------------------------- P9 -------
+
+def _tiny_run(L, m, E=3, G=1, T=40, s=4, seed=9):
+    rng = np.random.default_rng(seed)
+    Hkv, d = 2, 8
+    Hq = Hkv * G
+    K = rng.standard_normal((L, Hkv, T, d)); V = rng.standard_normal((L, Hkv, T, d))
+    Qw = rng.standard_normal((L, Hq, T, d))
+    q = rng.standard_normal((E, L, Hq, d)); kn = rng.standard_normal((E, L, Hkv, d))
+    vn = rng.standard_normal((E, L, Hkv, d))
+    p = O.Params(keep_ppm=500_000, cluster_size=s, fanouts=(2,), level_keep_ppm=(250_000, 500_000),
+                 share_every=m)
+    return O.run(lambda l, b: K[l], lambda l, b: V[l], lambda l, b: Qw[l],
+                 lambda e, l, b: q[e, l], lambda e, l, b: kn[e, l], lambda e, l, b: vn[e, l],
+                 [T], p, steps=E, layers=list(range(L)))
+
+
+def test_p9_sharing():
+    L = 7
+    solo = _tiny_run(L, 1)
+    for l in range(L):
+        assert (0, l, 0, 0) in solo.selected
+    shared = _tiny_run(L, 2)
+    for e in range(3):
+        for l in range(L):
+            lead = O.leader_of(l, 2)
+            for h in range(2):
+                assert np.array_equal(shared.selected[(e, l, 0, h)], shared.selected[(e, lead, 0, h)])
+                assert np.array_equal(shared.kept[(l, 0, h)], shared.kept[(lead, 0, h)])
+    # leaders are computed from their own inputs: same as the unshared run
+    for l in (0, 1, 2, 4, 6):
+        for h in range(2):
+            assert np.array_equal(shared.selected[(0, l, 0, h)], solo.selected[(0, l, 0, h)])
+
+
+# ---------------------------------------------------------------- P10 ------
+
+@pytest.mark.slow
+def test_p10_needles_survive_c5_shape():
+    """The 32k-token needle workload at full size (layer 0, two kv heads,
+    8 decode steps): every planted needle token is kept by static eviction and
+    attended at every decode step (inside a selected cluster or the tail).
+    At reduced lengths the coarsest level has too few nodes for a passage that
+    straddles two of them, so the check needs the real shape."""
+    from paper_2501_06807_gb300 import synth
+    w = synth.C5.replace(n_layers=1, decode_steps=8)
+    T = w.prompt_len
+    R = O.window_length(T)
+    x = synth.generate(w, R)
+    G, s = w.group, w.cluster_size
+    d = w.head_dim
+    for h in (0, 5):
+        K = x.k[0, 0, h, :T].double().numpy()
+        qw = x.q_win[0, 0, h * G:(h + 1) * G, R - R:].double().numpy()
+        score = O.accumulated_attention(qw, K, 1 / math.sqrt(d))
+        kept = O.static_evict(score, O.kept_count(T, w.keep_ppm))
+        start = int(x.needle_pos[0, 0, h])
+        needles = list(range(start, start + w.needle_len))
+        assert set(needles) <= set(kept.tolist())
+        cache = K[kept]
+        cache_idx = [int(np.searchsorted(kept, t)) for t in needles]
+        for e in range(8):
+            n_tok = len(kept) + e
+            levels = O.cluster_pyramid(cache[:n_tok], s, w.fanouts, w.alpha)
+            sel = O.hierarchical_select(x.q[e, 0, 0, h * G:(h + 1) * G].double().numpy(),
+                                        levels, w.fanouts, w.level_keep_ppm)
+            att = set(O.attended_tokens(n_tok, s, sel).tolist())
+            assert set(cache_idx) <= att
+            cache = np.vstack([cache, x.k_new[e, 0, 0, h].double().numpy()[None]])
+
+
+# ---------------------------------------------------------------- P11 ------
+
+def test_p11_commonality():
+    idx = [[3, 1, 2], [3, 1, 2], [3, 1, 2], [3, 1, 2]]
+    assert O.commonality(idx, 3, 1) == 1.0
+    assert O.commonality(idx, 3, 3) == 1.0
+    # hand-worked: layers {0,1,2}, {1,2,3}, {2,3,4}; k = 3, m = 1
+    # |L0 & L1| = 2, |L1 & L2| = 2 -> (2 + 2) / (3 * 2)
+    assert abs(O.commonality([[0, 1, 2], [1, 2, 3], [2, 3, 4]], 3, 1) - 4 / 6) < 1e-15
+    run = _tiny_run(6, 2, E=1)
+    sel = [list(run.selected[(0, l, 0, 0)]) for l in range(2, 6)]
+    k = len(sel[0])
+    assert O.commonality([sel[0], sel[1]], k, 1) == 1.0      # layers 2, 3 share
