@@ -1,0 +1,410 @@
+#!/usr/bin/env python3
+"""Benchmark of the MPCache decode path on one GB300 (or N replicas).
+
+One step = the whole method over one batch of synthetic input: look-once
+static eviction of the leader layers, gathering + clustering of every
+layer, then all E decode steps (selection for the leaders, append + sparse
+attention for every layer).  The metric is selected-KV tokens per second:
+the rows every decode step attends (selected clusters plus tail, summed over
+layers, sequences and kv heads) divided by the whole step's time.
+
+Prints one JSON line on rank 0.  ``--impl reference`` times the fp64 CPU
+oracle on a bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2501_06807_gb300 import synth  # noqa: E402
+
+METRIC = "selected-KV tokens/s"
+UNIT = "tokens/s"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# fp32 FFMA peak of a GB300 at its maximum SM clock: 152 SMs x 128 lanes x 2 flops
+FFMA_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=5)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default=synth.C5.name, choices=sorted(synth.WORKLOADS))
+    p.add_argument("--decode-steps", type=int, default=None)
+    p.add_argument("--no-e2e", action="store_true")
+    return p.parse_args()
+
+
+def peaks():
+    try:
+        with open(PEAKS_FILE) as f:
+            d = json.load(f)
+        return d, "measured"
+    except Exception:
+        return FALLBACK, "fallback"
+
+
+# ------------------------------------------------------------ workload ----
+
+def rules(w):
+    from paper_2501_06807_gb300 import mpcache
+    R = mpcache.window_rows_bound(w.prompt_len, w.window_ppm, w.long_window_ppm, w.long_prompt_threshold)
+    leaders = sorted({mpcache.sharing_leader(l, w.share_every) for l in range(w.n_layers)})
+    return R, leaders
+
+
+def static_flops(w, lens, n_leaders):
+    """Algorithmic FLOPs of the two score passes: every (window row, causal
+    key) pair of every leader layer and query head, 2 d flops per pass."""
+    from paper_2501_06807_gb300 import mpcache
+    total = 0
+    for T in lens:
+        wl = mpcache.ppm_count(T, w.long_window_ppm if T > w.long_prompt_threshold else w.window_ppm)
+        pairs = wl * (T - wl) + wl * (wl + 1) // 2
+        total += pairs
+    return 2 * 2 * w.head_dim * total * w.n_q_heads * n_leaders
+
+
+# ------------------------------------------------------------- clocks ----
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out = ""
+        rows = [r.split(",") for r in out.strip().splitlines() if r.strip()]
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[0]))
+                mx.append(float(r[1]))
+            except (ValueError, IndexError):
+                continue
+            for n, v in zip(names, r[4:8]):
+                if v.strip().lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------ our arm ----
+
+def run_ours(args, rank, world, dist):
+    from paper_2501_06807_gb300 import build, mpcache
+    build.build()
+    mpcache.load()
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    w = synth.WORKLOADS[args.workload]
+    if world > 1:
+        w = w.replace(seed=w.seed + 7919 * rank)  # independent replica per rank
+    E = args.decode_steps or w.decode_steps
+    R, leaders = rules(w)
+    x = synth.generate(w, R, device="cuda", decode_steps=E)
+    lens = x.prompt_lens.cuda()
+    pt = x.page_table.cuda() if x.page_table is not None else None
+    dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    eng = mpcache.Engine(n_layers=w.n_layers, batch=w.batch, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads,
+                         head_dim=w.head_dim, dtype=dt, t_max=w.prompt_len, keep_ppm=w.keep_ppm,
+                         cluster_size=w.cluster_size, fanouts=w.fanouts, level_keep_ppm=w.level_keep_ppm,
+                         share_every=w.share_every, max_decode_steps=E, alpha=w.alpha,
+                         window_ppm=w.window_ppm, long_window_ppm=w.long_window_ppm,
+                         long_prompt_threshold=w.long_prompt_threshold)
+    out_all = torch.empty((E, w.n_layers, w.batch, w.n_q_heads, w.head_dim), dtype=torch.float32, device=dev)
+
+    def prefill():
+        eng.prefill(x.k, x.v, x.q_win, lens, pt, w.page_size)
+
+    def decode_all():
+        for e in range(E):
+            eng.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=out_all[e])
+
+    # eager pass: counts the attended rows of every step, checks the status
+    prefill()
+    attended = 0
+    n_keep = eng.n_keep.cpu().tolist()
+    s = w.cluster_size
+    for e in range(E):
+        eng.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=out_all[e])
+        n_sel = eng.n_sel.cpu().tolist()
+        for b in range(w.batch):
+            n_tok = n_keep[b] + e
+            attended += (n_sel[b] * s + n_tok % s + 1) * w.n_layers * w.n_kv_heads
+    status = mpcache.device_status()
+    if status != 0:
+        raise RuntimeError(f"device status {status} after the eager pass")
+
+    graph = torch.cuda.CUDAGraph()
+    prefill()
+    torch.cuda.synchronize()
+    with torch.cuda.graph(graph):
+        decode_all()
+    torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        prefill()
+        graph.replay()
+    torch.cuda.synchronize()
+
+    stream = torch.cuda.current_stream()
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    marks = [(ev(), ev(), ev(), ev()) for _ in range(args.steps)]
+    clocks = ClockSampler(dev.index)
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t_start, t_end = ev(), ev()
+    t_start.record(stream)
+    for m in marks:
+        m[0].record(stream)
+        eng.static_evict(x.k, x.q_win, lens, pt, w.page_size)
+        m[1].record(stream)
+        eng.build_clusters(x.k, x.v, pt, w.page_size)
+        m[2].record(stream)
+        graph.replay()
+        m[3].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    if dist is not None:
+        dist.barrier()
+    total_ms = t_start.elapsed_time(t_end)
+    static_ms = sum(m[0].elapsed_time(m[1]) for m in marks) / args.steps
+    build_ms = sum(m[1].elapsed_time(m[2]) for m in marks) / args.steps
+    decode_ms = sum(m[2].elapsed_time(m[3]) for m in marks) / args.steps
+    if dist is not None:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = attended * world / (ms_per_step / 1e3)
+
+    # e2e through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        host = {n: getattr(x, n).cpu().pin_memory() for n in ("k", "v", "q_win", "q", "k_new", "v_new")}
+        host_lens = x.prompt_lens.pin_memory()
+        out_host = torch.empty(out_all.shape, dtype=out_all.dtype).pin_memory()
+        h2d = sum(t.numel() * t.element_size() for t in host.values()) + host_lens.numel() * 4
+        d2h = out_host.numel() * out_host.element_size()
+
+        def e2e_step():
+            for n, t in host.items():
+                getattr(x, n).copy_(t, non_blocking=True)
+            lens.copy_(host_lens, non_blocking=True)
+            prefill()
+            graph.replay()
+            out_host.copy_(out_all, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize()
+        a, b = ev(), ev()
+        if dist is not None:
+            dist.barrier()
+        a.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = a.elapsed_time(b) / args.steps
+        if dist is not None:
+            t = torch.tensor([e2e_ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_ms = float(t.item())
+        e2e = {"value": attended * world / (e2e_ms / 1e3), "unit": UNIT, "ms_per_step": e2e_ms,
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+
+    pk, pk_kind = peaks()
+    n_lead = len(leaders)
+    flops = static_flops(w, [int(t) for t in x.prompt_lens], n_lead)
+    static_tflops = flops / (static_ms / 1e3) / 1e12
+    esz = 2 if w.dtype == "bf16" else 4
+    # decode bytes: attended K and V rows, the leaders' summaries read by the
+    # selection (upper bound: every level's candidates), q, k_new, v_new, o
+    kv_bytes = attended * w.head_dim * 2 * esz
+    io_bytes = E * w.n_layers * w.batch * (w.n_q_heads * w.head_dim * (esz + 4) + 2 * w.n_kv_heads * w.head_dim * esz)
+    dec_bytes = kv_bytes + io_bytes
+    decode_gbs = dec_bytes / (decode_ms / 1e3) / 1e9
+    dominant_static = static_ms >= decode_ms
+    if dominant_static:
+        roof = {"kernel": "mpc_static_evict (rowstats + colsum + budget)", "bound": "alu",
+                "achieved": round(static_tflops, 3), "peak": round(FFMA_PEAK_TFLOPS, 1), "unit": "TFLOP/s",
+                "frac": round(static_tflops / FFMA_PEAK_TFLOPS, 4), "traffic": None,
+                "peak_source": "fp32 FFMA: 152 SMs x 128 lanes x 2 flops x 2.07 GHz"}
+    else:
+        roof = {"kernel": "decode step (mpc_select + mpc_sparse_decode_attn)", "bound": "hbm",
+                "achieved": round(decode_gbs, 1), "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": round(decode_gbs / pk["hbm_gbs"], 4), "traffic": None, "peak_source": pk_kind}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": w.dtype, "data": "synthetic (seeded generator, workload recipe in DESIGN.md)",
+        "config": {"workload": w.name, "layers": w.n_layers, "batch": w.batch, "q_heads": w.n_q_heads,
+                   "kv_heads": w.n_kv_heads, "head_dim": w.head_dim, "prompt_len": w.prompt_len,
+                   "decode_steps": E, "cluster_size": w.cluster_size, "fanouts": list(w.fanouts),
+                   "level_keep_ppm": list(w.level_keep_ppm), "keep_ppm": w.keep_ppm,
+                   "share_every": w.share_every, "parallelism": f"replicas{world}",
+                   "l2": "inputs larger than L2 (prompt KV %.1f GB per step)" % (
+                       (x.k.numel() + x.v.numel()) * x.k.element_size() / 1e9)},
+        "gpu_launches": args.steps * (3 + 1 + (1 if len(w.fanouts) else 0) + 2 * E),
+        "phases_ms": {"static_evict": static_ms, "build_clusters": build_ms, "decode_all_steps": decode_ms},
+        "decode_step_us": decode_ms / E * 1e3,
+        "decode": {"bytes_per_step": dec_bytes / E, "achieved_gbs": round(decode_gbs, 1),
+                   "frac_of_measured_hbm": round(decode_gbs / pk["hbm_gbs"], 4),
+                   "frac_of_8tbs": round(decode_gbs / 8000.0, 4)},
+        "static_scoring_tflops": round(static_tflops, 3),
+        "roofline": roof,
+        "clocks": clk,
+        "e2e": e2e,
+    }
+    return line
+
+
+# ------------------------------------------------------ oracle sample ----
+
+def oracle_sample(w, E_sample=4):
+    """Times the fp64 oracle on one (leader layer, sequence 0, kv head 0) unit
+    of the workload: static scoring, eviction, clustering and E_sample decode
+    steps (selection + attention), and extrapolates to the whole job."""
+    from oracle import mpcache_oracle as O
+    from paper_2501_06807_gb300 import mpcache
+    R, leaders = rules(w)
+    ws = w.replace(n_layers=1, batch=1)
+    x = synth.generate(ws, R, decode_steps=E_sample)
+    T = int(x.prompt_lens[0])
+    G, d, s = w.group, w.head_dim, w.cluster_size
+    K = x.k[0, 0, 0, :T].double().numpy()
+    V = x.v[0, 0, 0, :T].double().numpy()
+    wl = O.window_length(T, w.window_ppm, w.long_window_ppm, w.long_prompt_threshold)
+    qw = x.q_win[0, 0, :G, R - wl:].double().numpy()
+    t0 = time.perf_counter()
+    score = O.accumulated_attention(qw, K, 1 / math.sqrt(d))
+    kept = O.static_evict(score, O.kept_count(T, w.keep_ppm))
+    t1 = time.perf_counter()
+    ck, cv = K[kept], V[kept]
+    t_dec = 0.0
+    t_build = 0.0
+    for e in range(E_sample):
+        n_tok = len(ck)
+        tb = time.perf_counter()
+        levels = O.cluster_pyramid(ck, s, w.fanouts, w.alpha)
+        t_build += time.perf_counter() - tb
+        td = time.perf_counter()
+        qg = x.q[e, 0, 0, :G].double().numpy()
+        sel = O.hierarchical_select(qg, levels, w.fanouts, w.level_keep_ppm)
+        ck = np.vstack([ck, x.k_new[e, 0, 0, 0].double().numpy()[None]])
+        cv = np.vstack([cv, x.v_new[e, 0, 0, 0].double().numpy()[None]])
+        toks = O.attended_tokens(n_tok, s, sel)
+        for g in range(G):
+            O.sparse_attention(qg[g], ck[toks], cv[toks], 1 / math.sqrt(d))
+        t_dec += time.perf_counter() - td
+    t_static = t1 - t0
+    E = w.decode_steps
+    units = w.batch * w.n_kv_heads
+    whole = (t_static * len(leaders) * units + (t_build / E_sample) * len(leaders) * units
+             + (t_dec / E_sample) * E * w.n_layers * units)
+    n_keep = len(kept)
+    k1_of = {}
+
+    def k1(n_tok):
+        c1 = n_tok // s
+        if c1 not in k1_of:
+            zero = O.cluster_pyramid(np.zeros((c1 * s, 1)), s, w.fanouts, w.alpha)
+            k1_of[c1] = len(O.hierarchical_select(np.zeros((1, 1)), zero, w.fanouts, w.level_keep_ppm))
+        return k1_of[c1]
+
+    tokens = sum(k1(n_keep + e) * s + (n_keep + e) % s + 1 for e in range(E)) * w.n_layers * units
+    sample = (f"1 of {len(leaders) * units} leader units static-scored at full T={T} "
+              f"({t_static:.1f} s), {E_sample} decode steps of 1 unit; extrapolated to "
+              f"{len(leaders)} leaders x {units} (b, kv head) units and {E} steps x {w.n_layers} layers")
+    return {"value": tokens / whole, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+            "sample": sample, "seconds": t1 - t0 + t_build + t_dec, "whole_job_s_estimate": whole}
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return None
+    w = synth.WORKLOADS[args.workload]
+    for _ in range(args.warmup):
+        oracle_sample(w, E_sample=1)
+    vals, secs = [], []
+    for _ in range(args.steps):
+        r = oracle_sample(w, E_sample=2)
+        vals.append(r["value"])
+        secs.append(r["whole_job_s_estimate"])
+    v = statistics.median(vals)
+    return {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": statistics.median(secs) * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": w.name, "parallelism": "cpu"},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": r["sample"]},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = parse_args()
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    dist = None
+    if world > 1:
+        import torch.distributed as tdist
+        backend = "nccl" if torch.cuda.is_available() and args.impl == "ours" else "gloo"
+        if args.impl == "ours":
+            torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", 0)))
+        tdist.init_process_group(backend)
+        dist = tdist
+    if args.impl == "reference":
+        line = run_reference(args, rank, world)
+    else:
+        line = run_ours(args, rank, world, dist)
+        if rank == 0 and world == 1:
+            line["cpu_baseline"] = oracle_sample(synth.WORKLOADS[args.workload])
+    if rank == 0 and line is not None:
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

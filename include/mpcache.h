@@ -1,0 +1,285 @@
+/*
+ * mpcache.h - C ABI of the GB300 (sm_103a) MPCache decode path.
+ *
+ * MPCache (arXiv 2501.06807) shrinks the attention of LLM decoding in four
+ * steps; each step is one call of this library:
+ *
+ *   mpc_static_evict        look-once static eviction at prefill (Sec. 3.2,
+ *                           Alg. 2 Step 1)
+ *   mpc_build_clusters      token gathering of the kept set into a
+ *                           cluster-major cache plus the hierarchical cluster
+ *                           summaries r_max, r_min and the reordered
+ *                           representative of Eq. 3 (Sec. 3.3)
+ *   mpc_select              per decode step: MPC-friendly similarity (Eq. 3)
+ *                           and hierarchical top-k over the clusters, for the
+ *                           leader layer of a cross-layer sharing group
+ *                           (Sec. 3.3-3.4, Alg. 2 Step 2)
+ *   mpc_sparse_decode_attn  per decode step: append the new k, v, then
+ *                           softmax(q K'^T / sqrt(d)) V' over the selected
+ *                           clusters and the tail (Alg. 1 line 4)
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * - Pointers named "device" are CUDA device pointers owned by the caller; the
+ *   library never allocates, frees or retains them past the call.  Scratch
+ *   space is the caller's too: `*_workspace_size` reports how many bytes a
+ *   call needs and the call receives them as `workspace`.  A workspace must
+ *   be zero-filled once before its first use; calls leave it zero-filled.
+ * - Every call is asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *   default stream) and returns once its kernels are queued.  Arguments are
+ *   validated on the host before anything is launched.
+ * - Tensors are row-major with the head dimension d innermost.  `dtype` is
+ *   MPC_F32 or MPC_BF16 and applies to queries, keys, values and the
+ *   cluster-major cache; summaries, scores and outputs are float32.
+ * - One call may process several layers.  `refs[i]` names, for the i-th
+ *   processed layer, its index along every per-layer tensor of the call
+ *   (`layer`, scaled by that tensor's layer stride), its index along every
+ *   per-group tensor (`group`: kept sets, summaries, selections) and whether
+ *   it leads the group (`leader`, Sec. 3.4: the leader computes the shared
+ *   indices, the other layers of the group reuse them).
+ * - Ratios are integers in parts per million.  A count derived from a ratio
+ *   r over N items is min(N, max(1, ceil(N r / 1e6))), 0 when N = 0.
+ * - Return value: MPC_OK, or a negative MPC_ERR_* code; mpc_last_error()
+ *   gives a thread-local message for the last failing call of the thread.
+ *
+ * Cluster-major cache (output of mpc_build_clusters, read and appended to
+ * by mpc_sparse_decode_attn): per (layer, sequence, kv head) `cap_tokens`
+ * rows of d elements.  Row i is the i-th kept token in position order,
+ * followed by the tokens appended by decode steps.  Cluster c (finest level)
+ * is rows [c s, (c + 1) s); the rows after the last full cluster form the
+ * tail.  Inside a row the 16-byte chunks are permuted: logical chunk j of
+ * row i is stored at chunk j ^ (i & 7).  The permutation keeps the
+ * decode kernel's shared-memory reads free of bank conflicts.
+ *
+ * Summary pyramid (per group, sequence, kv head): `summary_rows` rows of d
+ * float32.  Level 1 (clusters of s tokens) starts at row 0 and has
+ * cap_1 = cap_tokens / s rows; level l + 1 starts after level l and has
+ * cap_{l+1} = ceil(cap_l / fanout[l]) rows.  Three such arrays hold r_max,
+ * r_min and rep = alpha r_max + (1 - alpha) r_min.
+ */
+#ifndef MPCACHE_H
+#define MPCACHE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define MPC_API __attribute__((visibility("default")))
+
+#define MPC_ABI_VERSION 1
+#define MPC_MAX_LEVELS 4
+#define MPC_MAX_REFS 128
+
+enum mpc_status {
+  MPC_OK = 0,
+  MPC_ERR_INVALID_ARG = -1,   /* NULL pointer, bad enum, struct_size mismatch */
+  MPC_ERR_BAD_SHAPE = -2,     /* a size or ratio outside the supported range */
+  MPC_ERR_WORKSPACE = -3,     /* workspace NULL or smaller than reported */
+  MPC_ERR_CUDA = -4           /* a CUDA launch or attribute call failed */
+};
+
+enum mpc_dtype { MPC_F32 = 0, MPC_BF16 = 1 };
+
+typedef struct {
+  int32_t layer;   /* index along per-layer tensors */
+  int32_t group;   /* index along per-group tensors */
+  int32_t leader;  /* nonzero if this layer computes the group's indices */
+} mpc_layer_ref;
+
+/* Prompt K or V of the processed layers, dense or paged.  Element
+ * (layer l, sequence b, kv head h, position t, channel c) lives at
+ *   dense: data + l*layer_stride + ((b*n_kv_heads + h)*t_max + t)*d + c
+ *   paged: data + l*layer_stride
+ *               + ((page_table[b*max_pages + t/page_size]*n_kv_heads + h)
+ *                  *page_size + t%page_size)*d + c
+ * (offsets in elements of the call's dtype). */
+typedef struct {
+  const void* data;            /* device */
+  int64_t layer_stride;        /* elements between consecutive layers */
+  const int32_t* page_table;   /* device [batch][max_pages], NULL = dense */
+  int32_t page_size;           /* tokens per page (paged only) */
+  int32_t max_pages;           /* page-table row length (paged only) */
+} mpc_kv_tensor;
+
+/* ---- mpc_static_evict ----------------------------------------------------
+ * Look-once static eviction (Sec. 3.2; Alg. 2 Step 1; App. E "Static
+ * eviction").  For every leader ref, sequence b and kv head h:
+ *   w_b     = ceil(T_b * rho_w), rho_w = long_window_ppm if T_b >
+ *             long_prompt_threshold else window_ppm (20% / 10% above 24k)
+ *   score_j = sum over the group's query heads g and window rows i of
+ *             softmax_{j' <= p_i}(q_{g,i} . k_{j'} * scale)_j,
+ *             p_i = T_b - w_b + i (causal attention map of the last rows)
+ *   kept    = the n_keep_b = count(T_b, keep_ppm) positions of highest score
+ *             (equal scores: lower position first), in ascending order.
+ * Outputs: out_scores[group][b][h][t_max] (positions >= T_b undefined),
+ * out_kept[group][b][h][keep_cap] (entries >= n_keep_b are -1) and
+ * out_n_keep[b].  Refs must all be leaders. */
+typedef struct {
+  uint32_t struct_size;        /* sizeof(mpc_static_args) */
+  int32_t n_refs;
+  const mpc_layer_ref* refs;   /* host [n_refs] */
+  int32_t batch, n_q_heads, n_kv_heads, head_dim, dtype;
+  int32_t t_max;               /* prompt capacity, >= every T_b */
+  const int32_t* prompt_lens;  /* device [batch], 1 <= T_b <= t_max */
+  const void* q_win;           /* device [layer][batch][n_q_heads][win_rows][d];
+                                  row r is prompt position T_b - win_rows + r */
+  int64_t q_win_layer_stride;  /* elements */
+  int32_t win_rows;            /* >= every w_b */
+  mpc_kv_tensor k;
+  int32_t window_ppm, long_window_ppm, long_prompt_threshold;
+  int32_t keep_ppm;
+  float scale;                 /* 0 selects 1/sqrt(d) */
+  int32_t keep_cap;            /* >= every n_keep_b */
+  float* out_scores;           /* device */
+  int32_t* out_kept;           /* device */
+  int32_t* out_n_keep;         /* device [batch] */
+} mpc_static_args;
+
+/* ---- mpc_build_clusters --------------------------------------------------
+ * Token gathering of the kept set (Alg. 2 Step 1, token_gather) into the
+ * cluster-major cache, and the summary pyramid of the leaders (Sec. 3.3:
+ * r_max / r_min of each cluster, the Eq. 3 representative; hierarchical
+ * clustering: level l + 1 groups fanout[l] consecutive level-l clusters and
+ * its r_max / r_min are taken over all member tokens).  Only the
+ * floor(n_keep_b / s) full clusters get summaries; the remaining rows are the
+ * tail.  For every ref: rows [0, n_keep_b) of its cache are written from the
+ * kept positions of its group; leaders also write their group's pyramid.
+ * out_n_tok[b] = n_keep_b starts the decode counter. */
+typedef struct {
+  uint32_t struct_size;        /* sizeof(mpc_cluster_args) */
+  int32_t n_refs;
+  const mpc_layer_ref* refs;   /* host [n_refs] */
+  int32_t batch, n_kv_heads, head_dim, dtype;
+  int32_t t_max;
+  mpc_kv_tensor k, v;          /* prompt keys and values */
+  const int32_t* kept;         /* device [group][batch][n_kv_heads][keep_cap] */
+  int32_t keep_cap;
+  const int32_t* n_keep;       /* device [batch] */
+  void* kc;                    /* device cluster-major keys [layer][batch][n_kv_heads][cap_tokens][d] */
+  void* vc;                    /* device cluster-major values, same layout */
+  int64_t cache_layer_stride;  /* elements between layers of kc / vc */
+  int32_t cap_tokens;          /* multiple of cluster_size, >= n_keep_b + decode steps */
+  float* r_max;                /* device [group][batch][n_kv_heads][summary_rows][d] */
+  float* r_min;
+  float* rep;
+  int32_t summary_rows;
+  int32_t cluster_size;        /* s */
+  int32_t n_levels;            /* 1 .. MPC_MAX_LEVELS */
+  int32_t fanout[MPC_MAX_LEVELS]; /* fanout[l] >= 2 for l < n_levels - 1 */
+  float alpha;                 /* Eq. 3 weight, default 0.6 */
+  int32_t* out_n_tok;          /* device [batch] */
+} mpc_cluster_args;
+
+/* ---- mpc_select ----------------------------------------------------------
+ * Dynamic selection of one decode step for leader layers (Sec. 3.3-3.4; Alg.
+ * 2 Step 2, Sim + topk).  With C_1 = floor(n_tok_b / s) sealed clusters and
+ * C_{l+1} = ceil(C_l / fanout[l]), for every ref, sequence b and kv head h:
+ *   sim(c) = (sum over the group's query heads of q) . rep_c      (Eq. 3)
+ *   the coarsest level ranks all of its clusters; every finer level ranks
+ *   the children of the clusters its parent level kept; level l keeps
+ *   k_l = count(C_l, level_keep_ppm[l]) (at most its candidates); equal
+ *   similarities rank the lower id first.
+ * out_sel[group][b][h][sel_cap] gets the kept finest-level ids ascending
+ * (entries >= out_n_sel[b] are -1).  n_tok is read-only here. */
+typedef struct {
+  uint32_t struct_size;        /* sizeof(mpc_select_args) */
+  int32_t n_refs;
+  const mpc_layer_ref* refs;   /* host [n_refs], all leaders */
+  int32_t batch, n_q_heads, n_kv_heads, head_dim, dtype;
+  const void* q;               /* device [layer][batch][n_q_heads][d] */
+  int64_t q_layer_stride;      /* elements */
+  const float* rep;            /* device [group][batch][n_kv_heads][summary_rows][d] */
+  int32_t summary_rows;
+  int32_t cap_tokens;
+  const int32_t* n_tok;        /* device [batch] cache rows before this step's append */
+  int32_t cluster_size, n_levels;
+  int32_t fanout[MPC_MAX_LEVELS];
+  int32_t level_keep_ppm[MPC_MAX_LEVELS]; /* finest level first */
+  int32_t sel_cap;             /* >= every k_1 */
+  int32_t* out_sel;            /* device */
+  int32_t* out_n_sel;          /* device [batch] */
+} mpc_select_args;
+
+/* ---- mpc_sparse_decode_attn ----------------------------------------------
+ * One decode step of attention for every ref (Alg. 1 line 4; Alg. 2 Step 2,
+ * gather + sparse attention; App. A decode append).  With n = n_tok_b and
+ * C_1 = floor(n / s):
+ *   1. k_new, v_new are written to row n of the layer's cache (append);
+ *   2. o_g = softmax(q_g K'^T * scale) V' over the rows of the selected
+ *      clusters of the ref's group (sel, n_sel) and the tail rows
+ *      [C_1 s, n] (which include the appended row);
+ *   3. if the tail now holds s rows it is sealed as cluster C_1: leaders
+ *      write its r_max / r_min / rep and merge it into the coarser levels;
+ *   4. if `advance` is nonzero, n_tok[b] += 1 once all refs are done.
+ * Outputs o[layer][b][n_q_heads][d] float32. */
+typedef struct {
+  uint32_t struct_size;        /* sizeof(mpc_attn_args) */
+  int32_t n_refs;
+  const mpc_layer_ref* refs;   /* host [n_refs] */
+  int32_t batch, n_q_heads, n_kv_heads, head_dim, dtype;
+  const void* q;               /* device [layer][batch][n_q_heads][d] */
+  const void* k_new;           /* device [layer][batch][n_kv_heads][d] */
+  const void* v_new;
+  int64_t q_layer_stride, kv_new_layer_stride;   /* elements */
+  void* kc;                    /* device cluster-major cache (in/out) */
+  void* vc;
+  int64_t cache_layer_stride;
+  int32_t cap_tokens;
+  const int32_t* sel;          /* device [group][batch][n_kv_heads][sel_cap] */
+  const int32_t* n_sel;        /* device [batch] */
+  int32_t sel_cap;
+  float* r_max;                /* device pyramid (in/out, leaders only); */
+  float* r_min;                /* may be NULL when no ref is a leader    */
+  float* rep;
+  int32_t summary_rows;
+  int32_t cluster_size, n_levels;
+  int32_t fanout[MPC_MAX_LEVELS];
+  float alpha;
+  int32_t* n_tok;              /* device [batch] */
+  int32_t advance;
+  float scale;                 /* 0 selects 1/sqrt(d) */
+  float* out;                  /* device [layer][batch][n_q_heads][d] */
+  int64_t out_layer_stride;    /* elements */
+} mpc_attn_args;
+
+/* Workspace byte counts (0 is a valid answer).  Same validation as the
+ * calls; the pointer fields of `args` may be NULL here. */
+MPC_API int mpc_static_evict_workspace_size(const mpc_static_args* args, size_t* bytes);
+MPC_API int mpc_build_clusters_workspace_size(const mpc_cluster_args* args, size_t* bytes);
+MPC_API int mpc_select_workspace_size(const mpc_select_args* args, size_t* bytes);
+MPC_API int mpc_sparse_decode_attn_workspace_size(const mpc_attn_args* args, size_t* bytes);
+
+MPC_API int mpc_static_evict(const mpc_static_args* args, void* workspace,
+                             size_t workspace_bytes, void* stream);
+MPC_API int mpc_build_clusters(const mpc_cluster_args* args, void* workspace,
+                               size_t workspace_bytes, void* stream);
+MPC_API int mpc_select(const mpc_select_args* args, void* workspace,
+                       size_t workspace_bytes, void* stream);
+MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace,
+                                   size_t workspace_bytes, void* stream);
+
+/* Rows of the summary pyramid for a cache of cap_tokens rows (the sum of the
+ * level capacities above), or a negative MPC_ERR_* code. */
+MPC_API int64_t mpc_summary_rows(int32_t cap_tokens, int32_t cluster_size,
+                                 int32_t n_levels, const int32_t* fanout);
+
+/* Thread-local description of the last error of this thread ("" if none). */
+MPC_API const char* mpc_last_error(void);
+
+/* Device status word of the current device: nonzero once a kernel of this
+ * library gave up a bounded wait (for a bulk copy that did not complete);
+ * such a kernel skips the rest of its work and returns.  Blocks on the
+ * device (cudaDeviceSynchronize), returns the flags and clears them. */
+MPC_API int mpc_device_status(int* flags);
+
+/* MPC_ABI_VERSION of the loaded library. */
+MPC_API int mpc_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MPCACHE_H */

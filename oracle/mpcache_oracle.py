@@ -185,14 +185,17 @@ def cluster_pyramid(keys: np.ndarray, s: int, fanouts: Sequence[int],
 
 
 def hierarchical_select(q_group: np.ndarray, levels: List[Level],
-                        fanouts: Sequence[int], level_keep_ppm: Sequence[int]) -> np.ndarray:
+                        fanouts: Sequence[int], level_keep_ppm: Sequence[int],
+                        trace: Optional[list] = None) -> np.ndarray:
     """Coarse-to-fine cluster selection (Sec. 3.3; Alg. 2 Sim + topk).
 
     q_group: [G][d] decode queries of one kv group; the similarity of cluster c
     is (sum_g q_g) . rep_c (Eq. 3 summed over the group).  At the coarsest
     level every cluster is a candidate; at each finer level the candidates are
     the children of the kept parents.  Returns the kept finest-level ids in
-    ascending order.
+    ascending order.  ``trace``, if given, receives per level (coarsest
+    first) the candidate ids, their similarities and k, for tests that need
+    the margin at each cut.
     """
     qsum = np.asarray(q_group, dtype=np.float64).sum(axis=0)
     n = len(levels)
@@ -202,6 +205,8 @@ def hierarchical_select(q_group: np.ndarray, levels: List[Level],
         lev = levels[lvl]
         sim = lev.rep[cand] @ qsum if len(cand) else np.zeros(0)
         k = selected_count(lev.rep.shape[0], level_keep_ppm[lvl], len(cand))
+        if trace is not None:
+            trace.append((np.asarray(cand), np.asarray(sim), k))
         kept = np.sort(rank_desc(sim, cand)[:k]) if k else np.zeros(0, dtype=np.int64)
         if lvl > 0:
             f = fanouts[lvl - 1]

@@ -1,0 +1,476 @@
+// C ABI of the MPCache library: argument validation (host only, before any
+// CUDA call), workspace sizing, launch planning and kernel launches.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+
+#include "kernels.cuh"
+
+namespace mpc {
+namespace {
+
+thread_local std::string g_err;
+
+int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return code;
+}
+
+int ok() {
+  g_err.clear();
+  return MPC_OK;
+}
+
+#define MPC_TRY(expr)         \
+  do {                        \
+    const int _rc = (expr);   \
+    if (_rc != MPC_OK) return _rc; \
+  } while (0)
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int esize(int dtype) { return dtype == MPC_BF16 ? 2 : 4; }
+
+int check_common(int batch, int hq, int hkv, int d, int dtype) {
+  if (dtype != MPC_F32 && dtype != MPC_BF16) return fail(MPC_ERR_INVALID_ARG, "dtype %d is not MPC_F32/MPC_BF16", dtype);
+  if (batch < 1) return fail(MPC_ERR_BAD_SHAPE, "batch %d < 1", batch);
+  if (hq < 1 || hkv < 1 || hq % hkv != 0)
+    return fail(MPC_ERR_BAD_SHAPE, "n_q_heads %d must be a positive multiple of n_kv_heads %d", hq, hkv);
+  if (d != 64 && d != 128) return fail(MPC_ERR_BAD_SHAPE, "head_dim %d not in {64, 128}", d);
+  return MPC_OK;
+}
+
+int check_refs(int n, const mpc_layer_ref* refs, bool leaders_only, RefTable* t) {
+  if (refs == nullptr) return fail(MPC_ERR_INVALID_ARG, "refs is NULL");
+  if (n < 1 || n > kMaxRefs) return fail(MPC_ERR_BAD_SHAPE, "n_refs %d not in [1, %d]", n, kMaxRefs);
+  for (int i = 0; i < n; ++i) {
+    if (refs[i].layer < 0 || refs[i].group < 0)
+      return fail(MPC_ERR_BAD_SHAPE, "refs[%d] has a negative index", i);
+    if (leaders_only && !refs[i].leader) return fail(MPC_ERR_INVALID_ARG, "refs[%d] is not a leader", i);
+    if (t) {
+      t->layer[i] = refs[i].layer;
+      t->group[i] = refs[i].group;
+      t->leader[i] = refs[i].leader ? 1 : 0;
+    }
+  }
+  return MPC_OK;
+}
+
+int check_ppm(int v, const char* name) {
+  if (v < 1 || v > 1000000) return fail(MPC_ERR_BAD_SHAPE, "%s = %d ppm not in [1, 1e6]", name, v);
+  return MPC_OK;
+}
+
+int make_pyramid(int cap_tokens, int s, int n_levels, const int32_t* fanout, int summary_rows, Pyramid* p,
+                 bool need_rows) {
+  if (s < 1 || s > 4096) return fail(MPC_ERR_BAD_SHAPE, "cluster_size %d not in [1, 4096]", s);
+  if (n_levels < 1 || n_levels > kMaxLevels) return fail(MPC_ERR_BAD_SHAPE, "n_levels %d not in [1, %d]", n_levels, kMaxLevels);
+  if (cap_tokens < 1 || cap_tokens % s != 0)
+    return fail(MPC_ERR_BAD_SHAPE, "cap_tokens %d must be a positive multiple of cluster_size %d", cap_tokens, s);
+  memset(p, 0, sizeof(*p));
+  p->n_levels = n_levels;
+  p->s = s;
+  int rows = 0;
+  int cap = cap_tokens / s;
+  for (int l = 0; l < n_levels; ++l) {
+    if (l > 0) {
+      const int f = fanout[l - 1];
+      if (f < 2 || f > 4096) return fail(MPC_ERR_BAD_SHAPE, "fanout[%d] = %d not in [2, 4096]", l - 1, f);
+      p->fanout[l - 1] = f;
+      cap = (cap + f - 1) / f;
+    }
+    p->cap[l] = cap;
+    p->off[l] = rows;
+    rows += cap;
+  }
+  p->rows = rows;
+  if (need_rows && summary_rows < rows)
+    return fail(MPC_ERR_BAD_SHAPE, "summary_rows %d < %d rows the pyramid needs", summary_rows, rows);
+  if (need_rows) p->rows = summary_rows;
+  return MPC_OK;
+}
+
+int window_bound(int t_max, int wppm, int lppm, int thr) {
+  const int a = count_from_ppm(t_max < thr ? t_max : thr, wppm);
+  const int b = t_max > thr ? count_from_ppm(t_max, lppm) : 0;
+  return a > b ? a : b;
+}
+
+// -------------------------------------------------------------- static ----
+int validate_static(const mpc_static_args* a, StaticParams* p) {
+  if (a == nullptr) return fail(MPC_ERR_INVALID_ARG, "args is NULL");
+  if (a->struct_size != sizeof(mpc_static_args))
+    return fail(MPC_ERR_INVALID_ARG, "struct_size %u != %zu", a->struct_size, sizeof(mpc_static_args));
+  MPC_TRY(check_common(a->batch, a->n_q_heads, a->n_kv_heads, a->head_dim, a->dtype));
+  memset(p, 0, sizeof(*p));
+  MPC_TRY(check_refs(a->n_refs, a->refs, true, &p->refs));
+  MPC_TRY(check_ppm(a->window_ppm, "window_ppm"));
+  MPC_TRY(check_ppm(a->long_window_ppm, "long_window_ppm"));
+  MPC_TRY(check_ppm(a->keep_ppm, "keep_ppm"));
+  if (a->t_max < 1 || a->t_max > 49152) return fail(MPC_ERR_BAD_SHAPE, "t_max %d not in [1, 49152]", a->t_max);
+  if (a->long_prompt_threshold < 1) return fail(MPC_ERR_BAD_SHAPE, "long_prompt_threshold < 1");
+  const int wb = window_bound(a->t_max, a->window_ppm, a->long_window_ppm, a->long_prompt_threshold);
+  if (a->win_rows < wb) return fail(MPC_ERR_BAD_SHAPE, "win_rows %d < longest window %d", a->win_rows, wb);
+  const int kb = count_from_ppm(a->t_max, a->keep_ppm);
+  if (a->keep_cap < kb) return fail(MPC_ERR_BAD_SHAPE, "keep_cap %d < %d kept tokens at t_max", a->keep_cap, kb);
+  if (a->scale < 0.f || !std::isfinite(a->scale)) return fail(MPC_ERR_BAD_SHAPE, "scale must be finite and >= 0");
+  const mpc_kv_tensor& k = a->k;
+  if (k.page_table != nullptr && (k.page_size < 1 || k.max_pages < 1 ||
+                                  (int64_t)k.page_size * k.max_pages < a->t_max))
+    return fail(MPC_ERR_BAD_SHAPE, "paged keys: page_size * max_pages must cover t_max");
+  if (a->n_kv_heads * a->batch * a->n_refs > 65535 || a->n_q_heads * a->batch * a->n_refs > 65535)
+    return fail(MPC_ERR_BAD_SHAPE, "too many (ref, sequence, head) units for one call");
+  p->n_refs = a->n_refs;
+  p->B = a->batch;
+  p->Hq = a->n_q_heads;
+  p->Hkv = a->n_kv_heads;
+  p->G = a->n_q_heads / a->n_kv_heads;
+  p->t_max = a->t_max;
+  p->lens = a->prompt_lens;
+  p->q_win = a->q_win;
+  p->qw_ls = a->q_win_layer_stride;
+  p->win_rows = a->win_rows;
+  p->k = k.data;
+  p->k_ls = k.layer_stride;
+  p->page_table = k.page_table;
+  p->page_size = k.page_size;
+  p->max_pages = k.max_pages;
+  p->window_ppm = a->window_ppm;
+  p->long_window_ppm = a->long_window_ppm;
+  p->long_threshold = a->long_prompt_threshold;
+  p->keep_ppm = a->keep_ppm;
+  const float scale = a->scale > 0.f ? a->scale : 1.0f / sqrtf((float)a->head_dim);
+  p->scale_log2 = scale * 1.4426950408889634f;
+  p->keep_cap = a->keep_cap;
+  p->scores = a->out_scores;
+  p->kept = a->out_kept;
+  p->n_keep = a->out_n_keep;
+  return MPC_OK;
+}
+
+size_t static_ws(const StaticParams& p) { return (size_t)p.n_refs * p.B * p.Hq * p.win_rows * sizeof(float2); }
+
+// ------------------------------------------------------------ clusters ----
+int validate_clusters(const mpc_cluster_args* a, ClusterParams* p) {
+  if (a == nullptr) return fail(MPC_ERR_INVALID_ARG, "args is NULL");
+  if (a->struct_size != sizeof(mpc_cluster_args))
+    return fail(MPC_ERR_INVALID_ARG, "struct_size %u != %zu", a->struct_size, sizeof(mpc_cluster_args));
+  MPC_TRY(check_common(a->batch, a->n_kv_heads, a->n_kv_heads, a->head_dim, a->dtype));
+  memset(p, 0, sizeof(*p));
+  MPC_TRY(check_refs(a->n_refs, a->refs, false, &p->refs));
+  MPC_TRY(make_pyramid(a->cap_tokens, a->cluster_size, a->n_levels, a->fanout, a->summary_rows, &p->pyr, true));
+  if (a->t_max < 1) return fail(MPC_ERR_BAD_SHAPE, "t_max < 1");
+  if (a->keep_cap < 1) return fail(MPC_ERR_BAD_SHAPE, "keep_cap < 1");
+  if (a->alpha < 0.f || a->alpha > 1.f) return fail(MPC_ERR_BAD_SHAPE, "alpha %g not in [0, 1]", a->alpha);
+  const int es = esize(a->dtype);
+  if (!aligned16(a->kc) || !aligned16(a->vc) || (a->cache_layer_stride * es) % 16 != 0)
+    return fail(MPC_ERR_INVALID_ARG, "kc / vc and their layer stride must be 16-byte aligned");
+  if (!aligned16(a->k.data) || !aligned16(a->v.data) || (a->k.layer_stride * es) % 16 || (a->v.layer_stride * es) % 16)
+    return fail(MPC_ERR_INVALID_ARG, "prompt K / V and their layer strides must be 16-byte aligned");
+  if (a->n_kv_heads * a->batch * a->n_refs > 65535) return fail(MPC_ERR_BAD_SHAPE, "too many units for one call");
+  bool any_leader = false;
+  for (int i = 0; i < a->n_refs; ++i) any_leader |= a->refs[i].leader != 0;
+  if (any_leader && a->n_levels >= 1)
+    if (a->r_max == nullptr || a->r_min == nullptr || a->rep == nullptr)
+      return fail(MPC_ERR_INVALID_ARG, "a leader ref needs r_max, r_min and rep");
+  p->n_refs = a->n_refs;
+  p->B = a->batch;
+  p->Hkv = a->n_kv_heads;
+  p->t_max = a->t_max;
+  p->k = KvSrc{a->k.data, a->k.layer_stride, a->k.page_table, a->k.page_size, a->k.max_pages};
+  p->v = KvSrc{a->v.data, a->v.layer_stride, a->v.page_table, a->v.page_size, a->v.max_pages};
+  p->kept = a->kept;
+  p->keep_cap = a->keep_cap;
+  p->n_keep = a->n_keep;
+  p->kc = a->kc;
+  p->vc = a->vc;
+  p->cache_ls = a->cache_layer_stride;
+  p->cap_tokens = a->cap_tokens;
+  p->rmax = a->r_max;
+  p->rmin = a->r_min;
+  p->rep = a->rep;
+  p->alpha = a->alpha;
+  p->out_n_tok = a->out_n_tok;
+  return MPC_OK;
+}
+
+// -------------------------------------------------------------- select ----
+int validate_select(const mpc_select_args* a, SelectParams* p) {
+  if (a == nullptr) return fail(MPC_ERR_INVALID_ARG, "args is NULL");
+  if (a->struct_size != sizeof(mpc_select_args))
+    return fail(MPC_ERR_INVALID_ARG, "struct_size %u != %zu", a->struct_size, sizeof(mpc_select_args));
+  MPC_TRY(check_common(a->batch, a->n_q_heads, a->n_kv_heads, a->head_dim, a->dtype));
+  memset(p, 0, sizeof(*p));
+  MPC_TRY(check_refs(a->n_refs, a->refs, true, &p->refs));
+  MPC_TRY(make_pyramid(a->cap_tokens, a->cluster_size, a->n_levels, a->fanout, a->summary_rows, &p->pyr, true));
+  for (int l = 0; l < a->n_levels; ++l) MPC_TRY(check_ppm(a->level_keep_ppm[l], "level_keep_ppm"));
+  if (!aligned16(a->rep)) return fail(MPC_ERR_INVALID_ARG, "rep must be 16-byte aligned");
+  // bound on the candidates of any level
+  int kmax[kMaxLevels] = {0};
+  long long mc = 0;
+  for (int l = a->n_levels - 1; l >= 0; --l) {
+    long long cand = p->pyr.cap[l];
+    if (l < a->n_levels - 1) {
+      const long long ch = (long long)p->pyr.fanout[l] * kmax[l + 1];
+      if (ch < cand) cand = ch;
+    }
+    kmax[l] = count_from_ppm(p->pyr.cap[l], a->level_keep_ppm[l]);
+    if (cand > mc) mc = cand;
+  }
+  if (mc > 8192) return fail(MPC_ERR_BAD_SHAPE, "up to %lld candidates at one level exceed 8192", mc);
+  int P = 1;
+  while (P < mc) P <<= 1;
+  if (a->sel_cap < kmax[0]) return fail(MPC_ERR_BAD_SHAPE, "sel_cap %d < %d selected clusters", a->sel_cap, kmax[0]);
+  if (a->n_kv_heads * a->batch * a->n_refs > 65535) return fail(MPC_ERR_BAD_SHAPE, "too many units for one call");
+  p->n_refs = a->n_refs;
+  p->B = a->batch;
+  p->Hq = a->n_q_heads;
+  p->Hkv = a->n_kv_heads;
+  p->G = a->n_q_heads / a->n_kv_heads;
+  p->q = a->q;
+  p->q_ls = a->q_layer_stride;
+  p->rep = a->rep;
+  p->n_tok = a->n_tok;
+  for (int l = 0; l < a->n_levels; ++l) p->keep_ppm[l] = a->level_keep_ppm[l];
+  p->sel_cap = a->sel_cap;
+  p->out_sel = a->out_sel;
+  p->out_n_sel = a->out_n_sel;
+  p->max_cand = P;
+  return MPC_OK;
+}
+
+// ---------------------------------------------------------- attention ----
+struct AttnPlan {
+  int units, n_split, tps;
+  size_t part_off, ucnt_off, gcnt_off, bytes;
+};
+
+int validate_attn(const mpc_attn_args* a, AttnParams* p, AttnPlan* plan) {
+  if (a == nullptr) return fail(MPC_ERR_INVALID_ARG, "args is NULL");
+  if (a->struct_size != sizeof(mpc_attn_args))
+    return fail(MPC_ERR_INVALID_ARG, "struct_size %u != %zu", a->struct_size, sizeof(mpc_attn_args));
+  MPC_TRY(check_common(a->batch, a->n_q_heads, a->n_kv_heads, a->head_dim, a->dtype));
+  memset(p, 0, sizeof(*p));
+  MPC_TRY(check_refs(a->n_refs, a->refs, false, &p->refs));
+  MPC_TRY(make_pyramid(a->cap_tokens, a->cluster_size, a->n_levels, a->fanout, a->summary_rows, &p->pyr, false));
+  const int G = a->n_q_heads / a->n_kv_heads;
+  if (G > (a->dtype == MPC_BF16 ? 16 : 8))
+    return fail(MPC_ERR_BAD_SHAPE, "%d query heads per kv head exceed %d", G, a->dtype == MPC_BF16 ? 16 : 8);
+  if (a->sel_cap < 0) return fail(MPC_ERR_BAD_SHAPE, "sel_cap < 0");
+  if (a->alpha < 0.f || a->alpha > 1.f) return fail(MPC_ERR_BAD_SHAPE, "alpha %g not in [0, 1]", a->alpha);
+  if (a->scale < 0.f || !std::isfinite(a->scale)) return fail(MPC_ERR_BAD_SHAPE, "scale must be finite and >= 0");
+  const int es = esize(a->dtype);
+  if (!aligned16(a->kc) || !aligned16(a->vc) || (a->cache_layer_stride * es) % 16 != 0)
+    return fail(MPC_ERR_INVALID_ARG, "kc / vc and their layer stride must be 16-byte aligned");
+  if (!aligned16(a->q) || !aligned16(a->k_new) || !aligned16(a->v_new) || (a->q_layer_stride * es) % 16 ||
+      (a->kv_new_layer_stride * es) % 16)
+    return fail(MPC_ERR_INVALID_ARG, "q / k_new / v_new and their layer strides must be 16-byte aligned");
+  bool any_leader = false;
+  for (int i = 0; i < a->n_refs; ++i) any_leader |= a->refs[i].leader != 0;
+  if (any_leader && a->r_max != nullptr) {
+    if (a->r_min == nullptr || a->rep == nullptr) return fail(MPC_ERR_INVALID_ARG, "r_max given without r_min / rep");
+    if (a->summary_rows < p->pyr.rows)
+      return fail(MPC_ERR_BAD_SHAPE, "summary_rows %d < %d rows the pyramid needs", a->summary_rows, p->pyr.rows);
+  }
+  p->pyr.rows = a->summary_rows > p->pyr.rows ? a->summary_rows : p->pyr.rows;
+
+  const int units = a->n_refs * a->batch * a->n_kv_heads;
+  if (units > 65535) return fail(MPC_ERR_BAD_SHAPE, "too many (ref, sequence, kv head) units for one call");
+  // tiles of the longest list: sel_cap clusters plus a tail of at most s rows
+  const long long rows_max = (long long)a->sel_cap * a->cluster_size + a->cluster_size;
+  const int tiles_max = (int)((rows_max + 15) / 16);
+  int n_split = (1024 + units - 1) / units;
+  if (n_split > 64) n_split = 64;
+  if (n_split > tiles_max) n_split = tiles_max;
+  if (n_split < 1) n_split = 1;
+  int tps = (tiles_max + n_split - 1) / n_split;
+  n_split = (tiles_max + tps - 1) / tps;
+  plan->units = units;
+  plan->n_split = n_split;
+  plan->tps = tps;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += (bytes + 255) & ~size_t(255);
+    return o;
+  };
+  plan->part_off = take(n_split > 1 ? (size_t)units * n_split * G * (a->head_dim + 4) * sizeof(float) : 0);
+  plan->ucnt_off = take((size_t)units * sizeof(int));
+  plan->gcnt_off = take(sizeof(int));
+  plan->bytes = off;
+
+  p->n_refs = a->n_refs;
+  p->B = a->batch;
+  p->Hq = a->n_q_heads;
+  p->Hkv = a->n_kv_heads;
+  p->G = G;
+  p->q = a->q;
+  p->k_new = a->k_new;
+  p->v_new = a->v_new;
+  p->q_ls = a->q_layer_stride;
+  p->kvn_ls = a->kv_new_layer_stride;
+  p->kc = a->kc;
+  p->vc = a->vc;
+  p->cache_ls = a->cache_layer_stride;
+  p->cap_tokens = a->cap_tokens;
+  p->sel = a->sel;
+  p->n_sel = a->n_sel;
+  p->sel_cap = a->sel_cap;
+  if (any_leader && a->r_max != nullptr) {
+    p->rmax = a->r_max;
+    p->rmin = a->r_min;
+    p->rep = a->rep;
+  }
+  p->alpha = a->alpha;
+  p->n_tok = a->n_tok;
+  p->advance = a->advance != 0;
+  const float scale = a->scale > 0.f ? a->scale : 1.0f / sqrtf((float)a->head_dim);
+  p->scale_log2 = scale * 1.4426950408889634f;
+  p->out = a->out;
+  p->out_ls = a->out_layer_stride;
+  p->n_split = n_split;
+  p->tiles_per_split = tps;
+  return MPC_OK;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+  return fail(MPC_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+}  // namespace
+}  // namespace mpc
+
+using namespace mpc;
+
+extern "C" {
+
+MPC_API int mpc_abi_version(void) { return MPC_ABI_VERSION; }
+
+MPC_API const char* mpc_last_error(void) { return g_err.c_str(); }
+
+MPC_API int64_t mpc_summary_rows(int32_t cap_tokens, int32_t cluster_size, int32_t n_levels, const int32_t* fanout) {
+  Pyramid p;
+  int32_t none[kMaxLevels] = {0, 0, 0, 0};
+  const int rc = make_pyramid(cap_tokens, cluster_size, n_levels, fanout ? fanout : none, 0, &p, false);
+  if (rc != MPC_OK) return rc;
+  return p.rows;
+}
+
+MPC_API int mpc_device_status(int* flags) {
+  if (flags == nullptr) return fail(MPC_ERR_INVALID_ARG, "flags is NULL");
+  const cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
+  const int parts[4] = {take_status_attn(), take_status_select(), take_status_clusters(), take_status_static()};
+  int v = 0;
+  for (int x : parts) {
+    if (x < 0) return fail(MPC_ERR_CUDA, "reading the device status word failed");
+    v |= x;
+  }
+  *flags = v;
+  return ok();
+}
+
+MPC_API int mpc_static_evict_workspace_size(const mpc_static_args* args, size_t* bytes) {
+  if (bytes == nullptr) return fail(MPC_ERR_INVALID_ARG, "bytes is NULL");
+  StaticParams p;
+  MPC_TRY(validate_static(args, &p));
+  *bytes = static_ws(p);
+  return ok();
+}
+
+MPC_API int mpc_static_evict(const mpc_static_args* args, void* workspace, size_t workspace_bytes, void* stream) {
+  StaticParams p;
+  MPC_TRY(validate_static(args, &p));
+  if (!args->q_win || !args->k.data || !args->prompt_lens || !args->out_scores || !args->out_kept || !args->out_n_keep)
+    return fail(MPC_ERR_INVALID_ARG, "a required pointer is NULL");
+  const size_t need = static_ws(p);
+  if (workspace == nullptr || workspace_bytes < need)
+    return fail(MPC_ERR_WORKSPACE, "workspace of %zu bytes needed", need);
+  p.stats = static_cast<float2*>(workspace);
+  const cudaError_t e = launch_static(p, args->dtype, args->head_dim, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "mpc_static_evict launch");
+  return ok();
+}
+
+MPC_API int mpc_build_clusters_workspace_size(const mpc_cluster_args* args, size_t* bytes) {
+  if (bytes == nullptr) return fail(MPC_ERR_INVALID_ARG, "bytes is NULL");
+  ClusterParams p;
+  MPC_TRY(validate_clusters(args, &p));
+  *bytes = 0;
+  return ok();
+}
+
+MPC_API int mpc_build_clusters(const mpc_cluster_args* args, void* workspace, size_t workspace_bytes, void* stream) {
+  (void)workspace;
+  (void)workspace_bytes;
+  ClusterParams p;
+  MPC_TRY(validate_clusters(args, &p));
+  if (!args->k.data || !args->v.data || !args->kept || !args->n_keep || !args->kc || !args->vc || !args->out_n_tok)
+    return fail(MPC_ERR_INVALID_ARG, "a required pointer is NULL");
+  const int units = args->n_refs * args->batch * args->n_kv_heads;
+  const int clusters = (args->keep_cap + args->cluster_size - 1) / args->cluster_size;
+  const int gx = (clusters + 3) / 4;
+  bool any_leader = false;
+  for (int i = 0; i < args->n_refs; ++i) any_leader |= args->refs[i].leader != 0;
+  const cudaError_t e = launch_clusters(p, args->dtype, args->head_dim, units, gx > 0 ? gx : 1, any_leader,
+                                        static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "mpc_build_clusters launch");
+  return ok();
+}
+
+MPC_API int mpc_select_workspace_size(const mpc_select_args* args, size_t* bytes) {
+  if (bytes == nullptr) return fail(MPC_ERR_INVALID_ARG, "bytes is NULL");
+  SelectParams p;
+  MPC_TRY(validate_select(args, &p));
+  *bytes = 0;
+  return ok();
+}
+
+MPC_API int mpc_select(const mpc_select_args* args, void* workspace, size_t workspace_bytes, void* stream) {
+  (void)workspace;
+  (void)workspace_bytes;
+  SelectParams p;
+  MPC_TRY(validate_select(args, &p));
+  if (!args->q || !args->rep || !args->n_tok || !args->out_sel || !args->out_n_sel)
+    return fail(MPC_ERR_INVALID_ARG, "a required pointer is NULL");
+  const int units = args->n_refs * args->batch * args->n_kv_heads;
+  const cudaError_t e = launch_select(p, args->dtype, args->head_dim, units, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "mpc_select launch");
+  return ok();
+}
+
+MPC_API int mpc_sparse_decode_attn_workspace_size(const mpc_attn_args* args, size_t* bytes) {
+  if (bytes == nullptr) return fail(MPC_ERR_INVALID_ARG, "bytes is NULL");
+  AttnParams p;
+  AttnPlan plan;
+  MPC_TRY(validate_attn(args, &p, &plan));
+  *bytes = plan.bytes;
+  return ok();
+}
+
+MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace, size_t workspace_bytes, void* stream) {
+  AttnParams p;
+  AttnPlan plan;
+  MPC_TRY(validate_attn(args, &p, &plan));
+  if (!args->q || !args->k_new || !args->v_new || !args->kc || !args->vc || !args->n_tok || !args->out ||
+      (args->sel_cap > 0 && (!args->sel || !args->n_sel)))
+    return fail(MPC_ERR_INVALID_ARG, "a required pointer is NULL");
+  if (workspace == nullptr || workspace_bytes < plan.bytes)
+    return fail(MPC_ERR_WORKSPACE, "workspace of %zu bytes needed", plan.bytes);
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  p.part = reinterpret_cast<float*>(ws + plan.part_off);
+  p.unit_counter = reinterpret_cast<int*>(ws + plan.ucnt_off);
+  p.grid_counter = reinterpret_cast<int*>(ws + plan.gcnt_off);
+  const cudaError_t e = launch_attn(p, args->dtype, args->head_dim, plan.units, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "mpc_sparse_decode_attn launch");
+  return ok();
+}
+
+}  // extern "C"

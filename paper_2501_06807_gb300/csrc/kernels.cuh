@@ -1,0 +1,114 @@
+// Kernel parameter blocks and launchers of the MPCache library.
+#pragma once
+
+#include "common.cuh"
+
+namespace mpc {
+
+struct AttnParams {
+  RefTable refs;
+  int n_refs, B, Hq, Hkv, G;
+  const void* q;
+  const void* k_new;
+  const void* v_new;
+  int64_t q_ls, kvn_ls;
+  void* kc;
+  void* vc;
+  int64_t cache_ls;
+  int cap_tokens;
+  const int* sel;
+  const int* n_sel;
+  int sel_cap;
+  float* rmax;
+  float* rmin;
+  float* rep;
+  Pyramid pyr;
+  float alpha;
+  int* n_tok;
+  int advance;
+  float scale_log2;  // softmax scale times log2(e)
+  float* out;
+  int64_t out_ls;
+  int n_split, tiles_per_split;
+  float* part;        // [unit][split][G][D + 4]
+  int* unit_counter;  // [unit]
+  int* grid_counter;  // [1]
+};
+
+struct SelectParams {
+  RefTable refs;
+  int n_refs, B, Hq, Hkv, G;
+  const void* q;
+  int64_t q_ls;
+  const float* rep;
+  Pyramid pyr;
+  const int* n_tok;
+  int keep_ppm[kMaxLevels];
+  int sel_cap;
+  int* out_sel;
+  int* out_n_sel;
+  int max_cand;  // power of two, capacity of the shared candidate arrays
+};
+
+struct StaticParams {
+  RefTable refs;
+  int n_refs, B, Hq, Hkv, G, t_max;
+  const int* lens;
+  const void* q_win;
+  int64_t qw_ls;
+  int win_rows;
+  const void* k;
+  int64_t k_ls;
+  const int* page_table;
+  int page_size, max_pages;
+  int window_ppm, long_window_ppm, long_threshold, keep_ppm;
+  float scale_log2;
+  int keep_cap;
+  float* scores;      // [group][b][Hkv][t_max]
+  int* kept;          // [group][b][Hkv][keep_cap]
+  int* n_keep;        // [b]
+  float2* stats;      // [ref][b][Hq][win_rows]: (m, 1 / l)
+};
+
+struct KvSrc {
+  const void* data;
+  int64_t layer_stride;
+  const int* page_table;
+  int page_size, max_pages;
+};
+
+struct ClusterParams {
+  RefTable refs;
+  int n_refs, B, Hkv, t_max;
+  KvSrc k, v;
+  const int* kept;
+  int keep_cap;
+  const int* n_keep;
+  void* kc;
+  void* vc;
+  int64_t cache_ls;
+  int cap_tokens;
+  float* rmax;
+  float* rmin;
+  float* rep;
+  Pyramid pyr;
+  float alpha;
+  int* out_n_tok;
+};
+
+cudaError_t launch_attn(const AttnParams& p, int dtype, int D, int n_units, cudaStream_t st);
+int attn_smem_bytes(int dtype, int D, int G);
+cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cudaStream_t st);
+int select_smem_bytes(int D, int max_cand);
+cudaError_t launch_clusters(const ClusterParams& p, int dtype, int D, int n_units, int groups_x,
+                            bool any_leader, cudaStream_t st);
+cudaError_t launch_static(const StaticParams& p, int dtype, int D, cudaStream_t st);
+int static_tile_smem(int D);
+
+// Device status word of each translation unit: read it and clear it.
+int take_status_attn();
+int take_status_select();
+int take_status_clusters();
+int take_status_static();
+
+}  // namespace mpc

@@ -1,0 +1,386 @@
+"""Python binding of libmpcache.so (include/mpcache.h).
+
+Argument marshalling only: every step of the method runs in the library's
+CUDA kernels.  Tensors are torch tensors on the current CUDA device; calls
+are queued on torch's current stream.  The library must have been built
+(``paper_2501_06807_gb300.build.build()``); importing this module without it
+raises, there is no fallback.
+
+``Engine`` owns the device buffers of one batch (cluster-major cache, summary
+pyramid, selections, workspaces) and runs the method: ``prefill`` (static
+eviction of the leader layers, then gathering and clustering of every layer)
+and ``decode_step`` (selection for the leaders, then append + sparse attention
+for every layer, all layers of a step in one launch each).
+"""
+from __future__ import annotations
+
+import ctypes as C
+import math
+import os
+from typing import List, Optional, Sequence
+
+import torch
+
+from . import build as _build
+
+MPC_OK, MPC_ERR_INVALID_ARG, MPC_ERR_BAD_SHAPE, MPC_ERR_WORKSPACE, MPC_ERR_CUDA = 0, -1, -2, -3, -4
+MPC_F32, MPC_BF16 = 0, 1
+MAX_LEVELS = 4
+MAX_REFS = 128
+PPM = 1_000_000
+
+
+class LayerRef(C.Structure):
+    _fields_ = [("layer", C.c_int32), ("group", C.c_int32), ("leader", C.c_int32)]
+
+
+class KvTensor(C.Structure):
+    _fields_ = [("data", C.c_void_p), ("layer_stride", C.c_int64), ("page_table", C.c_void_p),
+                ("page_size", C.c_int32), ("max_pages", C.c_int32)]
+
+
+class StaticArgs(C.Structure):
+    _fields_ = [("struct_size", C.c_uint32), ("n_refs", C.c_int32), ("refs", C.POINTER(LayerRef)),
+                ("batch", C.c_int32), ("n_q_heads", C.c_int32), ("n_kv_heads", C.c_int32),
+                ("head_dim", C.c_int32), ("dtype", C.c_int32), ("t_max", C.c_int32),
+                ("prompt_lens", C.c_void_p), ("q_win", C.c_void_p), ("q_win_layer_stride", C.c_int64),
+                ("win_rows", C.c_int32), ("k", KvTensor), ("window_ppm", C.c_int32),
+                ("long_window_ppm", C.c_int32), ("long_prompt_threshold", C.c_int32),
+                ("keep_ppm", C.c_int32), ("scale", C.c_float), ("keep_cap", C.c_int32),
+                ("out_scores", C.c_void_p), ("out_kept", C.c_void_p), ("out_n_keep", C.c_void_p)]
+
+
+class ClusterArgs(C.Structure):
+    _fields_ = [("struct_size", C.c_uint32), ("n_refs", C.c_int32), ("refs", C.POINTER(LayerRef)),
+                ("batch", C.c_int32), ("n_kv_heads", C.c_int32), ("head_dim", C.c_int32),
+                ("dtype", C.c_int32), ("t_max", C.c_int32), ("k", KvTensor), ("v", KvTensor),
+                ("kept", C.c_void_p), ("keep_cap", C.c_int32), ("n_keep", C.c_void_p),
+                ("kc", C.c_void_p), ("vc", C.c_void_p), ("cache_layer_stride", C.c_int64),
+                ("cap_tokens", C.c_int32), ("r_max", C.c_void_p), ("r_min", C.c_void_p),
+                ("rep", C.c_void_p), ("summary_rows", C.c_int32), ("cluster_size", C.c_int32),
+                ("n_levels", C.c_int32), ("fanout", C.c_int32 * MAX_LEVELS), ("alpha", C.c_float),
+                ("out_n_tok", C.c_void_p)]
+
+
+class SelectArgs(C.Structure):
+    _fields_ = [("struct_size", C.c_uint32), ("n_refs", C.c_int32), ("refs", C.POINTER(LayerRef)),
+                ("batch", C.c_int32), ("n_q_heads", C.c_int32), ("n_kv_heads", C.c_int32),
+                ("head_dim", C.c_int32), ("dtype", C.c_int32), ("q", C.c_void_p),
+                ("q_layer_stride", C.c_int64), ("rep", C.c_void_p), ("summary_rows", C.c_int32),
+                ("cap_tokens", C.c_int32), ("n_tok", C.c_void_p), ("cluster_size", C.c_int32),
+                ("n_levels", C.c_int32), ("fanout", C.c_int32 * MAX_LEVELS),
+                ("level_keep_ppm", C.c_int32 * MAX_LEVELS), ("sel_cap", C.c_int32),
+                ("out_sel", C.c_void_p), ("out_n_sel", C.c_void_p)]
+
+
+class AttnArgs(C.Structure):
+    _fields_ = [("struct_size", C.c_uint32), ("n_refs", C.c_int32), ("refs", C.POINTER(LayerRef)),
+                ("batch", C.c_int32), ("n_q_heads", C.c_int32), ("n_kv_heads", C.c_int32),
+                ("head_dim", C.c_int32), ("dtype", C.c_int32), ("q", C.c_void_p),
+                ("k_new", C.c_void_p), ("v_new", C.c_void_p), ("q_layer_stride", C.c_int64),
+                ("kv_new_layer_stride", C.c_int64), ("kc", C.c_void_p), ("vc", C.c_void_p),
+                ("cache_layer_stride", C.c_int64), ("cap_tokens", C.c_int32), ("sel", C.c_void_p),
+                ("n_sel", C.c_void_p), ("sel_cap", C.c_int32), ("r_max", C.c_void_p),
+                ("r_min", C.c_void_p), ("rep", C.c_void_p), ("summary_rows", C.c_int32),
+                ("cluster_size", C.c_int32), ("n_levels", C.c_int32), ("fanout", C.c_int32 * MAX_LEVELS),
+                ("alpha", C.c_float), ("n_tok", C.c_void_p), ("advance", C.c_int32),
+                ("scale", C.c_float), ("out", C.c_void_p), ("out_layer_stride", C.c_int64)]
+
+
+ENTRY_POINTS = ("mpc_static_evict_workspace_size", "mpc_build_clusters_workspace_size",
+                "mpc_select_workspace_size", "mpc_sparse_decode_attn_workspace_size",
+                "mpc_static_evict", "mpc_build_clusters", "mpc_select", "mpc_sparse_decode_attn",
+                "mpc_summary_rows", "mpc_last_error", "mpc_device_status", "mpc_abi_version")
+
+_LIB = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(path: Optional[str] = None) -> C.CDLL:
+    """Load libmpcache.so (raises OSError if it has not been built)."""
+    global _LIB
+    if _LIB is not None and path is None:
+        return _LIB
+    p = path or library_path()
+    if not os.path.exists(p):
+        raise OSError(f"libmpcache.so not found at {p}; run paper_2501_06807_gb300.build.build()")
+    lib = C.CDLL(p)
+    for name in ("mpc_static_evict_workspace_size", "mpc_build_clusters_workspace_size",
+                 "mpc_select_workspace_size", "mpc_sparse_decode_attn_workspace_size"):
+        getattr(lib, name).restype = C.c_int
+        getattr(lib, name).argtypes = [C.c_void_p, C.POINTER(C.c_size_t)]
+    for name in ("mpc_static_evict", "mpc_build_clusters", "mpc_select", "mpc_sparse_decode_attn"):
+        getattr(lib, name).restype = C.c_int
+        getattr(lib, name).argtypes = [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]
+    lib.mpc_summary_rows.restype = C.c_int64
+    lib.mpc_summary_rows.argtypes = [C.c_int32, C.c_int32, C.c_int32, C.POINTER(C.c_int32)]
+    lib.mpc_last_error.restype = C.c_char_p
+    lib.mpc_device_status.restype = C.c_int
+    lib.mpc_device_status.argtypes = [C.POINTER(C.c_int)]
+    lib.mpc_abi_version.restype = C.c_int
+    if path is None:
+        _LIB = lib
+    return lib
+
+
+class MPCError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"mpcache error {code}: {msg}")
+        self.code = code
+
+
+def _check(rc: int) -> None:
+    if rc != MPC_OK:
+        raise MPCError(rc, load().mpc_last_error().decode())
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _stream() -> int:
+    return torch.cuda.current_stream().cuda_stream
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return MPC_F32
+    if t.dtype == torch.bfloat16:
+        return MPC_BF16
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _refs(refs: Sequence[tuple]):
+    arr = (LayerRef * len(refs))(*[LayerRef(int(l), int(g), int(bool(ld))) for l, g, ld in refs])
+    return arr
+
+
+def _fan(fanouts: Sequence[int]):
+    a = (C.c_int32 * MAX_LEVELS)()
+    for i, f in enumerate(fanouts):
+        a[i] = int(f)
+    return a
+
+
+def _ws_zero(nbytes: int, cache: dict, key) -> torch.Tensor:
+    ws = cache.get(key)
+    if ws is None or ws.numel() < nbytes:
+        ws = torch.zeros(max(nbytes, 256), dtype=torch.uint8, device="cuda")
+        cache[key] = ws
+    return ws
+
+
+# ----------------------------------------------------------- host rules ----
+
+def ppm_count(n: int, ppm: int) -> int:
+    """min(n, max(1, ceil(n * ppm / 1e6))), 0 for n = 0 (the library's rule)."""
+    if n <= 0:
+        return 0
+    return min(n, max(1, (n * ppm + PPM - 1) // PPM))
+
+
+def window_rows_bound(t_max: int, window_ppm: int, long_ppm: int, threshold: int) -> int:
+    """Longest static-eviction window over prompt lengths 1..t_max."""
+    a = ppm_count(min(t_max, threshold), window_ppm)
+    b = ppm_count(t_max, long_ppm) if t_max > threshold else 0
+    return max(a, b)
+
+
+def sharing_leader(layer: int, share_every: int) -> int:
+    """Leader layer of ``layer`` under cross-layer index sharing: layers 0 and 1
+    lead themselves, later layers form groups of ``share_every``."""
+    if share_every <= 1 or layer < 2:
+        return layer
+    return 2 + share_every * ((layer - 2) // share_every)
+
+
+def summary_rows(cap_tokens: int, s: int, fanouts: Sequence[int]) -> int:
+    arr = (C.c_int32 * MAX_LEVELS)(*([int(f) for f in fanouts] + [0] * (MAX_LEVELS - len(fanouts))))
+    r = load().mpc_summary_rows(cap_tokens, s, 1 + len(fanouts), arr)
+    if r < 0:
+        _check(int(r))
+    return int(r)
+
+
+def device_status() -> int:
+    v = C.c_int(0)
+    _check(load().mpc_device_status(C.byref(v)))
+    return v.value
+
+
+# -------------------------------------------------------------- engine ----
+
+class Engine:
+    """Device state of one batch of the MPCache decode path."""
+
+    def __init__(self, *, n_layers: int, batch: int, n_q_heads: int, n_kv_heads: int, head_dim: int,
+                 dtype: torch.dtype, t_max: int, keep_ppm: int, cluster_size: int,
+                 fanouts: Sequence[int], level_keep_ppm: Sequence[int], share_every: int,
+                 max_decode_steps: int, alpha: float = 0.6, window_ppm: int = 200_000,
+                 long_window_ppm: int = 100_000, long_prompt_threshold: int = 24_576,
+                 scale: float = 0.0, layers: Optional[Sequence[int]] = None):
+        load()
+        self.L, self.B, self.Hq, self.Hkv, self.d = n_layers, batch, n_q_heads, n_kv_heads, head_dim
+        self.dtype = dtype
+        self.dcode = MPC_BF16 if dtype == torch.bfloat16 else MPC_F32
+        self.t_max, self.keep_ppm, self.s = t_max, keep_ppm, cluster_size
+        self.fanouts = tuple(fanouts)
+        self.n_levels = 1 + len(self.fanouts)
+        self.level_keep_ppm = tuple(level_keep_ppm)
+        assert len(self.level_keep_ppm) == self.n_levels
+        self.share_every = share_every
+        self.alpha, self.scale = alpha, scale
+        self.window_ppm, self.long_window_ppm, self.long_threshold = window_ppm, long_window_ppm, long_prompt_threshold
+        self.layers = list(range(n_layers)) if layers is None else list(layers)
+        lead = [sharing_leader(l, share_every) for l in range(n_layers)]
+        self.leaders = sorted(set(lead[l] for l in self.layers))
+        self.group_of = {l: self.leaders.index(lead[l]) for l in self.layers}
+        self.refs_all = [(l, self.group_of[l], lead[l] == l) for l in self.layers]
+        self.refs_lead = [(l, self.group_of[l], True) for l in self.leaders]
+        missing = [l for l in self.leaders if l not in self.layers]
+        if missing:
+            raise ValueError(f"leader layers {missing} must be among the processed layers")
+        self.n_groups = len(self.leaders)
+        self.win_rows = window_rows_bound(t_max, window_ppm, long_window_ppm, long_prompt_threshold)
+        self.keep_cap = ppm_count(t_max, keep_ppm)
+        s = cluster_size
+        self.cap_tokens = ((self.keep_cap + max_decode_steps + s - 1) // s) * s + s
+        self.rows = summary_rows(self.cap_tokens, s, self.fanouts)
+        self.sel_cap = max(1, ppm_count(self.cap_tokens // s, self.level_keep_ppm[0]))
+        dev = "cuda"
+        f32, i32 = dict(dtype=torch.float32, device=dev), dict(dtype=torch.int32, device=dev)
+        G, B, Hkv, d = self.n_groups, batch, n_kv_heads, head_dim
+        self.scores = torch.zeros((G, B, Hkv, t_max), **f32)
+        self.kept = torch.zeros((G, B, Hkv, self.keep_cap), **i32)
+        self.n_keep = torch.zeros((B,), **i32)
+        self.kc = torch.zeros((n_layers, B, Hkv, self.cap_tokens, d), dtype=dtype, device=dev)
+        self.vc = torch.zeros_like(self.kc)
+        self.rmax = torch.zeros((G, B, Hkv, self.rows, d), **f32)
+        self.rmin = torch.zeros_like(self.rmax)
+        self.rep = torch.zeros_like(self.rmax)
+        self.n_tok = torch.zeros((B,), **i32)
+        self.sel = torch.full((G, B, Hkv, self.sel_cap), -1, **i32)
+        self.n_sel = torch.zeros((B,), **i32)
+        self.out = torch.zeros((n_layers, B, n_q_heads, d), **f32)
+        self._ws = {}
+
+    # --------------------------------------------------------- prefill ----
+    def static_args(self, k: torch.Tensor, q_win: torch.Tensor, lens: torch.Tensor,
+                    page_table: Optional[torch.Tensor] = None, page_size: int = 16) -> StaticArgs:
+        refs = _refs(self.refs_lead)
+        a = StaticArgs()
+        a.struct_size = C.sizeof(StaticArgs)
+        a.n_refs = len(self.refs_lead)
+        a.refs = C.cast(refs, C.POINTER(LayerRef))
+        a.batch, a.n_q_heads, a.n_kv_heads, a.head_dim, a.dtype = self.B, self.Hq, self.Hkv, self.d, self.dcode
+        a.t_max = self.t_max
+        a.prompt_lens = _ptr(lens)
+        a.q_win = _ptr(q_win)
+        a.q_win_layer_stride = q_win.stride(0)
+        a.win_rows = q_win.shape[3]
+        a.k = self._kv(k, page_table, page_size)
+        a.window_ppm, a.long_window_ppm, a.long_prompt_threshold = (self.window_ppm, self.long_window_ppm,
+                                                                   self.long_threshold)
+        a.keep_ppm = self.keep_ppm
+        a.scale = self.scale
+        a.keep_cap = self.keep_cap
+        a.out_scores, a.out_kept, a.out_n_keep = _ptr(self.scores), _ptr(self.kept), _ptr(self.n_keep)
+        a._refs = refs
+        return a
+
+    def _kv(self, t: torch.Tensor, page_table, page_size) -> KvTensor:
+        kv = KvTensor()
+        kv.data = _ptr(t)
+        kv.layer_stride = t.stride(0)
+        if page_table is not None:
+            kv.page_table = _ptr(page_table)
+            kv.page_size = page_size
+            kv.max_pages = page_table.shape[1]
+        return kv
+
+    def static_evict(self, k, q_win, lens, page_table=None, page_size=16):
+        lib = load()
+        a = self.static_args(k, q_win, lens, page_table, page_size)
+        n = C.c_size_t(0)
+        _check(lib.mpc_static_evict_workspace_size(C.byref(a), C.byref(n)))
+        ws = _ws_zero(n.value, self._ws, "static")
+        _check(lib.mpc_static_evict(C.byref(a), C.c_void_p(_ptr(ws)), n.value, C.c_void_p(_stream())))
+
+    def build_clusters(self, k, v, page_table=None, page_size=16):
+        lib = load()
+        refs = _refs(self.refs_all)
+        a = ClusterArgs()
+        a.struct_size = C.sizeof(ClusterArgs)
+        a.n_refs = len(self.refs_all)
+        a.refs = C.cast(refs, C.POINTER(LayerRef))
+        a.batch, a.n_kv_heads, a.head_dim, a.dtype = self.B, self.Hkv, self.d, self.dcode
+        a.t_max = self.t_max
+        a.k = self._kv(k, page_table, page_size)
+        a.v = self._kv(v, page_table, page_size)
+        a.kept, a.keep_cap, a.n_keep = _ptr(self.kept), self.keep_cap, _ptr(self.n_keep)
+        a.kc, a.vc, a.cache_layer_stride, a.cap_tokens = _ptr(self.kc), _ptr(self.vc), self.kc.stride(0), self.cap_tokens
+        a.r_max, a.r_min, a.rep, a.summary_rows = _ptr(self.rmax), _ptr(self.rmin), _ptr(self.rep), self.rows
+        a.cluster_size, a.n_levels, a.fanout, a.alpha = self.s, self.n_levels, _fan(self.fanouts), self.alpha
+        a.out_n_tok = _ptr(self.n_tok)
+        _check(lib.mpc_build_clusters(C.byref(a), None, 0, C.c_void_p(_stream())))
+
+    def prefill(self, k, v, q_win, lens, page_table=None, page_size=16):
+        """Static eviction (leaders) + gathering and clustering (all layers)."""
+        self.static_evict(k, q_win, lens, page_table, page_size)
+        self.build_clusters(k, v, page_table, page_size)
+
+    # ---------------------------------------------------------- decode ----
+    def select(self, q: torch.Tensor):
+        """q: [L][B][Hq][d] queries of this step (only the leaders' are read)."""
+        lib = load()
+        refs = _refs(self.refs_lead)
+        a = SelectArgs()
+        a.struct_size = C.sizeof(SelectArgs)
+        a.n_refs = len(self.refs_lead)
+        a.refs = C.cast(refs, C.POINTER(LayerRef))
+        a.batch, a.n_q_heads, a.n_kv_heads, a.head_dim, a.dtype = self.B, self.Hq, self.Hkv, self.d, self.dcode
+        a.q, a.q_layer_stride = _ptr(q), q.stride(0)
+        a.rep, a.summary_rows, a.cap_tokens, a.n_tok = _ptr(self.rep), self.rows, self.cap_tokens, _ptr(self.n_tok)
+        a.cluster_size, a.n_levels, a.fanout = self.s, self.n_levels, _fan(self.fanouts)
+        a.level_keep_ppm = _fan(self.level_keep_ppm)
+        a.sel_cap, a.out_sel, a.out_n_sel = self.sel_cap, _ptr(self.sel), _ptr(self.n_sel)
+        _check(lib.mpc_select(C.byref(a), None, 0, C.c_void_p(_stream())))
+
+    def attn_args(self, q, k_new, v_new, advance=True, refs_list=None, out=None) -> AttnArgs:
+        refs_list = self.refs_all if refs_list is None else refs_list
+        refs = _refs(refs_list)
+        a = AttnArgs()
+        a.struct_size = C.sizeof(AttnArgs)
+        a.n_refs = len(refs_list)
+        a.refs = C.cast(refs, C.POINTER(LayerRef))
+        a.batch, a.n_q_heads, a.n_kv_heads, a.head_dim, a.dtype = self.B, self.Hq, self.Hkv, self.d, self.dcode
+        a.q, a.k_new, a.v_new = _ptr(q), _ptr(k_new), _ptr(v_new)
+        a.q_layer_stride, a.kv_new_layer_stride = q.stride(0), k_new.stride(0)
+        a.kc, a.vc, a.cache_layer_stride, a.cap_tokens = _ptr(self.kc), _ptr(self.vc), self.kc.stride(0), self.cap_tokens
+        a.sel, a.n_sel, a.sel_cap = _ptr(self.sel), _ptr(self.n_sel), self.sel_cap
+        a.r_max, a.r_min, a.rep, a.summary_rows = _ptr(self.rmax), _ptr(self.rmin), _ptr(self.rep), self.rows
+        a.cluster_size, a.n_levels, a.fanout, a.alpha = self.s, self.n_levels, _fan(self.fanouts), self.alpha
+        a.n_tok, a.advance, a.scale = _ptr(self.n_tok), int(bool(advance)), self.scale
+        out = self.out if out is None else out
+        a.out, a.out_layer_stride = _ptr(out), out.stride(0)
+        a._refs = refs  # keeps the host array alive as long as the args
+        return a
+
+    def attend(self, q, k_new, v_new, advance=True, out=None):
+        """Append + sparse attention for every layer; writes ``out``
+        ([L][B][Hq][d] float32, default ``self.out``)."""
+        lib = load()
+        a = self.attn_args(q, k_new, v_new, advance, out=out)
+        n = C.c_size_t(0)
+        _check(lib.mpc_sparse_decode_attn_workspace_size(C.byref(a), C.byref(n)))
+        ws = _ws_zero(n.value, self._ws, "attn")
+        _check(lib.mpc_sparse_decode_attn(C.byref(a), C.c_void_p(_ptr(ws)), n.value, C.c_void_p(_stream())))
+
+    def decode_step(self, q, k_new, v_new, out=None):
+        """One decode step of every layer: q [L][B][Hq][d], k_new / v_new
+        [L][B][Hkv][d] (layer index = position along dim 0)."""
+        self.select(q)
+        self.attend(q, k_new, v_new, advance=True, out=out)

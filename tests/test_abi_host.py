@@ -1,0 +1,170 @@
+"""Host-side checks of the C ABI (no GPU needed): the library loads and
+exports every entry point of include/mpcache.h, the ctypes mirrors of the
+argument structs match the C layout, and argument validation rejects bad
+input with the documented codes before any CUDA call."""
+import ctypes as C
+import os
+import re
+import subprocess
+
+import pytest
+import torch
+
+from paper_2501_06807_gb300 import build, mpcache
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "mpcache.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return mpcache.load()
+
+
+def test_exports_every_declared_symbol(lib):
+    text = open(HEADER).read()
+    names = re.findall(r"MPC_API\s+[\w\s\*]+?\b(mpc_\w+)\s*\(", text)
+    assert len(names) >= 12
+    assert set(names) == set(mpcache.ENTRY_POINTS)
+    for n in names:
+        assert hasattr(lib, n), n
+    out = subprocess.run(["nm", "-D", "--defined-only", mpcache.library_path()],
+                         capture_output=True, text=True).stdout
+    exported = set(re.findall(r"\b(mpc_\w+)\b", out))
+    assert set(names) <= exported
+    assert lib.mpc_abi_version() == 1
+
+
+def test_struct_layout_matches_c(tmp_path):
+    structs = {"mpc_layer_ref": mpcache.LayerRef, "mpc_kv_tensor": mpcache.KvTensor,
+               "mpc_static_args": mpcache.StaticArgs, "mpc_cluster_args": mpcache.ClusterArgs,
+               "mpc_select_args": mpcache.SelectArgs, "mpc_attn_args": mpcache.AttnArgs}
+    lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "mpcache.h"', 'int main(void){']
+    for cname, py in structs.items():
+        lines.append(f'printf("{cname} size %zu\\n", sizeof({cname}));')
+        for fname, _ in py._fields_:
+            lines.append(f'printf("{cname} {fname} %zu\\n", offsetof({cname}, {fname}));')
+    lines.append("return 0;}")
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines))
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)], check=True)
+    got = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split("\n")
+    for line in got:
+        if not line:
+            continue
+        cname, field, val = line.split()
+        py = structs[cname]
+        want = C.sizeof(py) if field == "size" else getattr(py, field).offset
+        assert int(val) == want, (cname, field, val, want)
+
+
+def _attn_args(**over):
+    a = mpcache.AttnArgs()
+    a.struct_size = C.sizeof(mpcache.AttnArgs)
+    refs = (mpcache.LayerRef * 2)(mpcache.LayerRef(0, 0, 1), mpcache.LayerRef(1, 0, 0))
+    a.n_refs, a.refs = 2, C.cast(refs, C.POINTER(mpcache.LayerRef))
+    a.batch, a.n_q_heads, a.n_kv_heads, a.head_dim, a.dtype = 1, 8, 2, 128, mpcache.MPC_BF16
+    a.kc = a.vc = a.q = a.k_new = a.v_new = 4096
+    a.cap_tokens, a.sel_cap, a.summary_rows = 512, 4, 64
+    a.cluster_size, a.n_levels = 16, 2
+    a.fanout[0] = 4
+    a.alpha = 0.6
+    for k, v in over.items():
+        setattr(a, k, v)
+    a._refs = refs
+    return a
+
+
+def _ws(lib, fn, a):
+    n = C.c_size_t(0)
+    rc = getattr(lib, fn)(C.byref(a), C.byref(n))
+    return rc, n.value
+
+
+def test_attn_validation(lib):
+    rc, n = _ws(lib, "mpc_sparse_decode_attn_workspace_size", _attn_args())
+    assert rc == 0 and n > 0
+    cases = [
+        (dict(struct_size=8), mpcache.MPC_ERR_INVALID_ARG),
+        (dict(head_dim=96), mpcache.MPC_ERR_BAD_SHAPE),
+        (dict(dtype=7), mpcache.MPC_ERR_INVALID_ARG),
+        (dict(n_q_heads=7), mpcache.MPC_ERR_BAD_SHAPE),
+        (dict(n_refs=0), mpcache.MPC_ERR_BAD_SHAPE),
+        (dict(cap_tokens=500), mpcache.MPC_ERR_BAD_SHAPE),
+        (dict(cluster_size=0), mpcache.MPC_ERR_BAD_SHAPE),
+        (dict(n_levels=5), mpcache.MPC_ERR_BAD_SHAPE),
+        (dict(alpha=1.5), mpcache.MPC_ERR_BAD_SHAPE),
+        (dict(kc=4100), mpcache.MPC_ERR_INVALID_ARG),
+        (dict(n_q_heads=2 * 17, n_kv_heads=2), mpcache.MPC_ERR_BAD_SHAPE),
+    ]
+    for over, code in cases:
+        rc, _ = _ws(lib, "mpc_sparse_decode_attn_workspace_size", _attn_args(**over))
+        assert rc == code, (over, rc, lib.mpc_last_error())
+        assert lib.mpc_last_error()
+    a = _attn_args()
+    a.fanout[0] = 1
+    assert _ws(lib, "mpc_sparse_decode_attn_workspace_size", a)[0] == mpcache.MPC_ERR_BAD_SHAPE
+    # the call itself rejects a missing workspace before launching anything
+    a = _attn_args()
+    a.n_tok = a.out = a.sel = a.n_sel = 8192
+    assert lib.mpc_sparse_decode_attn(C.byref(a), None, 0, None) == mpcache.MPC_ERR_WORKSPACE
+    assert lib.mpc_sparse_decode_attn(None, None, 0, None) == mpcache.MPC_ERR_INVALID_ARG
+
+
+def test_select_and_static_validation(lib):
+    s = mpcache.SelectArgs()
+    s.struct_size = C.sizeof(mpcache.SelectArgs)
+    refs = (mpcache.LayerRef * 1)(mpcache.LayerRef(0, 0, 0))
+    s.n_refs, s.refs = 1, C.cast(refs, C.POINTER(mpcache.LayerRef))
+    s.batch, s.n_q_heads, s.n_kv_heads, s.head_dim, s.dtype = 1, 4, 4, 64, mpcache.MPC_F32
+    s.rep, s.cap_tokens, s.cluster_size, s.n_levels = 4096, 256, 16, 1
+    s.summary_rows, s.sel_cap = 16, 4
+    s.level_keep_ppm[0] = 250_000
+    assert _ws(lib, "mpc_select_workspace_size", s)[0] == mpcache.MPC_ERR_INVALID_ARG  # not a leader
+    refs[0].leader = 1
+    assert _ws(lib, "mpc_select_workspace_size", s) == (0, 0)
+    s.sel_cap = 3
+    assert _ws(lib, "mpc_select_workspace_size", s)[0] == mpcache.MPC_ERR_BAD_SHAPE
+    s.sel_cap = 4
+    s.level_keep_ppm[0] = 0
+    assert _ws(lib, "mpc_select_workspace_size", s)[0] == mpcache.MPC_ERR_BAD_SHAPE
+    s.level_keep_ppm[0] = 250_000
+    s.summary_rows = 15
+    assert _ws(lib, "mpc_select_workspace_size", s)[0] == mpcache.MPC_ERR_BAD_SHAPE
+
+    a = mpcache.StaticArgs()
+    a.struct_size = C.sizeof(mpcache.StaticArgs)
+    a.n_refs, a.refs = 1, C.cast(refs, C.POINTER(mpcache.LayerRef))
+    a.batch, a.n_q_heads, a.n_kv_heads, a.head_dim, a.dtype = 2, 8, 2, 128, mpcache.MPC_BF16
+    a.t_max, a.win_rows, a.keep_cap = 32768, 4916, 8192
+    a.window_ppm, a.long_window_ppm, a.long_prompt_threshold, a.keep_ppm = 200_000, 100_000, 24576, 250_000
+    rc, n = _ws(lib, "mpc_static_evict_workspace_size", a)
+    assert rc == 0 and n == 1 * 2 * 8 * 4916 * 8
+    a.win_rows = 4915      # the longest window (T = 24576) needs 4916 rows
+    assert _ws(lib, "mpc_static_evict_workspace_size", a)[0] == mpcache.MPC_ERR_BAD_SHAPE
+    a.win_rows, a.keep_cap = 4916, 8191
+    assert _ws(lib, "mpc_static_evict_workspace_size", a)[0] == mpcache.MPC_ERR_BAD_SHAPE
+
+
+def test_summary_rows(lib):
+    assert mpcache.summary_rows(8192 + 512, 16, (8, 8)) == 544 + 68 + 9
+    assert mpcache.summary_rows(256, 16, ()) == 16
+    arr = (C.c_int32 * 4)(1, 0, 0, 0)
+    assert lib.mpc_summary_rows(256, 16, 2, arr) == mpcache.MPC_ERR_BAD_SHAPE
+
+
+def test_host_rules_match_oracle():
+    from oracle import mpcache_oracle as O
+    for t in (1, 7, 512, 1000, 2048, 24_576, 24_577, 32_768):
+        for ppm in (1, 50_000, 125_000, 200_000, 333_333, 1_000_000):
+            assert mpcache.ppm_count(t, ppm) == O.kept_count(t, ppm)
+    for m in (1, 2, 4):
+        for l in range(40):
+            assert mpcache.sharing_leader(l, m) == O.leader_of(l, m)
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    with pytest.raises(OSError):
+        mpcache.load(str(tmp_path / "nope.so"))

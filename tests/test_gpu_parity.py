@@ -1,0 +1,384 @@
+"""GPU parity of the CUDA path (through the C ABI) against the fp64 oracle.
+
+Tolerances:
+* attention outputs: max |o - o_ref| / max |o_ref| per output vector
+  <= 1e-5 (fp32 KV) and <= 2e-3 (bf16 KV);
+* summaries: r_max / r_min bit-exact, rep within fp32 rounding;
+* cache contents: bit-exact;
+* scores and index sets: within bands derived from the kernels' fp32
+  arithmetic (``static_band`` / ``select_band``); an index set must equal
+  the oracle's unless the oracle's margin at a cut is inside the band (a tie
+  at the kernel's precision), in which case only its validity is checked.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import mpcache_oracle as O
+from paper_2501_06807_gb300 import synth
+from tests import helpers as H
+
+pytestmark = pytest.mark.gpu
+U = 2.0 ** -24
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2501_06807_gb300 import build
+    build.build()
+
+
+def _tol(dtype):
+    return 1e-5 if dtype == torch.float32 else 2e-3
+
+
+def static_band(qw, K, scale, w, G):
+    """Relative error bound of the GPU's accumulated scores: fp32 dot products
+    over d channels (|error| <= d u sum|q k|), the log2 rescale, two ex2.approx
+    per probability and the row / column sums."""
+    A = (np.abs(qw.reshape(-1, qw.shape[-1])) @ np.abs(K).T).max()
+    d, T = K.shape[1], K.shape[0]
+    return 2 * scale * d * U * A + 3 * U * scale * 1.4427 * A + 4 * 2.0 ** -22 + (T / 64 + w * G / 64 + 64) * U
+
+
+def select_band(q_group, levels):
+    """Absolute error bound of the GPU's cluster similarities (fp32 q-sum,
+    fp32 rep, fp32 dot over d channels), doubled for a pair of candidates."""
+    qa = np.abs(q_group).sum(0)
+    qs = np.abs(q_group.sum(0))
+    d, G = q_group.shape[1], q_group.shape[0]
+    b = 0.0
+    for lev in levels:
+        if len(lev.r_max):
+            mag = np.abs(lev.r_max) + np.abs(lev.r_min)
+            b = max(b, float(((d + 4) * U * (mag @ qs) + G * U * (mag @ qa)).max()))
+    return 2 * b + 1e-30
+
+
+def unique_selection(trace, band):
+    for cand, sim, k in trace:
+        if 0 < k < len(cand):
+            srt = np.sort(sim)[::-1]
+            if srt[k - 1] - srt[k] <= band:
+                return False
+    return True
+
+
+# ------------------------------------------------ attention in isolation ----
+
+ATTN_CASES = [
+    # dtype, d, Hq, Hkv, s, fanouts, n_keep, steps
+    (torch.float32, 64, 2, 1, 16, (), 83, 20),
+    (torch.float32, 128, 8, 1, 32, (2,), 150, 36),
+    (torch.bfloat16, 128, 4, 1, 16, (4,), 200, 35),
+    (torch.bfloat16, 128, 8, 2, 16, (8, 8), 600, 18),
+    (torch.bfloat16, 64, 2, 2, 8, (3,), 77, 17),
+    (torch.bfloat16, 128, 16, 1, 4, (2, 2), 61, 9),
+    (torch.bfloat16, 64, 1, 1, 1, (4,), 40, 5),
+    (torch.bfloat16, 128, 4, 2, 16, (4,), 5, 13),   # starts with no full cluster
+]
+
+
+@pytest.mark.parametrize("dtype,d,Hq,Hkv,s,fan,N,E", ATTN_CASES)
+def test_attention_cache_and_seal(dtype, d, Hq, Hkv, s, fan, N, E):
+    g = torch.Generator().manual_seed(N * 7 + d)
+    L, B, T = 4, 2, N + 37
+    G = Hq // Hkv
+    keep = tuple([O.PPM] * (1 + len(fan)))
+    eng = H.make_engine(synth.Workload("t", L, B, Hq, Hkv, d, "f32" if dtype == torch.float32 else "bf16",
+                                       T, T, O.PPM, s, fan, keep, 2, E, "iid"), E)
+    K = torch.randn((L, B, Hkv, T, d), generator=g).to(dtype)
+    V = torch.randn((L, B, Hkv, T, d), generator=g).to(dtype)
+    kept = torch.zeros((eng.n_groups, B, Hkv, N), dtype=torch.int32)
+    for idx in np.ndindex(eng.n_groups, B, Hkv):
+        kept[idx] = torch.sort(torch.randperm(T, generator=g)[:N]).values.to(torch.int32)
+    eng.kept[..., :N] = kept.cuda()
+    eng.n_keep.fill_(N)
+    eng.build_clusters(K.cuda(), V.cuda())
+    torch.cuda.synchronize()
+    assert eng.n_tok.tolist() == [N] * B
+    # cache rows are the kept rows, bit-exact
+    caches = {}
+    for l in range(L):
+        grp = eng.group_of[l]
+        for b in range(B):
+            for h in range(Hkv):
+                ids = kept[grp, b, h].long()
+                got_k = H.unswizzle(eng.kc[l, b, h, :N].cpu())
+                got_v = H.unswizzle(eng.vc[l, b, h, :N].cpu())
+                assert torch.equal(got_k, K[l, b, h, ids]) and torch.equal(got_v, V[l, b, h, ids])
+                caches[(l, b, h)] = [K[l, b, h, ids].double().numpy(), V[l, b, h, ids].double().numpy()]
+
+    def check_pyramid(n_tok):
+        for l in eng.leaders:
+            grp = eng.group_of[l]
+            for b in range(B):
+                for h in range(Hkv):
+                    lev = O.cluster_pyramid(caches[(l, b, h)][0][:n_tok], s, fan, 0.6)
+                    for li, lv in enumerate(lev):
+                        n = len(lv.members)
+                        rows = slice(_off(eng, li), _off(eng, li) + n)
+                        assert np.array_equal(eng.rmax[grp, b, h, rows].cpu().double().numpy(), lv.r_max)
+                        assert np.array_equal(eng.rmin[grp, b, h, rows].cpu().double().numpy(), lv.r_min)
+                        rep = eng.rep[grp, b, h, rows].cpu().double().numpy()
+                        assert np.allclose(rep, lv.rep, rtol=4e-7, atol=4e-7 * np.abs(lv.rep).max(initial=0))
+
+    check_pyramid(N)
+    scale = 1 / math.sqrt(d)
+    for e in range(E):
+        n_tok = N + e
+        C1 = n_tok // s
+        k = int(torch.randint(0, min(C1, eng.sel_cap) + 1, (1,), generator=g)) if e % 5 else min(C1, eng.sel_cap)
+        sel = torch.full((eng.n_groups, B, Hkv, eng.sel_cap), -1, dtype=torch.int32)
+        for idx in np.ndindex(eng.n_groups, B, Hkv):
+            sel[idx][:k] = torch.sort(torch.randperm(C1, generator=g)[:k]).values.to(torch.int32)
+        eng.sel.copy_(sel.cuda())
+        eng.n_sel.fill_(k)
+        q = torch.randn((L, B, Hq, d), generator=g).to(dtype)
+        kn = torch.randn((L, B, Hkv, d), generator=g).to(dtype)
+        vn = torch.randn((L, B, Hkv, d), generator=g).to(dtype)
+        eng.attend(q.cuda(), kn.cuda(), vn.cuda(), advance=True)
+        out = eng.out.cpu().double().numpy()
+        for l in range(L):
+            grp = eng.group_of[l]
+            for b in range(B):
+                for h in range(Hkv):
+                    c = caches[(l, b, h)]
+                    c[0] = np.vstack([c[0], kn[l, b, h].double().numpy()[None]])
+                    c[1] = np.vstack([c[1], vn[l, b, h].double().numpy()[None]])
+                    toks = O.attended_tokens(n_tok, s, sel[grp, b, h, :k].numpy())
+                    for gg in range(G):
+                        ref = O.sparse_attention(q[l, b, h * G + gg].double().numpy(), c[0][toks], c[1][toks], scale)
+                        err = H.rel_err(out[l, b, h * G + gg], ref)
+                        assert err <= _tol(dtype), (e, l, b, h, gg, err)
+        if (n_tok + 1) % s == 0:
+            check_pyramid(n_tok + 1)
+    torch.cuda.synchronize()
+    assert eng.n_tok.tolist() == [N + E] * B
+    # appended rows landed in the cache
+    for l in range(L):
+        got = H.unswizzle(eng.kc[l, 0, 0, :N + E].cpu()).double().numpy()
+        assert np.array_equal(got, caches[(l, 0, 0)][0])
+    from paper_2501_06807_gb300 import mpcache
+    assert mpcache.device_status() == 0
+
+
+def _off(eng, level):
+    cap = eng.cap_tokens // eng.s
+    off = 0
+    for li in range(level):
+        off += cap
+        cap = -(-cap // eng.fanouts[li])
+    return off
+
+
+# ------------------------------------------------- selection in isolation ----
+
+SELECT_CASES = [
+    # dtype, d, Hq, Hkv, s, fanouts, keep ppm (finest first), n_tok
+    (torch.float32, 64, 3, 3, 16, (), (250_000,), 16 * 37 + 5),
+    (torch.bfloat16, 128, 4, 4, 16, (4,), (125_000, 500_000), 1024),
+    (torch.bfloat16, 128, 32, 8, 16, (8, 8), (50_000, 250_000, 500_000), 8192 + 7),
+    (torch.bfloat16, 128, 8, 2, 16, (8,), (100_000, 500_000), 2048 + 15),
+    (torch.bfloat16, 64, 2, 1, 1, (), (30_000,), 3000),       # token-wise (s = 1)
+    (torch.float32, 128, 2, 1, 4, (3, 2), (200_000, 400_000, 600_000), 997),
+    (torch.bfloat16, 128, 4, 1, 16, (4,), (1_000_000, 1_000_000), 320),  # keep all
+]
+
+
+@pytest.mark.parametrize("dtype,d,Hq,Hkv,s,fan,keep,N", SELECT_CASES)
+def test_selection(dtype, d, Hq, Hkv, s, fan, keep, N):
+    g = torch.Generator().manual_seed(N + d)
+    L, B = 1, 2
+    G = Hq // Hkv
+    eng = H.make_engine(synth.Workload("t", L, B, Hq, Hkv, d, "f32" if dtype == torch.float32 else "bf16",
+                                       N, N, O.PPM, s, fan, keep, 1, 4, "iid"), 4)
+    K = (torch.randn((L, B, Hkv, N, d), generator=g) * torch.rand((1, 1, Hkv, 1, d), generator=g) * 3).to(dtype)
+    eng.kept[..., :N] = torch.arange(N, dtype=torch.int32).cuda()
+    eng.n_keep.fill_(N)
+    eng.build_clusters(K.cuda(), K.cuda())
+    ties = 0
+    for rep_i in range(3):
+        q = (torch.randn((L, B, Hq, d), generator=g) * 2).to(dtype)
+        eng.select(q.cuda())
+        sel = eng.sel.cpu().numpy()
+        n_sel = eng.n_sel.cpu().numpy()
+        for b in range(B):
+            for h in range(Hkv):
+                levels = O.cluster_pyramid(K[0, b, h].double().numpy(), s, fan, 0.6)
+                qg = q[0, b, h * G:(h + 1) * G].double().numpy()
+                tr = []
+                ref = O.hierarchical_select(qg, levels, fan, keep, trace=tr)
+                got = sel[0, b, h, :n_sel[b]]
+                assert n_sel[b] == len(ref)
+                assert (sel[0, b, h, n_sel[b]:] == -1).all()
+                if unique_selection(tr, select_band(qg, levels)):
+                    assert np.array_equal(got, ref), (b, h)
+                else:
+                    ties += 1
+                    assert np.all(np.diff(got) > 0) and got.min(initial=0) >= 0
+                    assert got.max(initial=-1) < N // s
+    assert ties <= 2
+
+
+# ----------------------------------------------- static eviction alone ----
+
+STATIC_CASES = [
+    # dtype, d, Hq, Hkv, lens, keep_ppm, paged
+    (torch.float32, 64, 4, 4, (512,), 500_000, False),
+    (torch.bfloat16, 128, 8, 2, (1000,), 250_000, False),
+    (torch.bfloat16, 64, 2, 1, (129, 300, 64), 500_000, False),
+    (torch.bfloat16, 128, 4, 4, (777, 1500), 125_000, True),
+    (torch.float32, 128, 2, 2, (33,), 1_000_000, False),
+    (torch.bfloat16, 128, 4, 1, (1,), 500_000, False),
+]
+
+
+@pytest.mark.parametrize("dtype,d,Hq,Hkv,lens,keep,paged", STATIC_CASES)
+def test_static_eviction(dtype, d, Hq, Hkv, lens, keep, paged):
+    g = torch.Generator().manual_seed(sum(lens) + d)
+    B, T = len(lens), max(lens)
+    G = Hq // Hkv
+    w = synth.Workload("t", 1, B, Hq, Hkv, d, "f32" if dtype == torch.float32 else "bf16", T, min(lens),
+                       keep, 16, (), (O.PPM,), 1, 1, "iid", paged=paged)
+    eng = H.make_engine(w, 1)
+    R = eng.win_rows
+    K = torch.zeros((1, B, Hkv, T, d))
+    Q = torch.zeros((1, B, Hq, R, d))
+    for b, t in enumerate(lens):
+        K[0, b, :, :t] = torch.randn((Hkv, t, d), generator=g) * 1.5
+        Q[0, b, :, R - min(R, t):] = torch.randn((Hq, min(R, t), d), generator=g) * 1.5
+    K, Q = K.to(dtype), Q.to(dtype)
+    lens_t = torch.tensor(lens, dtype=torch.int32)
+    if paged:
+        P = 16
+        n_pages = [(t + P - 1) // P for t in lens]
+        perm = torch.randperm(sum(n_pages), generator=g).to(torch.int32)
+        pt = torch.full((B, (T + P - 1) // P), -1, dtype=torch.int32)
+        pool = torch.zeros((1, sum(n_pages), Hkv, P, d), dtype=dtype)
+        o = 0
+        for b, t in enumerate(lens):
+            pt[b, :n_pages[b]] = perm[o:o + n_pages[b]]
+            o += n_pages[b]
+            for j in range(n_pages[b]):
+                seg = K[0, b, :, j * P:(j + 1) * P]
+                pool[0, int(pt[b, j]), :, :seg.shape[1]] = seg
+        eng.static_evict(pool.cuda(), Q.cuda(), lens_t.cuda(), pt.cuda(), P)
+    else:
+        eng.static_evict(K.cuda(), Q.cuda(), lens_t.cuda())
+    scores = eng.scores.cpu().double().numpy()
+    kept = eng.kept.cpu().numpy()
+    assert eng.n_keep.cpu().tolist() == [O.kept_count(t, keep) for t in lens]
+    for b, t in enumerate(lens):
+        wl = O.window_length(t)
+        for h in range(Hkv):
+            qw = Q[0, b, h * G:(h + 1) * G, R - wl:].double().numpy()
+            kk = K[0, b, h, :t].double().numpy()
+            ref = O.accumulated_attention(qw, kk, 1 / math.sqrt(d))
+            tau = static_band(qw, kk, 1 / math.sqrt(d), wl, G)
+            got = scores[0, b, h, :t]
+            assert np.all(np.abs(got - ref) <= tau * np.maximum(ref, 1e-30) + 1e-30), (b, h, tau)
+            nk = O.kept_count(t, keep)
+            ref_kept = O.static_evict(ref, nk)
+            assert np.all(kept[0, b, h, nk:] == -1)
+            H.set_parity(kept[0, b, h, :nk], ref_kept, lambda ids: ref[ids], nk,
+                         band=2 * tau * ref[ref_kept].min())
+
+
+# ------------------------------------------------------- full pipeline ----
+
+def _pipeline(w: synth.Workload, E: int, layers, max_skip=0.05, device="cpu"):
+    R = H.window_rows_for(w)
+    x = synth.generate(w, R, device=device, decode_steps=E)
+    xc = H.to_cuda(x)
+    eng = H.make_engine(w, E)
+    lens = x.prompt_lens.cuda()
+    pt = xc.page_table.cuda() if xc.page_table is not None else None
+    eng.prefill(xc.k, xc.v, xc.q_win, lens, pt, w.page_size)
+    torch.cuda.synchronize()
+    g_scores, g_kept = eng.scores.cpu().double().numpy(), eng.kept.cpu().numpy()
+    sels, outs = [], []
+    for e in range(E):
+        eng.decode_step(xc.q[e], xc.k_new[e], xc.v_new[e])
+        sels.append(eng.sel.cpu().numpy().copy())
+        outs.append(eng.out.cpu().double().numpy().copy())
+    res = H.oracle_run(x, E, layers)
+    G = w.group
+    diverged = set()   # (l, b, h) whose kept set is a tie-variant
+    taus = {}
+    units = 0
+    for l in layers:
+        lead = O.leader_of(l, w.share_every)
+        grp = eng.group_of[l]
+        for b in range(w.batch):
+            T = int(x.prompt_lens[b])
+            for h in range(w.n_kv_heads):
+                if lead == l:
+                    ref = res.scores[(l, b, h)]
+                    kk, _ = x.dense_kv(l, b)
+                    qw = x.q_win[l, b, h * G:(h + 1) * G, R - O.window_length(T):].double().numpy()
+                    tau = static_band(qw, kk[h].double().numpy(), 1 / math.sqrt(w.head_dim),
+                                      O.window_length(T), G)
+                    got = g_scores[grp, b, h, :T]
+                    assert np.all(np.abs(got - ref) <= tau * ref + 1e-30), (l, b, h)
+                    taus[(l, b, h)] = tau
+                nk = len(res.kept[(l, b, h)])
+                gk = g_kept[grp, b, h, :nk]
+                if not np.array_equal(gk, res.kept[(l, b, h)]):
+                    sc = res.scores[(lead, b, h)]
+                    H.set_parity(gk, res.kept[(l, b, h)], lambda ids: sc[ids], nk,
+                                 band=2 * taus[(lead, b, h)] * sc[res.kept[(l, b, h)]].min())
+                    diverged.add((l, b, h))
+    skipped = 0
+    for e in range(E):
+        for l in layers:
+            lead = O.leader_of(l, w.share_every)
+            grp = eng.group_of[l]
+            for b in range(w.batch):
+                n_sel = None
+                for h in range(w.n_kv_heads):
+                    units += 1
+                    if (lead, b, h) in diverged or (l, b, h) in diverged:
+                        skipped += 1
+                        continue
+                    ref_sel = res.selected[(e, l, b, h)]
+                    got_sel = sels[e][grp, b, h, :len(ref_sel)]
+                    if not np.array_equal(got_sel, ref_sel):
+                        levels = res.levels[(e, lead, b, h)]
+                        qg = x.q[e, lead, b, h * G:(h + 1) * G].double().numpy()
+                        tr = []
+                        O.hierarchical_select(qg, levels, w.fanouts, w.level_keep_ppm, trace=tr)
+                        assert not unique_selection(tr, select_band(qg, levels)), (e, l, b, h, got_sel, ref_sel)
+                        skipped += 1
+                        continue
+                    for gg in range(G):
+                        err = H.rel_err(outs[e][l, b, h * G + gg], res.out[(e, l, b)][h * G + gg])
+                        assert err <= (1e-5 if w.dtype == "f32" else 2e-3), (e, l, b, h, gg, err)
+    assert skipped <= max_skip * units, (skipped, units)
+    from paper_2501_06807_gb300 import mpcache
+    assert mpcache.device_status() == 0
+    return eng, x, res
+
+
+def test_pipeline_c1_full():
+    """The GPT-2-small workload exactly as configured: 12 heads, 512 tokens,
+    fp32, 8 decode steps."""
+    _pipeline(synth.C1, synth.C1.decode_steps, [0], max_skip=0.0)
+
+
+def test_pipeline_llama2_shape_reduced():
+    w = synth.C2.replace(n_layers=5, prompt_len=1024, prompt_len_min=1024, n_q_heads=8, n_kv_heads=8)
+    _pipeline(w, 21, list(range(5)))
+
+
+def test_pipeline_gqa_three_levels_needles():
+    w = synth.C5.replace(n_layers=3, prompt_len=4096, prompt_len_min=4096, n_q_heads=8, n_kv_heads=2,
+                         level_keep_ppm=(100_000, 250_000, 500_000))
+    _pipeline(w, 18, [0, 1, 2])
+
+
+def test_pipeline_paged_ragged_batch():
+    w = synth.C4.replace(n_layers=3, batch=3, prompt_len=700, prompt_len_min=300, n_q_heads=4, n_kv_heads=4)
+    _pipeline(w, 10, [0, 1, 2])
