@@ -195,7 +195,11 @@ def test_selection(dtype, d, Hq, Hkv, s, fan, keep, N):
     G = Hq // Hkv
     eng = H.make_engine(synth.Workload("t", L, B, Hq, Hkv, d, "f32" if dtype == torch.float32 else "bf16",
                                        N, N, O.PPM, s, fan, keep, 1, 4, "iid"), 4)
-    K = (torch.randn((L, B, Hkv, N, d), generator=g) * torch.rand((1, 1, Hkv, 1, d), generator=g) * 3).to(dtype)
+    # keys with token-wise locality (a slow drift per channel), the structure
+    # clustering relies on; iid keys make coarse summaries indistinguishable
+    drift = torch.cumsum(torch.randn((L, B, Hkv, N, d), generator=g) * 0.15, dim=3)
+    K = ((torch.randn((L, B, Hkv, N, d), generator=g) + drift)
+         * torch.rand((1, 1, Hkv, 1, d), generator=g) * 3).to(dtype)
     eng.kept[..., :N] = torch.arange(N, dtype=torch.int32).cuda()
     eng.n_keep.fill_(N)
     eng.build_clusters(K.cuda(), K.cuda())
@@ -216,11 +220,11 @@ def test_selection(dtype, d, Hq, Hkv, s, fan, keep, N):
                 assert (sel[0, b, h, n_sel[b]:] == -1).all()
                 if unique_selection(tr, select_band(qg, levels)):
                     assert np.array_equal(got, ref), (b, h)
-                else:
+                elif not np.array_equal(got, ref):
                     ties += 1
                     assert np.all(np.diff(got) > 0) and got.min(initial=0) >= 0
                     assert got.max(initial=-1) < N // s
-    assert ties <= 2
+    assert ties <= 1
 
 
 # ----------------------------------------------- static eviction alone ----
