@@ -261,6 +261,25 @@ MPC_API int mpc_select(const mpc_select_args* args, void* workspace,
 MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace,
                                    size_t workspace_bytes, void* stream);
 
+/* ---- mpc_sparse_decode_attn_static_scratch --------------------------------
+ * The same decode step as mpc_sparse_decode_attn, for callers that cannot
+ * allocate device memory (a runtime that forbids raw cudaMalloc, a plugin
+ * that only receives fixed input/output buffers, a path that must not
+ * allocate after start-up).  The paper has no counterpart: it is a property
+ * of this library's interface, not of the method.
+ * - Scratch is a 4 MiB array inside the library's device image, held by every
+ *   GPU that loads the library until the process exits.  A call whose
+ *   workspace (mpc_sparse_decode_attn_workspace_size) exceeds 4 MiB is
+ *   rejected with MPC_ERR_WORKSPACE and nothing is launched.
+ * - The first call on each device looks up the array's device address (with
+ *   that device current); make that first call before any stream capture.
+ * - Each call clears the part of the array it uses (an asynchronous memset
+ *   on `stream`) and then runs the regular kernels.  Every call shares the
+ *   one array: calls that overlap on the GPU (different streams, no
+ *   ordering between them) race and corrupt each other's results.
+ * - Allocates nothing (no cudaMalloc / cudaFree). */
+MPC_API int mpc_sparse_decode_attn_static_scratch(const mpc_attn_args* args, void* stream);
+
 /* Rows of the summary pyramid for a cache of cap_tokens rows (the sum of the
  * level capacities above), or a negative MPC_ERR_* code. */
 MPC_API int64_t mpc_summary_rows(int32_t cap_tokens, int32_t cluster_size,

@@ -345,6 +345,9 @@ int cuda_fail(cudaError_t e, const char* what) {
 }
 
 }  // namespace
+
+int set_error(int code, const char* msg) { return fail(code, "%s", msg); }
+
 }  // namespace mpc
 
 using namespace mpc;

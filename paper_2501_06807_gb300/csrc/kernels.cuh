@@ -105,6 +105,9 @@ cudaError_t launch_clusters(const ClusterParams& p, int dtype, int D, int n_unit
 cudaError_t launch_static(const StaticParams& p, int dtype, int D, cudaStream_t st);
 int static_tile_smem(int D);
 
+// Records `msg` as this thread's last error (mpc_last_error) and returns code.
+int set_error(int code, const char* msg);
+
 // Device status word of each translation unit: read it and clear it.
 int take_status_attn();
 int take_status_select();

@@ -1,0 +1,68 @@
+// Decode attention for callers that cannot allocate device memory.
+//
+// Some callers cannot call cudaMalloc at all: code that runs inside a
+// memory-pool-managed runtime that forbids raw allocations, plugins handed
+// only fixed input/output buffers by their host, or paths that must not
+// allocate after start-up (allocation can block or fail).  The regular
+// mpc_sparse_decode_attn asks its caller for a workspace; this entry point
+// instead uses a fixed scratch array that lives in the library's own device
+// image, so the caller passes only inputs and outputs.
+//
+// The array is a file-scope __device__ variable.  Host code cannot use its
+// name as a device address, so the address is looked up with
+// cudaGetSymbolAddress, once per device, the first time the entry point runs
+// on that device (with that device current).
+#include <mutex>
+
+#include "kernels.cuh"
+
+namespace mpc {
+namespace {
+
+constexpr size_t kStaticScratchBytes = size_t(4) << 20;  // 4 MiB per device
+
+static __device__ __align__(256) unsigned char g_attn_scratch[kStaticScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+void* g_scratch_addr[kMaxDevices] = {};
+
+// Device address of g_attn_scratch on the current device.
+int scratch_address(void** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return set_error(MPC_ERR_CUDA, cudaGetErrorString(e));
+  if (dev < 0 || dev >= kMaxDevices) return set_error(MPC_ERR_INVALID_ARG, "device ordinal out of range");
+  std::lock_guard<std::mutex> lk(g_scratch_mu);
+  if (g_scratch_addr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_attn_scratch);
+    if (e != cudaSuccess || p == nullptr)
+      return set_error(MPC_ERR_CUDA, "cudaGetSymbolAddress of the static scratch array failed");
+    g_scratch_addr[dev] = p;
+  }
+  *out = g_scratch_addr[dev];
+  return MPC_OK;
+}
+
+}  // namespace
+}  // namespace mpc
+
+extern "C" MPC_API int mpc_sparse_decode_attn_static_scratch(const mpc_attn_args* args, void* stream) {
+  using namespace mpc;
+  size_t need = 0;
+  int rc = mpc_sparse_decode_attn_workspace_size(args, &need);
+  if (rc != MPC_OK) return rc;
+  if (need > kStaticScratchBytes)
+    return set_error(MPC_ERR_WORKSPACE,
+                     "this call needs more scratch than the 4 MiB static array holds; "
+                     "use mpc_sparse_decode_attn with a caller workspace");
+  void* ws = nullptr;
+  rc = scratch_address(&ws);
+  if (rc != MPC_OK) return rc;
+  // the split counters must start at zero; the array keeps the previous
+  // call's contents, so clear the part this call uses
+  const cudaError_t e = cudaMemsetAsync(ws, 0, need, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return set_error(MPC_ERR_CUDA, cudaGetErrorString(e));
+  return mpc_sparse_decode_attn(args, ws, need, stream);
+}

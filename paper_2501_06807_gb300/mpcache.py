@@ -90,7 +90,8 @@ class AttnArgs(C.Structure):
 ENTRY_POINTS = ("mpc_static_evict_workspace_size", "mpc_build_clusters_workspace_size",
                 "mpc_select_workspace_size", "mpc_sparse_decode_attn_workspace_size",
                 "mpc_static_evict", "mpc_build_clusters", "mpc_select", "mpc_sparse_decode_attn",
-                "mpc_summary_rows", "mpc_last_error", "mpc_device_status", "mpc_abi_version")
+                "mpc_summary_rows", "mpc_last_error", "mpc_device_status", "mpc_abi_version",
+                "mpc_sparse_decode_attn_static_scratch")
 
 _LIB = None
 
@@ -121,6 +122,8 @@ def load(path: Optional[str] = None) -> C.CDLL:
     lib.mpc_device_status.restype = C.c_int
     lib.mpc_device_status.argtypes = [C.POINTER(C.c_int)]
     lib.mpc_abi_version.restype = C.c_int
+    lib.mpc_sparse_decode_attn_static_scratch.restype = C.c_int
+    lib.mpc_sparse_decode_attn_static_scratch.argtypes = [C.c_void_p, C.c_void_p]
     if path is None:
         _LIB = lib
     return lib
