@@ -265,7 +265,16 @@ def run_ours(args, rank, world, dist):
     dec_bytes = kv_bytes + io_bytes
     decode_gbs = dec_bytes / (decode_ms / 1e3) / 1e9
     dominant_static = static_ms >= decode_ms
-    if dominant_static:
+    tensor_path = w.dtype == "bf16" and not w.paged
+    if dominant_static and tensor_path:
+        # tcgen05 score passes; the kernel runs inside a long step, so the
+        # sustained bf16 figure is the denominator
+        peak_t = pk.get("bf16_tflops_sustained", pk["bf16_tflops"])
+        roof = {"kernel": "mpc_static_evict (score_tc_kernel pass 0 + pass 1 + budget)", "bound": "tensor",
+                "achieved": round(static_tflops, 3), "peak": peak_t, "unit": "TFLOP/s",
+                "frac": round(static_tflops / peak_t, 4), "traffic": None,
+                "peak_source": pk_kind + " bf16_tflops_sustained"}
+    elif dominant_static:
         roof = {"kernel": "mpc_static_evict (rowstats + colsum + budget)", "bound": "alu",
                 "achieved": round(static_tflops, 3), "peak": round(FFMA_PEAK_TFLOPS, 1), "unit": "TFLOP/s",
                 "frac": round(static_tflops / FFMA_PEAK_TFLOPS, 4), "traffic": None,
@@ -286,6 +295,7 @@ def run_ours(args, rank, world, dist):
                    "l2": "inputs larger than L2 (prompt KV %.1f GB per step)" % (
                        (x.k.numel() + x.v.numel()) * x.k.element_size() / 1e9)},
         "gpu_launches": args.steps * (3 + 1 + (1 if len(w.fanouts) else 0) + 2 * E),
+        "static_scoring_path": "tcgen05" if tensor_path else "simt",
         "phases_ms": {"static_evict": static_ms, "build_clusters": build_ms, "decode_all_steps": decode_ms},
         "decode_step_us": decode_ms / E * 1e3,
         "decode": {"bytes_per_step": dec_bytes / E, "achieved_gbs": round(decode_gbs, 1),

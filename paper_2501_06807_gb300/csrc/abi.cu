@@ -122,6 +122,9 @@ int validate_static(const mpc_static_args* a, StaticParams* p) {
   if (a->keep_cap < kb) return fail(MPC_ERR_BAD_SHAPE, "keep_cap %d < %d kept tokens at t_max", a->keep_cap, kb);
   if (a->scale < 0.f || !std::isfinite(a->scale)) return fail(MPC_ERR_BAD_SHAPE, "scale must be finite and >= 0");
   const mpc_kv_tensor& k = a->k;
+  if (a->dtype == MPC_BF16 && k.page_table == nullptr &&
+      (!aligned16(a->q_win) || !aligned16(k.data) || (a->q_win_layer_stride * 2) % 16 || (k.layer_stride * 2) % 16))
+    return fail(MPC_ERR_INVALID_ARG, "bf16 q_win / k and their layer strides must be 16-byte aligned");
   if (k.page_table != nullptr && (k.page_size < 1 || k.max_pages < 1 ||
                                   (int64_t)k.page_size * k.max_pages < a->t_max))
     return fail(MPC_ERR_BAD_SHAPE, "paged keys: page_size * max_pages must cover t_max");
@@ -155,7 +158,11 @@ int validate_static(const mpc_static_args* a, StaticParams* p) {
   return MPC_OK;
 }
 
-size_t static_ws(const StaticParams& p) { return (size_t)p.n_refs * p.B * p.Hq * p.win_rows * sizeof(float2); }
+// Row statistics (m, 1/l) of every window row, plus 1 KB so that a 128-row
+// bulk read of the last rows stays inside the workspace.
+size_t static_ws(const StaticParams& p) {
+  return (size_t)p.n_refs * p.B * p.Hq * p.win_rows * sizeof(float2) + 1024;
+}
 
 // ------------------------------------------------------------ clusters ----
 int validate_clusters(const mpc_cluster_args* a, ClusterParams* p) {
@@ -370,7 +377,8 @@ MPC_API int mpc_device_status(int* flags) {
   if (flags == nullptr) return fail(MPC_ERR_INVALID_ARG, "flags is NULL");
   const cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
-  const int parts[4] = {take_status_attn(), take_status_select(), take_status_clusters(), take_status_static()};
+  const int parts[5] = {take_status_attn(), take_status_select(), take_status_clusters(), take_status_static(),
+                        take_status_score_tc()};
   int v = 0;
   for (int x : parts) {
     if (x < 0) return fail(MPC_ERR_CUDA, "reading the device status word failed");
@@ -397,7 +405,9 @@ MPC_API int mpc_static_evict(const mpc_static_args* args, void* workspace, size_
   if (workspace == nullptr || workspace_bytes < need)
     return fail(MPC_ERR_WORKSPACE, "workspace of %zu bytes needed", need);
   p.stats = static_cast<float2*>(workspace);
-  const cudaError_t e = launch_static(p, args->dtype, args->head_dim, static_cast<cudaStream_t>(stream));
+  int span = 0;
+  for (int i = 0; i < args->n_refs; ++i) span = args->refs[i].layer + 1 > span ? args->refs[i].layer + 1 : span;
+  const cudaError_t e = launch_static(p, args->dtype, args->head_dim, span, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "mpc_static_evict launch");
   return ok();
 }

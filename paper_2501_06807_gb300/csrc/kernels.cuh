@@ -1,6 +1,8 @@
 // Kernel parameter blocks and launchers of the MPCache library.
 #pragma once
 
+#include <cuda.h>
+
 #include "common.cuh"
 
 namespace mpc {
@@ -70,6 +72,23 @@ struct StaticParams {
   float2* stats;      // [ref][b][Hq][win_rows]: (m, 1 / l)
 };
 
+// Window scoring on tcgen05 (bf16 queries and dense keys).
+struct ScoreTcParams {
+  CUtensorMap map_q;  // [layer][B*Hq*win_rows][d], 128 x 64 boxes, 128B swizzle
+  CUtensorMap map_k;  // [layer][B*Hkv*t_max][d]
+  RefTable refs;
+  int n_refs, B, Hq, Hkv, G, t_max, win_rows;
+  const int* lens;
+  const void* q_win;
+  int64_t qw_ls;
+  const void* k;
+  int64_t k_ls;
+  int window_ppm, long_window_ppm, long_threshold;
+  float scale_log2;
+  float* scores;
+  float2* stats;
+};
+
 struct KvSrc {
   const void* data;
   int64_t layer_stride;
@@ -102,7 +121,8 @@ cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cu
 int select_smem_bytes(int D, int max_cand);
 cudaError_t launch_clusters(const ClusterParams& p, int dtype, int D, int n_units, int groups_x,
                             bool any_leader, cudaStream_t st);
-cudaError_t launch_static(const StaticParams& p, int dtype, int D, cudaStream_t st);
+cudaError_t launch_static(const StaticParams& p, int dtype, int D, int n_layer_span, cudaStream_t st);
+cudaError_t launch_score_tc(ScoreTcParams& p, int D, int n_layer_span, cudaStream_t st);
 int static_tile_smem(int D);
 
 // Records `msg` as this thread's last error (mpc_last_error) and returns code.
@@ -113,5 +133,6 @@ int take_status_attn();
 int take_status_select();
 int take_status_clusters();
 int take_status_static();
+int take_status_score_tc();
 
 }  // namespace mpc

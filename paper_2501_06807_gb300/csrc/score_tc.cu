@@ -1,0 +1,442 @@
+// Window scoring of look-once static eviction on the 5th-generation tensor
+// cores (Sec. 3.2; Alg. 2 Step 1): the two passes of the accumulated window
+// attention for bf16 queries and dense keys.
+//
+//   pass 0 (row statistics): one CTA per (ref, sequence, query head, 128
+//     window rows).  A = the 128 query rows (fixed), B = 128-key tiles
+//     streamed over every key a row can see.  S = A B^T lands in TMEM with
+//     one window row per TMEM lane, so each epilogue thread owns a row and
+//     keeps its online max m and sum l of 2^(s - m) without any cross-thread
+//     reduction.
+//   pass 1 (column sums): one CTA per (ref, sequence, kv head, 128 keys).
+//     A = the 128 key rows (fixed), B = 128-row tiles of window queries of
+//     every query head of the GQA group.  S^T = A B^T puts one key per TMEM
+//     lane, so each thread sums 2^(s_ij - m_i) / l_i over the rows i in its
+//     own registers, in a fixed order (deterministic scores).
+//
+// Roles: warp 0 issues TMA tile loads (128B-swizzled, K-major boxes of
+// 128 rows x 64 channels), warp 1 allocates TMEM and issues tcgen05.mma
+// (M = N = 128, K = 16, bf16 in, fp32 accumulate) into one of two 128-column
+// accumulators, warps 2-5 drain the other accumulator with tcgen05.ld.
+// Every wait is bounded; a timeout sets the device status word and an abort
+// flag that stops the other roles, and TMEM is always released.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "kernels.cuh"
+
+namespace mpc {
+namespace {
+
+constexpr int kTcThreads = 192;
+constexpr int kStagesTc = 2;
+constexpr int kBoxBytes = 128 * 128;  // 128 rows x 64 bf16 channels
+
+template <int D>
+struct TcSmem {
+  static constexpr int KH = D / 64;                 // 64-channel halves
+  static constexpr int TILE = KH * kBoxBytes;       // one 128-row operand tile
+  static constexpr int A_OFF = 0;
+  static constexpr int B_OFF = TILE;
+  static constexpr int STAGE = TILE;                // one streamed B tile
+  static constexpr int STATS_OFF = B_OFF + kStagesTc * STAGE;  // 2 x 128 row stats (pass 1)
+  static constexpr int BAR_OFF = STATS_OFF + 2 * 128 * 8;
+  static constexpr int USED = BAR_OFF + 256 + 1024;  // + alignment slack
+  // at least 80 KB so that at most two CTAs (2 x 256 TMEM columns) share an SM
+  static constexpr int TOTAL = USED > 80 * 1024 ? USED : 80 * 1024;
+};
+
+// Barrier of the 128 epilogue threads that also ANDs a flag over them, so
+// all four warps take the same branch after it.
+__device__ __forceinline__ bool epilogue_all(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred pi, po;\n setp.ne.u32 pi, %1, 0;\n bar.red.and.pred po, 1, 128, pi;\n"
+      " selp.u32 %0, 1, 0, po;\n}"
+      : "=r"(r)
+      : "r"((uint32_t)v)
+      : "memory");
+  return r != 0;
+}
+
+// ----------------------------------------------------------------- PTX ----
+
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int c0, int c1, int c2,
+                                            uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, "
+      "%4}], [%5];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_alloc(uint32_t* dst, uint32_t cols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst)), "r"(cols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t cols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(cols) : "memory");
+}
+
+// D[tmem] (+)= A[smem desc] * B[smem desc]^T, bf16 x bf16 -> fp32.
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrives on `bar` once every tcgen05.mma issued so far by this thread is done.
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,"
+      "%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
+// 1024 bytes apart (the layout a 128B-swizzled TMA box of 128-byte rows
+// produces).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)1 << 16;            // leading byte offset (unused for swizzled K-major)
+  d |= (uint64_t)(1024 >> 4) << 32;  // stride byte offset: next 8-row group
+  d |= (uint64_t)1 << 46;            // descriptor version of tcgen05
+  d |= (uint64_t)2 << 61;            // 128-byte swizzle
+  return d;
+}
+
+// Instruction descriptor: bf16 A and B (K-major), fp32 D, M = N = 128.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
+
+// Bounded wait that also gives up when another role has aborted.
+__device__ __forceinline__ bool wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (*abort) return false;
+    if (global_timer_ns() - t0 > 1000000000ull) {
+      atomicOr(&g_mpc_status, kStatusWaitTimeout);
+      *abort = 1;
+      return false;
+    }
+  }
+  return true;
+}
+
+__device__ __forceinline__ int win_rows_of(const ScoreTcParams& p, int T) {
+  return count_from_ppm(T, T > p.long_threshold ? p.long_window_ppm : p.window_ppm);
+}
+
+template <int PASS, int D>
+__global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(const __grid_constant__ ScoreTcParams p) {
+  using S = TcSmem<D>;
+  constexpr int KH = S::KH;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::BAR_OFF);
+  uint64_t* empty = full + kStagesTc;
+  uint64_t* a_full = empty + kStagesTc;
+  uint64_t* acc_full = a_full + 1;
+  uint64_t* acc_empty = acc_full + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
+  volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // ---- work unit
+  const int HEADS = PASS == 0 ? p.Hq : p.Hkv;
+  const int unit = blockIdx.y;
+  const int head = unit % HEADS, b = (unit / HEADS) % p.B, ri = unit / (HEADS * p.B);
+  const int layer = p.refs.layer[ri], group = p.refs.group[ri];
+  const int T_b = p.lens[b];
+  const bool valid_len = T_b >= 1 && T_b <= p.t_max;
+  const int w = valid_len ? win_rows_of(p, T_b) : 0;
+  const int qoff = p.win_rows - w;
+  const int base = T_b - w;  // position of window row 0
+  int n_tiles = 0, i0 = 0, j0 = 0, i_start = 0, tiles_per_g = 0;
+  if (valid_len && w <= p.win_rows) {
+    if (PASS == 0) {
+      i0 = blockIdx.x * 128;  // window rows of this CTA
+      if (i0 < w) {
+        const int pos_last = base + min(i0 + 127, w - 1);
+        n_tiles = pos_last / 128 + 1;  // key tiles 0 .. pos_last
+      }
+    } else {
+      j0 = blockIdx.x * 128;  // keys of this CTA
+      if (j0 < T_b) {
+        const int i_first = max(0, j0 - base);  // first row that sees key j0
+        i_start = (i_first / 128) * 128;
+        tiles_per_g = (w - i_start + 127) / 128;
+        n_tiles = p.G * tiles_per_g;
+      }
+    }
+  }
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStagesTc; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(a_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], 4);
+    }
+    *abort = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 256);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0 && lane == 0 && n_tiles > 0) {
+    // ---------------------------------------------------- TMA producer
+    int n_issued = 0;
+    const int qrow0 = (b * p.Hq) * p.win_rows + qoff;       // + hq * win_rows + i
+    const int krow0 = (b * p.Hkv) * p.t_max;                 // + hk * t_max + j
+    mbar_arrive_expect_tx(a_full, S::TILE);
+    for (int kh = 0; kh < KH; ++kh) {
+      if (PASS == 0)
+        tma_load_3d(smem + S::A_OFF + kh * kBoxBytes, &p.map_q, kh * 64, qrow0 + head * p.win_rows + i0, layer, a_full);
+      else
+        tma_load_3d(smem + S::A_OFF + kh * kBoxBytes, &p.map_k, kh * 64, krow0 + head * p.t_max + j0, layer, a_full);
+    }
+    for (int t = 0; t < n_tiles; ++t) {
+      const int s = t % kStagesTc;
+      if (t >= kStagesTc && !wait_or_abort(&empty[s], ((t / kStagesTc) - 1) & 1, abort)) break;
+      uint8_t* st = smem + S::B_OFF + s * S::STAGE;
+      if (PASS == 0) {
+        mbar_arrive_expect_tx(&full[s], S::TILE);
+        const int kj = t * 128;
+        for (int kh = 0; kh < KH; ++kh)
+          tma_load_3d(st + kh * kBoxBytes, &p.map_k, kh * 64, krow0 + (head / p.G) * p.t_max + kj, layer, &full[s]);
+      } else {
+        const int g = t / tiles_per_g, it = i_start + (t % tiles_per_g) * 128;
+        const int hq = head * p.G + g;
+        mbar_arrive_expect_tx(&full[s], S::TILE);
+        for (int kh = 0; kh < KH; ++kh)
+          tma_load_3d(st + kh * kBoxBytes, &p.map_q, kh * 64, qrow0 + hq * p.win_rows + it, layer, &full[s]);
+      }
+      n_issued = t + 1;
+    }
+    // leave no copy in flight: wait (bounded) for the last stages issued
+    for (int t = n_issued > kStagesTc ? n_issued - kStagesTc : 0; t < n_issued; ++t) {
+      int never = 0;
+      wait_or_abort(&full[t % kStagesTc], (t / kStagesTc) & 1, &never);
+    }
+  } else if (warp == 1 && lane == 0 && n_tiles > 0) {
+    // ---------------------------------------------------- MMA issuer
+    int n_mma = 0;
+    if (wait_or_abort(a_full, 0, abort)) {
+      const uint32_t a_base = smem_u32(smem + S::A_OFF);
+      for (int t = 0; t < n_tiles; ++t) {
+        const int s = t % kStagesTc, buf = t & 1;
+        if (!wait_or_abort(&full[s], (t / kStagesTc) & 1, abort)) break;
+        if (t >= 2 && !wait_or_abort(&acc_empty[buf], ((t >> 1) - 1) & 1, abort)) break;
+        tc_fence_after();
+        const uint32_t b_base = smem_u32(smem + S::B_OFF + s * S::STAGE);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * kBoxBytes + (kk & 3) * 32;
+          umma_bf16(tmem + buf * 128, sw128_desc(a_base + off), sw128_desc(b_base + off), kIdesc, kk > 0);
+        }
+        umma_commit(&empty[s]);
+        umma_commit(&acc_full[buf]);
+        n_mma = t + 1;
+      }
+    }
+    // leave no MMA in flight before TMEM is released (bounded)
+    if (n_mma > 0) {
+      int never = 0;
+      wait_or_abort(&acc_full[(n_mma - 1) & 1], ((n_mma - 1) >> 1) & 1, &never);
+    }
+  } else if (warp >= 2) {
+    // ---------------------------------------------------- epilogue
+    const int quarter = warp & 3;               // TMEM lanes 32*quarter ..
+    const int r = quarter * 32 + lane;          // this thread's TMEM lane
+    const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
+    float m = kNegInf, l = 0.f, acc = 0.f;
+    const int i_row = i0 + r;                   // pass 0: window row
+    const int pos_row = base + i_row;
+    const int j_key = j0 + r;                   // pass 1: key
+    float2* stats_s = reinterpret_cast<float2*>(smem + S::STATS_OFF);
+    // pass 1: (m, 1/l) of the 128 window rows of a tile; thread r fetches row
+    // r of the next tile while the current one is processed
+    auto row_stats = [&](int t) -> float2 {
+      const int g = t / tiles_per_g, it = i_start + (t % tiles_per_g) * 128;
+      if (it + r >= w) return make_float2(0.f, 0.f);
+      return p.stats[(((int64_t)ri * p.B + b) * p.Hq + head * p.G + g) * p.win_rows + it + r];
+    };
+    float2 next_stats = make_float2(0.f, 0.f);
+    if (PASS == 1 && n_tiles > 0) next_stats = row_stats(0);
+    for (int t = 0; t < n_tiles; ++t) {
+      const int buf = t & 1;
+      if (PASS == 1) {
+        stats_s[buf * 128 + r] = next_stats;
+        if (t + 1 < n_tiles) next_stats = row_stats(t + 1);
+      }
+      const bool ok = wait_or_abort(&acc_full[buf], (t >> 1) & 1, abort);
+      if (!epilogue_all(ok)) break;
+      tc_fence_after();
+      if (PASS == 0) {
+        const int kj = t * 128;
+        const bool need_mask = kj + 127 > base + i0;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          tmem_ld32(lane_addr + buf * 128 + c * 32, v);
+          float mx = kNegInf;
+#pragma unroll
+          for (int k = 0; k < 32; ++k) {
+            if (need_mask && kj + c * 32 + k > pos_row) v[k] = kNegInf;
+            mx = fmaxf(mx, v[k]);
+          }
+          const float mnew = fmaxf(m, mx * p.scale_log2);
+          if (mnew != kNegInf) {
+            float sum = 0.f;
+#pragma unroll
+            for (int k = 0; k < 32; ++k) sum += fast_exp2(fmaf(v[k], p.scale_log2, -mnew));
+            l = (m == kNegInf) ? sum : l * fast_exp2(m - mnew) + sum;
+            m = mnew;
+          }
+        }
+      } else {
+        const int it = i_start + (t % tiles_per_g) * 128;
+        const float2* st = stats_s + buf * 128;
+        // rows it .. it+127; row i sees key j when j <= base + i and i < w
+        const bool need_mask = (j0 + 127 > base + it) || (it + 127 >= w);
+        float tsum = 0.f;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          tmem_ld32(lane_addr + buf * 128 + c * 32, v);
+#pragma unroll
+          for (int k = 0; k < 32; k += 2) {
+            const float4 ml = *reinterpret_cast<const float4*>(st + c * 32 + k);
+            float e0 = fast_exp2(fmaf(v[k], p.scale_log2, -ml.x)) * ml.y;
+            float e1 = fast_exp2(fmaf(v[k + 1], p.scale_log2, -ml.z)) * ml.w;
+            if (need_mask) {
+              const int ia = it + c * 32 + k;
+              if (ia >= w || j_key > base + ia) e0 = 0.f;
+              if (ia + 1 >= w || j_key > base + ia + 1) e1 = 0.f;
+            }
+            tsum += e0;
+            tsum += e1;
+          }
+        }
+        acc += tsum;
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[buf]);
+    }
+    if (!*abort) {
+      if (PASS == 0) {
+        if (i_row < w && n_tiles > 0)
+          p.stats[(((int64_t)ri * p.B + b) * p.Hq + head) * p.win_rows + i_row] = make_float2(m, 1.f / l);
+      } else {
+        if (n_tiles > 0 && j_key < T_b)
+          p.scores[((int64_t)(group * p.B + b) * p.Hkv + head) * p.t_max + j_key] = acc;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 256);
+  }
+}
+
+// ------------------------------------------------------------- host side ----
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static std::mutex mu;
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::lock_guard<std::mutex> lk(mu);
+  if (fn == nullptr) {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  }
+  return fn;
+}
+
+// 3-D map over [layers][rows][d] bf16 with 128-row x 64-channel boxes.
+bool make_map(CUtensorMap* map, const void* base, int d, int64_t rows, int layers, int64_t layer_stride_elems) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  const cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)rows, (cuuint64_t)layers};
+  const cuuint64_t strides[2] = {(cuuint64_t)d * 2, (cuuint64_t)layer_stride_elems * 2};
+  const cuuint32_t box[3] = {64, 128, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int PASS, int D>
+cudaError_t launch_pass(const ScoreTcParams& p, dim3 grid, cudaStream_t st) {
+  const int smem = TcSmem<D>::TOTAL;
+  cudaError_t e = ensure_dyn_smem((const void*)score_tc_kernel<PASS, D>, smem);
+  if (e != cudaSuccess) return e;
+  score_tc_kernel<PASS, D><<<grid, kTcThreads, smem, st>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_score_tc(ScoreTcParams& p, int D, int n_layer_span, cudaStream_t st) {
+  if (!make_map(&p.map_q, p.q_win, D, (int64_t)p.B * p.Hq * p.win_rows, n_layer_span, p.qw_ls) ||
+      !make_map(&p.map_k, p.k, D, (int64_t)p.B * p.Hkv * p.t_max, n_layer_span, p.k_ls))
+    return cudaErrorInvalidValue;
+  const dim3 g0((p.win_rows + 127) / 128, p.n_refs * p.B * p.Hq);
+  const dim3 g1((p.t_max + 127) / 128, p.n_refs * p.B * p.Hkv);
+  cudaError_t e;
+  if (D == 64) {
+    if ((e = launch_pass<0, 64>(p, g0, st)) != cudaSuccess) return e;
+    return launch_pass<1, 64>(p, g1, st);
+  }
+  if ((e = launch_pass<0, 128>(p, g0, st)) != cudaSuccess) return e;
+  return launch_pass<1, 128>(p, g1, st);
+}
+
+int take_status_score_tc() { return take_status(); }
+
+}  // namespace mpc

@@ -15,6 +15,8 @@
 //                    compaction that emits the kept positions ascending.
 // The two score passes are register-tiled FFMA products: a 16 x 16 thread
 // block computes a 64 x 64 tile, 4 x 4 outputs per thread.
+#include <cstring>
+
 #include "kernels.cuh"
 
 namespace mpc {
@@ -301,11 +303,36 @@ static cudaError_t set_smem(K kernel, int bytes) {
   return ensure_dyn_smem((const void*)kernel, bytes);
 }
 
-cudaError_t launch_static(const StaticParams& p, int dtype, int D, cudaStream_t st) {
-  const int smem = static_tile_smem(D);
-  const dim3 g1((p.win_rows + kTile - 1) / kTile, p.n_refs * p.B * p.Hq);
-  const dim3 g2((p.t_max + kTile - 1) / kTile, p.n_refs * p.B * p.Hkv);
+cudaError_t launch_static(const StaticParams& p, int dtype, int D, int n_layer_span, cudaStream_t st) {
   cudaError_t e = cudaSuccess;
+  if (dtype == MPC_BF16 && p.page_table == nullptr) {
+    // both score passes on the tensor cores
+    ScoreTcParams t;
+    memset(&t, 0, sizeof(t));
+    t.refs = p.refs;
+    t.n_refs = p.n_refs;
+    t.B = p.B;
+    t.Hq = p.Hq;
+    t.Hkv = p.Hkv;
+    t.G = p.G;
+    t.t_max = p.t_max;
+    t.win_rows = p.win_rows;
+    t.lens = p.lens;
+    t.q_win = p.q_win;
+    t.qw_ls = p.qw_ls;
+    t.k = p.k;
+    t.k_ls = p.k_ls;
+    t.window_ppm = p.window_ppm;
+    t.long_window_ppm = p.long_window_ppm;
+    t.long_threshold = p.long_threshold;
+    t.scale_log2 = p.scale_log2;
+    t.scores = p.scores;
+    t.stats = p.stats;
+    if ((e = launch_score_tc(t, D, n_layer_span, st)) != cudaSuccess) return e;
+  } else {
+    const int smem = static_tile_smem(D);
+    const dim3 g1((p.win_rows + kTile - 1) / kTile, p.n_refs * p.B * p.Hq);
+    const dim3 g2((p.t_max + kTile - 1) / kTile, p.n_refs * p.B * p.Hkv);
 #define MPC_STATIC_CASE(TT, DD)                                                        \
   if ((e = set_smem(rowstats_kernel<TT, DD>, smem)) != cudaSuccess) return e;          \
   if ((e = set_smem(colsum_kernel<TT, DD>, smem)) != cudaSuccess) return e;            \
@@ -313,11 +340,12 @@ cudaError_t launch_static(const StaticParams& p, int dtype, int D, cudaStream_t 
   if ((e = cudaGetLastError()) != cudaSuccess) return e;                               \
   colsum_kernel<TT, DD><<<g2, 256, smem, st>>>(p);                                     \
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  if (dtype == MPC_BF16 && D == 64) { MPC_STATIC_CASE(bf16, 64) }
-  else if (dtype == MPC_BF16) { MPC_STATIC_CASE(bf16, 128) }
-  else if (D == 64) { MPC_STATIC_CASE(float, 64) }
-  else { MPC_STATIC_CASE(float, 128) }
+    if (dtype == MPC_BF16 && D == 64) { MPC_STATIC_CASE(bf16, 64) }
+    else if (dtype == MPC_BF16) { MPC_STATIC_CASE(bf16, 128) }
+    else if (D == 64) { MPC_STATIC_CASE(float, 64) }
+    else { MPC_STATIC_CASE(float, 128) }
 #undef MPC_STATIC_CASE
+  }
   const int bsmem = p.t_max * 4;
   if ((e = set_smem(budget_kernel, bsmem)) != cudaSuccess) return e;
   budget_kernel<<<p.n_refs * p.B * p.Hkv, kBudgetThreads, bsmem, st>>>(p);
