@@ -158,11 +158,8 @@ int validate_static(const mpc_static_args* a, StaticParams* p) {
   return MPC_OK;
 }
 
-// Row statistics (m, 1/l) of every window row, plus 1 KB so that a 128-row
-// bulk read of the last rows stays inside the workspace.
-size_t static_ws(const StaticParams& p) {
-  return (size_t)p.n_refs * p.B * p.Hq * p.win_rows * sizeof(float2) + 1024;
-}
+// Row statistics (m, 1/l) of every window row.
+size_t static_ws(const StaticParams& p) { return (size_t)p.n_refs * p.B * p.Hq * p.win_rows * sizeof(float2); }
 
 // ------------------------------------------------------------ clusters ----
 int validate_clusters(const mpc_cluster_args* a, ClusterParams* p) {
@@ -308,7 +305,14 @@ int validate_attn(const mpc_attn_args* a, AttnParams* p, AttnPlan* plan) {
     off += (bytes + 255) & ~size_t(255);
     return o;
   };
-  plan->part_off = take(n_split > 1 ? (size_t)units * n_split * G * (a->head_dim + 4) * sizeof(float) : 0);
+  if (a->dtype == MPC_BF16) {
+    // persistent kernel: two partial records per warp of the grid
+    if (a->batch > attn_persist_batch_max())
+      return fail(MPC_ERR_BAD_SHAPE, "batch %d > %d sequences per call", a->batch, attn_persist_batch_max());
+    plan->part_off = take((size_t)2 * attn_persist_ctas_max() * 4 * G * (a->head_dim + 4) * sizeof(float));
+  } else {
+    plan->part_off = take(n_split > 1 ? (size_t)units * n_split * G * (a->head_dim + 4) * sizeof(float) : 0);
+  }
   plan->ucnt_off = take((size_t)units * sizeof(int));
   plan->gcnt_off = take(sizeof(int));
   plan->bytes = off;

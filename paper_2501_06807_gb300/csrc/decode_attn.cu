@@ -13,6 +13,8 @@
 // memory; with several chunks per unit the CTA writes (max, sum, o) to the
 // workspace and the last CTA of the unit (atomic ticket, no waiting) merges
 // them by log-sum-exp and writes o.
+#include <mutex>
+
 #include "kernels.cuh"
 
 namespace mpc {
@@ -29,26 +31,33 @@ struct Unit {
   const int* sel;
 };
 
-__device__ __forceinline__ Unit make_unit(const AttnParams& p) {
+__device__ __forceinline__ Unit make_unit_at(const AttnParams& p, int ri, int b, int h) {
   Unit u;
-  const int unit = blockIdx.y;
-  u.h = unit % p.Hkv;
-  u.b = (unit / p.Hkv) % p.B;
-  const int ri = unit / (p.Hkv * p.B);
+  u.h = h;
+  u.b = b;
   u.layer = p.refs.layer[ri];
   u.group = p.refs.group[ri];
   u.leader = p.refs.leader[ri];
   const int s = p.pyr.s;
-  u.n = p.n_tok[u.b];
+  u.n = p.n_tok[b];
   u.C1 = u.n / s;
   u.tail = u.n - u.C1 * s;
-  u.k1 = p.sel_cap > 0 ? min(p.n_sel[u.b], min(u.C1, p.sel_cap)) : 0;
+  u.k1 = p.sel_cap > 0 ? min(p.n_sel[b], min(u.C1, p.sel_cap)) : 0;
   u.n_sel_rows = u.k1 * s;
   u.n_att = u.n_sel_rows + u.tail + 1;
   u.n_tiles = (u.n_att + 15) / 16;
+  u.t_begin = 0;
+  u.t_end = u.n_tiles;
+  u.sel = p.sel + ((int64_t)(u.group * p.B + b) * p.Hkv + h) * p.sel_cap;
+  return u;
+}
+
+// Unit of a split-grid CTA: blockIdx.y = unit, blockIdx.x = chunk of tiles.
+__device__ __forceinline__ Unit make_unit(const AttnParams& p) {
+  const int unit = blockIdx.y;
+  Unit u = make_unit_at(p, unit / (p.Hkv * p.B), (unit / p.Hkv) % p.B, unit % p.Hkv);
   u.t_begin = blockIdx.x * p.tiles_per_split;
   u.t_end = min(u.n_tiles, u.t_begin + p.tiles_per_split);
-  u.sel = p.sel + ((int64_t)(u.group * p.B + u.b) * p.Hkv + u.h) * p.sel_cap;
   return u;
 }
 
@@ -73,7 +82,9 @@ __device__ __forceinline__ int src_row(const Unit& u, int s, int a) {
 template <int ROWB>
 __device__ __forceinline__ void issue_tile(const Unit& u, int s, int t, const uint8_t* kbase,
                                            const uint8_t* vbase, uint8_t* sK, uint8_t* sV,
-                                           int8_t* keys, uint64_t* bar, int lane) {
+                                           int8_t* keys, uint64_t* bar, int lane,
+                                           const void* q_src = nullptr, void* q_dst = nullptr,
+                                           uint32_t q_bytes = 0) {
   const int r = lane & 15;
   const int a = t * 16 + r;
   const bool valid = a < u.n_att;
@@ -87,8 +98,9 @@ __device__ __forceinline__ void issue_tile(const Unit& u, int s, int t, const ui
   const uint32_t mstart = __ballot_sync(0xffffffffu, start) & 0xffffu;
   const uint32_t mcache = __ballot_sync(0xffffffffu, from_cache) & 0xffffu;
   const int ncache = __popc(mcache);  // cache rows form a prefix of the tile
-  if (lane == 0) mbar_arrive_expect_tx(bar, (uint32_t)(ncache * ROWB * 2));
+  if (lane == 0) mbar_arrive_expect_tx(bar, (uint32_t)(ncache * ROWB * 2) + (q_src ? q_bytes : 0u));
   __syncwarp();
+  if (q_src != nullptr && lane == 16) bulk_g2s(q_dst, q_src, q_bytes, bar);
   if (lane < 16 && start) {
     const uint32_t later = mstart & ~((2u << r) - 1u);
     int end = later ? (__ffs(later) - 1) : ncache;
@@ -201,8 +213,7 @@ template <typename T, int D>
 __device__ void seal_tail(const AttnParams& p, const Unit& u, const T* kcache) {
   const int s = p.pyr.s;
   if (!(u.leader && u.tail + 1 == s && p.rmax != nullptr)) return;
-  const int lane = threadIdx.x & 31;
-  if (threadIdx.x >= 32) return;
+  const int lane = threadIdx.x & 31;  // called by one warp
   const int c_new = u.C1;
   if (c_new >= p.pyr.cap[0]) {
     if (lane == 0) atomicOr(&g_mpc_status, 2);
@@ -215,6 +226,7 @@ __device__ void seal_tail(const AttnParams& p, const Unit& u, const T* kcache) {
     mx[i] = kNegInf;
     mn[i] = -kNegInf;
   }
+#pragma unroll 8
   for (int r = c_new * s; r < c_new * s + s; ++r) {
     const T* row = kcache + (int64_t)r * D;
 #pragma unroll
@@ -269,227 +281,562 @@ __device__ __forceinline__ void finish_grid(const AttnParams& p) {
   }
 }
 
-// ------------------------------------------------------------ bf16 path ----
+// ------------------------------------------------ bf16 path (persistent) ----
+//
+// One CTA per SM, four warps.  The tiles of all units (every selected
+// cluster row tile, tail and appended row of every (layer, sequence, kv
+// head)) form one list, cut into contiguous, equal ranges, one per warp slot
+// (slots interleaved over the CTAs, at most one slot per tile).  Every warp
+// streams its range through its own ring of shared-memory stages (1-D bulk
+// copies of K and V tile rows), so every SM moves the same amount of KV.
+//
+// Tiles are staged with cp.async (16 bytes per lane, committed as one group
+// per tile, so a warp keeps NST tiles in flight at the cost of a few
+// instructions each).  With s a multiple of 16 every tile is one run of
+// consecutive cache rows; other cluster sizes gather the rows one by one.
+//
+// Per tile the group's heads are the N dimension of the tensor-core products
+// (S^T = K Q^T, O^T = V^T P^T with m16n8k16 bf16 mma, P split into bf16 hi +
+// lo), so one 8-head n-tile covers a GQA group of up to 8 query heads.  P
+// moves from the accumulator layout of S^T to the operand layout of P^T with
+// movmatrix (an in-register 8x8 transpose).
+//
+// A unit finished inside one warp is written directly.  A unit split across
+// warps leaves partial (max, sum, o) records, two slots per warp (2 slot: the
+// warp's first piece when its unit began earlier, 2 slot + 1: its last piece
+// when the unit continues), and the warp that completes the unit's ticket
+// count merges them by log-sum-exp.
+
+constexpr int kMaxPersistCtas = 152;
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+constexpr int kMaxBatchPersist = 512;
+constexpr int kSelSmem = 256;  // selected ids staged per warp (longer lists are read from global)
+
 template <int D>
-__global__ void __launch_bounds__(128) attn_bf16_kernel(const __grid_constant__ AttnParams p) {
-  using S = Smem<D, 2>;
+struct PSmem {
+  static constexpr int ROWB = D * 2;
+  static constexpr int TILEB = 16 * ROWB;
+  static __host__ __device__ constexpr int qbytes(int G) { return ((G * D * 2 + 127) / 128) * 128; }
+  static __host__ __device__ constexpr int stage(int G) { return 2 * TILEB + qbytes(G); }
+  static __host__ __device__ constexpr int key_off(int G, int nst) { return kWarps * nst * stage(G); }
+  static __host__ __device__ constexpr int sel_off(int G, int nst) { return key_off(G, nst) + kWarps * nst * 16; }
+  static __host__ __device__ constexpr int scr_off(int G, int nst) { return sel_off(G, nst) + kWarps * kSelSmem * 4; }
+  static __host__ __device__ constexpr int tab_off(int G, int nst) { return scr_off(G, nst) + kWarps * 96 * 4; }
+  static __host__ __device__ constexpr int total(int G, int nst, int B) { return tab_off(G, nst) + (4 * B + 2) * 4; }
+};
+
+// Ring depth per warp for a head dimension and GQA group size (compile-time
+// for cp.async.wait_group): 5 stages (d 128, up to 8 heads), 4 (d 128, up
+// to 16 heads), 8 (d 64).
+inline int persist_stages(int D, int G) { return D == 64 ? 8 : (G <= 8 ? 5 : 4); }
+
+struct Cursor {
+  int ri, b, h, lt;
+};
+
+// In-register transpose of an 8x8 b16 matrix held in mma fragment layout.
+__device__ __forceinline__ uint32_t movmatrix_t(uint32_t a) {
+  uint32_t d;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
+  return d;
+}
+
+template <int D, int HN, int NST>
+__global__ void __launch_bounds__(128, 1) attn_bf16_persist_kernel(const __grid_constant__ AttnParams p) {
+  using S = PSmem<D>;
   constexpr int ROWB = S::ROWB;
-  constexpr int KS = D / 16;  // k-steps of the score product
+  constexpr int TILEB = S::TILEB;
+  constexpr int KS = D / 16;  // k-steps of S^T and m-tiles of O^T
   extern __shared__ __align__(128) uint8_t smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const Unit u = make_unit(p);
-  const int s = p.pyr.s;
-  const int G = p.G;
-  bf16* kcache = (bf16*)p.kc + u.layer * p.cache_ls + (int64_t)(u.b * p.Hkv + u.h) * p.cap_tokens * D;
-  bf16* vcache = (bf16*)p.vc + u.layer * p.cache_ls + (int64_t)(u.b * p.Hkv + u.h) * p.cap_tokens * D;
-  float* mw = reinterpret_cast<float*>(smem + S::MERGE_OFF);
+  const int G = p.G, B = p.B, Hkv = p.Hkv, s = p.pyr.s;
+  const int STAGE = S::stage(G);
+  constexpr int CH = ROWB / 16;  // 16-byte chunks per row
+  uint8_t* ring = smem + warp * NST * STAGE;
+  int8_t* keys = reinterpret_cast<int8_t*>(smem + S::key_off(G, NST)) + warp * NST * 16;
+  int* sel_s = reinterpret_cast<int*>(smem + S::sel_off(G, NST)) + warp * kSelSmem;
+  float* scr = reinterpret_cast<float*>(smem + S::scr_off(G, NST)) + warp * 96;  // merge scratch
+  int* s_nt = reinterpret_cast<int*>(smem + S::tab_off(G, NST));  // tiles per unit of sequence b
+  int* s_pre = s_nt + B;                                           // exclusive prefix of s_nt (B + 1)
+  int* s_n = s_pre + B + 1;                                        // cache rows before the append
+  int* s_k1 = s_n + B;                                             // selected clusters
 
-  if (u.n < 0 || u.n + 1 > p.cap_tokens) {  // no room for the append: report, write nothing
-    if (threadIdx.x == 0) atomicOr(&g_mpc_status, 2);
-    finish_grid(p);
-    return;
-  }
-
-  uint8_t* ring = smem + warp * kStages * S::STAGE_BYTES;
-  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + S::BAR_OFF) + warp * kStages;
-  int8_t* keys = reinterpret_cast<int8_t*>(smem + S::KEY_OFF) + warp * kStages * 16;
-
-  // zero the ring once so rows past the end of the list are finite
-  for (int i = lane; i < kStages * S::STAGE_BYTES / 16; i += 32)
-    reinterpret_cast<uint4*>(ring)[i] = make_uint4(0, 0, 0, 0);
-  if (lane == 0) {
-    for (int st = 0; st < kStages; ++st) mbar_init(&bar[st], 1);
-    fence_barrier_init();
-  }
-  fence_proxy_async_smem();
-  __syncwarp();
-
-  const int first = u.t_begin + warp;
-  const int nj = (u.t_end > first) ? (u.t_end - first + kWarps - 1) / kWarps : 0;
-
-  // query fragments: rows of the mma A operand are the group's heads
-  uint32_t qa[KS][4];
-  {
-    const bf16* qp = (const bf16*)p.q + u.layer * p.q_ls + ((int64_t)u.b * p.Hq + u.h * G) * D;
-    const int r0 = lane >> 2, r1 = r0 + 8, c0 = 2 * (lane & 3);
+  // ---- per-sequence table
+  if (warp == 0) {
+    int carry = 0;
+    for (int b0 = 0; b0 < B; b0 += 32) {
+      const int b = b0 + lane;
+      int nt = 0, n = 0, k1 = 0;
+      if (b < B) {
+        n = p.n_tok[b];
+        if (n < 0 || n + 1 > p.cap_tokens) {
+          atomicOr(&g_mpc_status, 2);  // no room for the append: skip the sequence
+        } else {
+          const int C1 = n / s;
+          k1 = p.sel_cap > 0 ? min(p.n_sel[b], min(C1, p.sel_cap)) : 0;
+          nt = (k1 * s + (n - C1 * s) + 1 + 15) / 16;
+        }
+      }
+      int incl = nt;
 #pragma unroll
-    for (int ks = 0; ks < KS; ++ks) {
-      const int c = ks * 16 + c0;
-      qa[ks][0] = (r0 < G) ? *reinterpret_cast<const uint32_t*>(qp + r0 * D + c) : 0u;
-      qa[ks][1] = (r1 < G) ? *reinterpret_cast<const uint32_t*>(qp + r1 * D + c) : 0u;
-      qa[ks][2] = (r0 < G) ? *reinterpret_cast<const uint32_t*>(qp + r0 * D + c + 8) : 0u;
-      qa[ks][3] = (r1 < G) ? *reinterpret_cast<const uint32_t*>(qp + r1 * D + c + 8) : 0u;
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      if (b < B) {
+        s_nt[b] = nt;
+        s_pre[b] = carry + incl - nt;
+        s_n[b] = n;
+        s_k1[b] = k1;
+      }
+      carry += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) s_pre[B] = carry;
+  }
+  __syncthreads();
+  const bool fast = (s & 15) == 0;  // every tile is one run of consecutive rows
+  const int s16 = s >> 4;
+
+  const int64_t TPR = (int64_t)Hkv * s_pre[B];
+  const int64_t NT = TPR * p.n_refs;
+  const int64_t NW_all = (int64_t)gridDim.x * kWarps;
+  const int NW = (int)(NW_all < NT ? NW_all : NT);
+  const int gw = warp * gridDim.x + blockIdx.x;
+  const int64_t x0 = gw < NW ? NT * gw / NW : 0, x1 = gw < NW ? NT * (gw + 1) / NW : 0;
+  auto warp_of = [&](int64_t x) { return (int)((x * NW + NW - 1) / NT); };
+  auto locate = [&](int64_t x) {
+    Cursor c;
+    c.ri = (int)(x / TPR);
+    const int64_t rem = x - c.ri * TPR;
+    int lo = 0, hi = B - 1;  // largest b with Hkv * pre[b] <= rem
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if ((int64_t)Hkv * s_pre[mid] <= rem) lo = mid;
+      else hi = mid - 1;
+    }
+    c.b = lo;
+    const int64_t rem2 = rem - (int64_t)Hkv * s_pre[lo];
+    c.h = (int)(rem2 / s_nt[lo]);
+    c.lt = (int)(rem2 % s_nt[lo]);
+    return c;
+  };
+  auto advance = [&](Cursor& c) {
+    if (++c.lt < s_nt[c.b]) return;
+    c.lt = 0;
+    if (++c.h < Hkv) return;
+    c.h = 0;
+    do {
+      if (++c.b == B) {
+        c.b = 0;
+        ++c.ri;
+      }
+    } while (s_nt[c.b] == 0);
+  };
+  auto unit_at = [&](const Cursor& c) {
+    Unit u;
+    u.h = c.h;
+    u.b = c.b;
+    u.layer = p.refs.layer[c.ri];
+    u.group = p.refs.group[c.ri];
+    u.leader = p.refs.leader[c.ri];
+    u.n = s_n[c.b];
+    u.C1 = u.n / s;
+    u.tail = u.n - u.C1 * s;
+    u.k1 = s_k1[c.b];
+    u.n_sel_rows = u.k1 * s;
+    u.n_att = u.n_sel_rows + u.tail + 1;
+    u.n_tiles = s_nt[c.b];
+    u.t_begin = 0;
+    u.t_end = u.n_tiles;
+    u.sel = p.sel + ((int64_t)(u.group * B + c.b) * Hkv + c.h) * p.sel_cap;
+    return u;
+  };
+  auto kv_base = [&](const Unit& u, int which) {
+    const bf16* base = (const bf16*)(which ? p.vc : p.kc) + u.layer * p.cache_ls +
+                       (int64_t)(u.b * Hkv + u.h) * p.cap_tokens * D;
+    return reinterpret_cast<const uint8_t*>(base);
+  };
+  const int nj = (int)(x1 - x0);
+
+  // ---- issue side: runs NST tiles ahead of the compute side
+  Unit iu;
+  const uint8_t* ikb = nullptr;
+  const uint8_t* ivb = nullptr;
+  auto issue = [&](const Cursor& c, int j) {
+    const bool first = (j == 0) || (c.lt == 0);
+    if (first) {
+      iu = unit_at(c);
+      ikb = kv_base(iu, 0);
+      ivb = kv_base(iu, 1);
+      if (iu.k1 <= kSelSmem) {  // stage the unit's selected ids once
+        __syncwarp();
+        for (int i = lane; i < iu.k1; i += 32) sel_s[i] = iu.sel[i];
+        __syncwarp();
+        iu.sel = sel_s;
+      }
+    }
+    uint8_t* sK = ring + (j % NST) * STAGE;
+    uint8_t* sV = sK + TILEB;
+    const int t = c.lt;
+    const int a0 = t * 16;
+    const int ncache = max(0, min(16, iu.n_att - 1 - a0));  // cache rows of the tile
+    if (fast) {
+      int src0;
+      if (a0 < iu.n_sel_rows) {
+        const int ci = t / s16;
+        int id = iu.sel[ci];
+        if (id < 0 || id >= iu.C1) {
+          if (lane == 0) atomicOr(&g_mpc_status, 4);
+          id = 0;
+        }
+        src0 = id * s + (a0 - ci * s);
+      } else {
+        src0 = iu.C1 * s + (a0 - iu.n_sel_rows);
+      }
+      const uint8_t* gk = ikb + (int64_t)src0 * ROWB;
+      const uint8_t* gv = ivb + (int64_t)src0 * ROWB;
+      for (int i = lane; i < ncache * CH; i += 32) {
+        cp_async16(sK + i * 16, gk + i * 16);
+        cp_async16(sV + i * 16, gv + i * 16);
+      }
+    } else {
+      const int r = lane & 15;
+      const int arow = a0 + r;
+      int src = 0;
+      if (r < ncache) src = src_row(iu, s, arow);
+      else if (arow == iu.n_att - 1) src = iu.n;
+      if (lane < 16) keys[(j % NST) * 16 + r] = (int8_t)((arow < iu.n_att) ? (src & 7) : (r & 7));
+#pragma unroll 4
+      for (int i = lane; i < 16 * CH; i += 32) {
+        const int row = i / CH, ch = i % CH;
+        const int srow = __shfl_sync(0xffffffffu, src, row);
+        if (row < ncache) {
+          cp_async16(sK + i * 16, ikb + (int64_t)srow * ROWB + ch * 16);
+          cp_async16(sV + i * 16, ivb + (int64_t)srow * ROWB + ch * 16);
+        }
+      }
+    }
+    if (first) {
+      const uint8_t* q = reinterpret_cast<const uint8_t*>((const bf16*)p.q + iu.layer * p.q_ls +
+                                                          ((int64_t)iu.b * p.Hq + iu.h * G) * D);
+      for (int i = lane; i < G * D * 2 / 16; i += 32) cp_async16(sK + 2 * TILEB + i * 16, q + i * 16);
+    }
+  };
+
+  Cursor cc, ic;
+  if (nj > 0) {
+    cc = locate(x0);
+    ic = cc;
+    for (int j = 0; j < NST; ++j) {
+      if (j < nj) {
+        issue(ic, j);
+        advance(ic);
+      }
+      cp_async_commit();
     }
   }
 
-  for (int j = 0; j < kStages && j < nj; ++j) {
-    uint8_t* sK = ring + j * S::STAGE_BYTES;
-    issue_tile<ROWB>(u, s, first + j * kWarps, (const uint8_t*)kcache, (const uint8_t*)vcache, sK,
-                     sK + S::TILEB, keys + j * 16, &bar[j], lane);
-  }
+  // ---- compute side
+  uint32_t qb[HN][KS][2];  // Q^T operand: k = channels, n = heads
+  float o[KS][HN][4];      // O^T accumulators: m = channels, n = heads
+  float m_run[HN][2], l_run[HN][2];
+  Unit u;
+  int u_ri = 0;
+  bool have = false;
+  const int r_tok = lane >> 2;      // token row of S^T (and +8)
+  const int h_off = 2 * (lane & 3);  // first of this thread's two heads in an n-tile
 
-  float o[D / 8][4];
+  auto flush = [&]() {
+    float lq[HN][2];
 #pragma unroll
-  for (int i = 0; i < D / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-  float m_run[2] = {kNegInf, kNegInf}, l_run[2] = {0.f, 0.f};
-  uint32_t phase = 0;
-  bool ok = true;
+    for (int hn = 0; hn < HN; ++hn)
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        float v = l_run[hn][e];
+        v += __shfl_xor_sync(0xffffffffu, v, 4);
+        v += __shfl_xor_sync(0xffffffffu, v, 8);
+        v += __shfl_xor_sync(0xffffffffu, v, 16);
+        lq[hn][e] = v;
+      }
+    const int64_t ustart = (int64_t)u_ri * TPR + (int64_t)Hkv * s_pre[u.b] + (int64_t)u.h * s_nt[u.b];
+    const int64_t uend = ustart + s_nt[u.b];
+    const bool before = ustart < x0, after = uend > x1;
+    float* outp = p.out + u.layer * p.out_ls + ((int64_t)u.b * p.Hq + u.h * G) * D;
+    if (!before && !after) {
+#pragma unroll
+      for (int hn = 0; hn < HN; ++hn)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int g = hn * 8 + h_off + e;
+          if (g < G) {
+            const float inv = 1.f / lq[hn][e];
+#pragma unroll
+            for (int mt = 0; mt < KS; ++mt) {
+              outp[g * D + mt * 16 + r_tok] = o[mt][hn][e] * inv;
+              outp[g * D + mt * 16 + r_tok + 8] = o[mt][hn][2 + e] * inv;
+            }
+          }
+        }
+    } else {
+      const int rec = 2 * gw + (before ? 0 : 1);
+      float* dst = p.part + (int64_t)rec * G * (D + 4);
+#pragma unroll
+      for (int hn = 0; hn < HN; ++hn)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int g = hn * 8 + h_off + e;
+          if (g < G) {
+            if (r_tok == 0) {
+              dst[g * (D + 4)] = m_run[hn][e];
+              dst[g * (D + 4) + 1] = lq[hn][e];
+            }
+#pragma unroll
+            for (int mt = 0; mt < KS; ++mt) {
+              dst[g * (D + 4) + 4 + mt * 16 + r_tok] = o[mt][hn][e];
+              dst[g * (D + 4) + 4 + mt * 16 + r_tok + 8] = o[mt][hn][2 + e];
+            }
+          }
+        }
+      __threadfence();
+      __syncwarp();
+      const int wa = warp_of(ustart), wb = warp_of(uend - 1);
+      const int64_t unit_id = ((int64_t)u_ri * B + u.b) * Hkv + u.h;
+      int ticket = 0;
+      if (lane == 0) ticket = atomicAdd(&p.unit_counter[unit_id], 1);
+      ticket = __shfl_sync(0xffffffffu, ticket, 0);
+      if (ticket == wb - wa) {
+        __threadfence();
+        const int nrec = wb - wa + 1;
+        auto rec_ptr = [&](int k, int g) {
+          const int r2 = k == 0 ? 2 * wa + 1 : 2 * (wa + k);
+          return p.part + ((int64_t)r2 * G + g) * (D + 4);
+        };
+        if (nrec * G <= 32 && nrec <= 8) {
+          // (max, sum) of every (record, head) in parallel, one pair per lane
+          const int pk = lane / G, pg = lane % G;
+          float mk = kNegInf, lk = 0.f;
+          if (lane < nrec * G) {
+            mk = __ldcg(rec_ptr(pk, pg));
+            lk = __ldcg(rec_ptr(pk, pg) + 1);
+          }
+          scr[lane] = mk;
+          __syncwarp();
+          float M = kNegInf;
+          for (int k = 0; k < nrec; ++k) M = fmaxf(M, scr[k * G + pg]);
+          const float wk = (lane < nrec * G && mk != kNegInf) ? fast_exp2(mk - M) : 0.f;
+          scr[32 + lane] = wk;
+          scr[64 + lane] = wk * lk;
+          __syncwarp();
+          for (int g = 0; g < G; ++g) {
+            float v[8][D / 32];
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+#pragma unroll
+              for (int t = 0; t < D / 32; ++t) v[k][t] = (k < nrec) ? __ldcg(rec_ptr(k, g) + 4 + lane + 32 * t) : 0.f;
+            float L = 0.f, acc[D / 32];
+#pragma unroll
+            for (int t = 0; t < D / 32; ++t) acc[t] = 0.f;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              if (k < nrec) {
+                const float wgt = scr[32 + k * G + g];
+                L += scr[64 + k * G + g];
+#pragma unroll
+                for (int t = 0; t < D / 32; ++t) acc[t] = fmaf(wgt, v[k][t], acc[t]);
+              }
+            }
+            const float inv = 1.f / L;
+#pragma unroll
+            for (int t = 0; t < D / 32; ++t) outp[g * D + lane + 32 * t] = acc[t] * inv;
+          }
+          __syncwarp();
+        } else {
+          for (int g = 0; g < G; ++g) {
+            float M = kNegInf;
+            for (int k = 0; k < nrec; ++k) M = fmaxf(M, __ldcg(rec_ptr(k, g)));
+            float L = 0.f;
+            float acc[D / 32];
+#pragma unroll
+            for (int t = 0; t < D / 32; ++t) acc[t] = 0.f;
+            for (int k = 0; k < nrec; ++k) {
+              const float* rp = rec_ptr(k, g);
+              const float mm = __ldcg(rp);
+              const float f = (mm == kNegInf) ? 0.f : fast_exp2(mm - M);
+              L += f * __ldcg(rp + 1);
+#pragma unroll
+              for (int t = 0; t < D / 32; ++t) acc[t] += f * __ldcg(rp + 4 + lane + 32 * t);
+            }
+            const float inv = 1.f / L;
+#pragma unroll
+            for (int t = 0; t < D / 32; ++t) outp[g * D + lane + 32 * t] = acc[t] * inv;
+          }
+        }
+        if (lane == 0) p.unit_counter[unit_id] = 0;
+      }
+    }
+    // the piece that holds the appended row seals a full tail
+    if (uend <= x1) seal_tail<bf16, D>(p, u, reinterpret_cast<const bf16*>(kv_base(u, 0)));
+  };
 
   for (int j = 0; j < nj; ++j) {
-    const int st = j % kStages;
-    const int t = first + j * kWarps;
-    uint8_t* sK = ring + st * S::STAGE_BYTES;
-    uint8_t* sV = sK + S::TILEB;
+    const int st = j % NST;
+    uint8_t* sK = ring + st * STAGE;
+    uint8_t* sV = sK + TILEB;
     int8_t* kk = keys + st * 16;
-    if (!mbar_wait_bounded(&bar[st], (phase >> st) & 1u)) {
-      ok = false;
-      break;
-    }
-    phase ^= (1u << st);
-    // the appended row goes straight from the inputs to the cache and the tile
-    const int cur_r = (u.n_att - 1) - t * 16;
-    if (cur_r >= 0 && cur_r < 16) {
-      const int64_t nb = u.layer * p.kvn_ls + (int64_t)(u.b * p.Hkv + u.h) * D;
-      const uint4* kn = reinterpret_cast<const uint4*>((const bf16*)p.k_new + nb);
-      const uint4* vn = reinterpret_cast<const uint4*>((const bf16*)p.v_new + nb);
-      constexpr int CH = ROWB / 16;
-      for (int i = lane; i < 2 * CH; i += 32) {
-        const int ch = i % CH;
-        const bool isv = i >= CH;
-        const uint4 val = isv ? vn[ch] : kn[ch];
-        const int pch = ch ^ (u.n & 7);
-        uint8_t* dst_s = (isv ? sV : sK) + cur_r * ROWB + pch * 16;
-        *reinterpret_cast<uint4*>(dst_s) = val;
-        bf16* dst_g = (isv ? vcache : kcache) + (int64_t)u.n * D;
-        reinterpret_cast<uint4*>(dst_g)[pch] = val;
+    const bool new_unit = (j == 0) || (cc.lt == 0);
+    if (new_unit) {
+      if (have) flush();
+      u = unit_at(cc);
+      u_ri = cc.ri;
+      have = true;
+#pragma unroll
+      for (int hn = 0; hn < HN; ++hn) {
+        m_run[hn][0] = m_run[hn][1] = kNegInf;
+        l_run[hn][0] = l_run[hn][1] = 0.f;
+#pragma unroll
+        for (int mt = 0; mt < KS; ++mt) o[mt][hn][0] = o[mt][hn][1] = o[mt][hn][2] = o[mt][hn][3] = 0.f;
       }
+    }
+    cp_async_wait<NST - 1>();  // this lane's copies of tile j have landed
+    __syncwarp();
+    if (new_unit) {
+      // Q^T operand from the stage's q slot: b0 = q[head][2c, 2c+1], b1 = +8
+      const bf16* qs = reinterpret_cast<const bf16*>(sK + 2 * TILEB);
+#pragma unroll
+      for (int hn = 0; hn < HN; ++hn) {
+        const int hq = hn * 8 + r_tok;
+#pragma unroll
+        for (int ks = 0; ks < KS; ++ks) {
+          const int c = ks * 16 + h_off;
+          qb[hn][ks][0] = (hq < G) ? *reinterpret_cast<const uint32_t*>(qs + hq * D + c) : 0u;
+          qb[hn][ks][1] = (hq < G) ? *reinterpret_cast<const uint32_t*>(qs + hq * D + c + 8) : 0u;
+        }
+      }
+    }
+    const int t = cc.lt;
+    const int n_valid = min(16, u.n_att - t * 16);
+    const int cur_r = (u.n_att - 1) - t * 16;
+    if (cur_r < 16 || n_valid < 16) {
+      constexpr int CH = ROWB / 16;
+      if (cur_r >= 0 && cur_r < 16) {
+        // the appended row goes from the inputs to the cache and to this tile
+        const int64_t nb = u.layer * p.kvn_ls + (int64_t)(u.b * Hkv + u.h) * D;
+        const uint4* kn = reinterpret_cast<const uint4*>((const bf16*)p.k_new + nb);
+        const uint4* vn = reinterpret_cast<const uint4*>((const bf16*)p.v_new + nb);
+        bf16* kcw = (bf16*)p.kc + u.layer * p.cache_ls + (int64_t)(u.b * Hkv + u.h) * p.cap_tokens * D;
+        bf16* vcw = (bf16*)p.vc + u.layer * p.cache_ls + (int64_t)(u.b * Hkv + u.h) * p.cap_tokens * D;
+        for (int i = lane; i < 2 * CH; i += 32) {
+          const int ch = i % CH;
+          const bool isv = i >= CH;
+          const uint4 val = isv ? vn[ch] : kn[ch];
+          const int pch = ch ^ (u.n & 7);
+          *reinterpret_cast<uint4*>((isv ? sV : sK) + cur_r * ROWB + pch * 16) = val;
+          reinterpret_cast<uint4*>((isv ? vcw : kcw) + (int64_t)u.n * D)[pch] = val;
+        }
+      }
+      // rows past the end of the list are zeroed so that P V sees finite values
+      for (int i = lane; i < (16 - n_valid) * CH; i += 32)
+        reinterpret_cast<uint4*>(sV + n_valid * ROWB)[i] = make_uint4(0, 0, 0, 0);
       __syncwarp();
     }
-
-    // scores S = Q K^T for 16 rows (two n-tiles of 8 keys)
-    float sacc[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}};
+    // S^T = K Q^T: 16 tokens x 8 heads per n-tile, two accumulators per
+    // n-tile (even / odd k-steps) to halve the dependency chain
+    float sc[HN][2][4];
+#pragma unroll
+    for (int hn = 0; hn < HN; ++hn)
+#pragma unroll
+      for (int a2 = 0; a2 < 2; ++a2) sc[hn][a2][0] = sc[hn][a2][1] = sc[hn][a2][2] = sc[hn][a2][3] = 0.f;
     {
-      const int tok = ((lane >> 4) << 3) + (lane & 7);
-      const int key = kk[tok];
+      // A = K tile: matrices (tok 0-7, ch 2ks), (tok 8-15, 2ks), (tok 0-7, 2ks+1), (tok 8-15, 2ks+1)
+      const int tok = ((lane >> 3) & 1) * 8 + (lane & 7);
+      const int key = fast ? (tok & 7) : kk[tok];
       const uint32_t base = smem_u32(sK + tok * ROWB);
-      const int chb = (lane >> 3) & 1;
-#pragma unroll
-      for (int ks = 0; ks < KS; ++ks) {
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(base + ((((2 * ks + chb) ^ key)) << 4), b0, b1, b2, b3);
-        mma_bf16(sacc[0], qa[ks], b0, b1);
-        mma_bf16(sacc[1], qa[ks], b2, b3);
-      }
-    }
-    // online softmax (log2 domain), rows lane/4 and lane/4 + 8
-    float x[2][4];
-#pragma unroll
-    for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int tk = nt * 8 + 2 * (lane & 3) + (e & 1);
-        x[nt][e] = (t * 16 + tk < u.n_att) ? sacc[nt][e] * p.scale_log2 : kNegInf;
-      }
-    float corr[2];
-#pragma unroll
-    for (int hr = 0; hr < 2; ++hr) {
-      float mx = fmaxf(fmaxf(x[0][2 * hr], x[0][2 * hr + 1]), fmaxf(x[1][2 * hr], x[1][2 * hr + 1]));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-      mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-      const float mnew = fmaxf(m_run[hr], mx);
-      corr[hr] = (m_run[hr] == kNegInf) ? 0.f : fast_exp2(m_run[hr] - mnew);
-      m_run[hr] = mnew;
-    }
-    float pr[2][4];
-#pragma unroll
-    for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) pr[nt][e] = fast_exp2(x[nt][e] - m_run[e >> 1]);
-#pragma unroll
-    for (int hr = 0; hr < 2; ++hr)
-      l_run[hr] = l_run[hr] * corr[hr] + (pr[0][2 * hr] + pr[0][2 * hr + 1] + pr[1][2 * hr] + pr[1][2 * hr + 1]);
-#pragma unroll
-    for (int i = 0; i < D / 8; ++i) {
-      o[i][0] *= corr[0];
-      o[i][1] *= corr[0];
-      o[i][2] *= corr[1];
-      o[i][3] *= corr[1];
-    }
-    // P as a 16x16 A operand, split into bf16 hi + lo parts for ~16-bit precision
-    uint32_t ph[4], pl[4];
-    {
-      const float v[4][2] = {{pr[0][0], pr[0][1]}, {pr[0][2], pr[0][3]}, {pr[1][0], pr[1][1]}, {pr[1][2], pr[1][3]}};
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const __nv_bfloat162 hi = __floats2bfloat162_rn(v[i][0], v[i][1]);
-        const float2 hf = __bfloat1622float2(hi);
-        ph[i] = *reinterpret_cast<const uint32_t*>(&hi);
-        pl[i] = pack_bf16(v[i][0] - hf.x, v[i][1] - hf.y);
-      }
-    }
-    // O += P V
-    {
-      const int tok = (((lane >> 3) & 1) << 3) + (lane & 7);
-      const int key = kk[tok];
-      const uint32_t base = smem_u32(sV + tok * ROWB);
       const int chb = lane >> 4;
 #pragma unroll
-      for (int jj = 0; jj < D / 16; ++jj) {
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(base + ((((2 * jj + chb) ^ key)) << 4), b0, b1, b2, b3);
-        mma_bf16(o[2 * jj], ph, b0, b1);
-        mma_bf16(o[2 * jj], pl, b0, b1);
-        mma_bf16(o[2 * jj + 1], ph, b2, b3);
-        mma_bf16(o[2 * jj + 1], pl, b2, b3);
+      for (int ks = 0; ks < KS; ++ks) {
+        uint32_t a[4];
+        ldsm_x4(base + ((((2 * ks + chb) ^ key)) << 4), a[0], a[1], a[2], a[3]);
+#pragma unroll
+        for (int hn = 0; hn < HN; ++hn) mma_bf16(sc[hn][ks & 1], a, qb[hn][ks][0], qb[hn][ks][1]);
+      }
+    }
+    uint32_t pbh[HN][2], pbl[HN][2];
+    float corr[HN][2];
+#pragma unroll
+    for (int hn = 0; hn < HN; ++hn) {
+      float x[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int tk = r_tok + (e >> 1) * 8;
+        x[e] = (t * 16 + tk < u.n_att) ? (sc[hn][0][e] + sc[hn][1][e]) * p.scale_log2 : kNegInf;
+      }
+      float pr[4];
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {  // this thread's two heads
+        float mx = fmaxf(x[e], x[e + 2]);
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+        const float mnew = fmaxf(m_run[hn][e], mx);
+        corr[hn][e] = (m_run[hn][e] == kNegInf) ? 0.f : fast_exp2(m_run[hn][e] - mnew);
+        m_run[hn][e] = mnew;
+        pr[e] = fast_exp2(x[e] - mnew);
+        pr[e + 2] = fast_exp2(x[e + 2] - mnew);
+        l_run[hn][e] = l_run[hn][e] * corr[hn][e] + pr[e] + pr[e + 2];
+      }
+      // P^T operand (k = tokens, n = heads): transpose the 8x8 blocks of P
+      const __nv_bfloat162 h01 = __floats2bfloat162_rn(pr[0], pr[1]);
+      const __nv_bfloat162 h23 = __floats2bfloat162_rn(pr[2], pr[3]);
+      const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+      pbh[hn][0] = movmatrix_t(*reinterpret_cast<const uint32_t*>(&h01));
+      pbh[hn][1] = movmatrix_t(*reinterpret_cast<const uint32_t*>(&h23));
+      pbl[hn][0] = movmatrix_t(pack_bf16(pr[0] - f01.x, pr[1] - f01.y));
+      pbl[hn][1] = movmatrix_t(pack_bf16(pr[2] - f23.x, pr[3] - f23.y));
+    }
+#pragma unroll
+    for (int mt = 0; mt < KS; ++mt)
+#pragma unroll
+      for (int hn = 0; hn < HN; ++hn) {
+        o[mt][hn][0] *= corr[hn][0];
+        o[mt][hn][1] *= corr[hn][1];
+        o[mt][hn][2] *= corr[hn][0];
+        o[mt][hn][3] *= corr[hn][1];
+      }
+    {
+      // A = V^T tile: transposed matrices (tok 0-7, ch 2mt), (tok 0-7, 2mt+1), (tok 8-15, 2mt), (tok 8-15, 2mt+1)
+      const int tok = (lane >> 4) * 8 + (lane & 7);
+      const int key = fast ? (tok & 7) : kk[tok];
+      const uint32_t base = smem_u32(sV + tok * ROWB);
+      const int chb = (lane >> 3) & 1;
+#pragma unroll
+      for (int mt = 0; mt < KS; ++mt) {
+        uint32_t a[4];
+        ldsm_x4_t(base + ((((2 * mt + chb) ^ key)) << 4), a[0], a[1], a[2], a[3]);
+#pragma unroll
+        for (int hn = 0; hn < HN; ++hn) {
+          mma_bf16(o[mt][hn], a, pbh[hn][0], pbh[hn][1]);
+          mma_bf16(o[mt][hn], a, pbl[hn][0], pbl[hn][1]);
+        }
       }
     }
     __syncwarp();
-    if (j + kStages < nj) {
-      fence_proxy_async_smem();
-      __syncwarp();
-      issue_tile<ROWB>(u, s, t + kStages * kWarps, (const uint8_t*)kcache, (const uint8_t*)vcache, sK,
-                       sV, kk, &bar[st], lane);
+    if (j + NST < nj) {
+      issue(ic, j + NST);
+      advance(ic);
     }
+    cp_async_commit();  // one group per tile, empty near the end
+    advance(cc);
   }
-  if (!ok) {
-    // drain this warp's outstanding copies (bounded) before leaving
-    for (int st = 0; st < kStages; ++st) mbar_wait_bounded(&bar[st], (phase >> st) & 1u);
-  }
-
-  // warp partial -> shared memory
-#pragma unroll
-  for (int hr = 0; hr < 2; ++hr) {
-    l_run[hr] += __shfl_xor_sync(0xffffffffu, l_run[hr], 1);
-    l_run[hr] += __shfl_xor_sync(0xffffffffu, l_run[hr], 2);
-  }
-#pragma unroll
-  for (int hr = 0; hr < 2; ++hr) {
-    const int g = (lane >> 2) + 8 * hr;
-    if (g < G) {
-      float* dst = mw + (warp * G + g) * (D + 4);
-      if ((lane & 3) == 0) {
-        dst[0] = (ok && nj > 0) ? m_run[hr] : kNegInf;
-        dst[1] = (ok && nj > 0) ? l_run[hr] : 0.f;
-      }
-#pragma unroll
-      for (int i = 0; i < D / 8; ++i) {
-        dst[4 + i * 8 + 2 * (lane & 3)] = ok ? o[i][2 * hr] : 0.f;
-        dst[4 + i * 8 + 2 * (lane & 3) + 1] = ok ? o[i][2 * hr + 1] : 0.f;
-      }
-    }
-  }
-  if (u.t_begin < u.n_tiles) {
-    merge_and_store<D>(p, u, mw, kWarps);
-    // the CTA holding the appended row seals a full tail
-    if ((u.n_att - 1) / 16 >= u.t_begin && (u.n_att - 1) / 16 < u.t_end) {
-      __syncthreads();
-      seal_tail<bf16, D>(p, u, kcache);
-    }
-  } else if (p.n_split > 1) {
-    // empty chunk: contribute nothing to the merge but take a ticket
-    for (int i = threadIdx.x; i < G * (D + 4); i += blockDim.x) mw[i] = (i % (D + 4) == 0) ? kNegInf : 0.f;
-    merge_and_store<D>(p, u, mw, 1);
-  }
+  cp_async_wait<0>();
+  if (have) flush();
   finish_grid(p);
 }
 
@@ -663,7 +1010,7 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const __grid_constant__ A
     merge_and_store<D>(p, u, mw, kWarps);
     if ((u.n_att - 1) / 16 >= u.t_begin && (u.n_att - 1) / 16 < u.t_end) {
       __syncthreads();
-      seal_tail<float, D>(p, u, kcache);
+      if (threadIdx.x < 32) seal_tail<float, D>(p, u, kcache);
     }
   } else if (p.n_split > 1) {
     for (int i = threadIdx.x; i < G * (D + 4); i += blockDim.x) mw[i] = (i % (D + 4) == 0) ? kNegInf : 0.f;
@@ -675,9 +1022,15 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const __grid_constant__ A
 // ------------------------------------------------------------- launch ----
 
 int attn_smem_bytes(int dtype, int D, int G) {
-  if (dtype == MPC_BF16) return D == 64 ? Smem<64, 2>::total(G) : Smem<128, 2>::total(G);
+  if (dtype == MPC_BF16) {
+    const int nst = persist_stages(D, G);
+    return D == 64 ? PSmem<64>::total(G, nst, kMaxBatchPersist) : PSmem<128>::total(G, nst, kMaxBatchPersist);
+  }
   return D == 64 ? Smem<64, 4>::total(G) : Smem<128, 4>::total(G);
 }
+
+int attn_persist_ctas_max() { return kMaxPersistCtas; }
+int attn_persist_batch_max() { return kMaxBatchPersist; }
 
 template <typename K>
 static cudaError_t launch_k(K kernel, dim3 grid, int smem, cudaStream_t st, const AttnParams& p) {
@@ -687,13 +1040,37 @@ static cudaError_t launch_k(K kernel, dim3 grid, int smem, cudaStream_t st, cons
   return cudaGetLastError();
 }
 
-cudaError_t launch_attn(const AttnParams& p, int dtype, int D, int n_units, cudaStream_t st) {
+// CTAs of the persistent grid: one per SM, at most kMaxPersistCtas.
+static int persist_ctas() {
+  static std::mutex mu;
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return kMaxPersistCtas;
+  std::lock_guard<std::mutex> lk(mu);
+  if (cached[dev] == 0) {
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
+      sms = kMaxPersistCtas;
+    cached[dev] = sms < kMaxPersistCtas ? sms : kMaxPersistCtas;
+  }
+  return cached[dev];
+}
+
+cudaError_t launch_attn(const AttnParams& p0, int dtype, int D, int n_units, cudaStream_t st) {
+  AttnParams p = p0;
+  if (dtype == MPC_BF16) {
+    p.n_stages = persist_stages(D, p.G);
+    const int smem = attn_smem_bytes(dtype, D, p.G);
+    const dim3 grid(persist_ctas());
+    if (p.G <= 8) {
+      if (D == 64) return launch_k(attn_bf16_persist_kernel<64, 1, 8>, grid, smem, st, p);
+      return launch_k(attn_bf16_persist_kernel<128, 1, 5>, grid, smem, st, p);
+    }
+    if (D == 64) return launch_k(attn_bf16_persist_kernel<64, 2, 8>, grid, smem, st, p);
+    return launch_k(attn_bf16_persist_kernel<128, 2, 4>, grid, smem, st, p);
+  }
   const dim3 grid(p.n_split, n_units);
   const int smem = attn_smem_bytes(dtype, D, p.G);
-  if (dtype == MPC_BF16) {
-    if (D == 64) return launch_k(attn_bf16_kernel<64>, grid, smem, st, p);
-    return launch_k(attn_bf16_kernel<128>, grid, smem, st, p);
-  }
   const int G = p.G;
 #define MPC_F32_CASE(DD, GG) \
   if (D == DD && G <= GG) return launch_k(attn_f32_kernel<DD, GG>, grid, smem, st, p);

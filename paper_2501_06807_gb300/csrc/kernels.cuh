@@ -31,8 +31,9 @@ struct AttnParams {
   float scale_log2;  // softmax scale times log2(e)
   float* out;
   int64_t out_ls;
-  int n_split, tiles_per_split;
-  float* part;        // [unit][split][G][D + 4]
+  int n_split, tiles_per_split;  // split grid (fp32)
+  int n_stages;                  // ring depth per warp (persistent bf16 kernel)
+  float* part;        // fp32: [unit][split][G][D + 4]; bf16: [2 * warps][G][D + 4]
   int* unit_counter;  // [unit]
   int* grid_counter;  // [1]
 };
@@ -117,6 +118,8 @@ struct ClusterParams {
 
 cudaError_t launch_attn(const AttnParams& p, int dtype, int D, int n_units, cudaStream_t st);
 int attn_smem_bytes(int dtype, int D, int G);
+int attn_persist_ctas_max();
+int attn_persist_batch_max();
 cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cudaStream_t st);
 int select_smem_bytes(int D, int max_cand);
 cudaError_t launch_clusters(const ClusterParams& p, int dtype, int D, int n_units, int groups_x,

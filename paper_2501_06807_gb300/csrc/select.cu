@@ -57,7 +57,8 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
   float* score = reinterpret_cast<float*>(cand + MC);
   int* kept = reinterpret_cast<int*>(score + MC);
   __shared__ int warp_tot[32];
-  __shared__ int s_total, s_ncand, s_nkept;
+  __shared__ int s_total, s_ncand;
+  __shared__ unsigned long long s_thr;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int unit = blockIdx.x;
@@ -88,30 +89,50 @@ __global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_consta
   int nk = 0;
   for (int l = top; l >= 0 && !overflow; --l) {
     const int n_cand = s_ncand;
-    // Eq. 3 similarity of every candidate
+    // Eq. 3 similarity of every candidate: a warp takes 4 candidates at a
+    // time so that four independent row loads are in flight per lane
     const float* rep = p.rep + (ubase + p.pyr.off[l]) * D;
-    for (int i = warp; i < n_cand; i += kSelThreads / 32) {
-      const float* row = rep + (int64_t)cand[i] * D;
-      float acc = 0.f;
+    for (int i0 = warp * 4; i0 < n_cand; i0 += (kSelThreads / 32) * 4) {
+      float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
       for (int c4 = lane; c4 < D / 4; c4 += 32) {
-        const float4 r = *reinterpret_cast<const float4*>(row + 4 * c4);
         const float4 qv = *reinterpret_cast<const float4*>(qsum + 4 * c4);
-        acc = fmaf(r.x, qv.x, acc);
-        acc = fmaf(r.y, qv.y, acc);
-        acc = fmaf(r.z, qv.z, acc);
-        acc = fmaf(r.w, qv.w, acc);
+        float4 r[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          r[u] = (i0 + u < n_cand) ? __ldg(reinterpret_cast<const float4*>(rep + (int64_t)cand[i0 + u] * D) + c4)
+                                   : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          acc[u] = fmaf(r[u].x, qv.x, acc[u]);
+          acc[u] = fmaf(r[u].y, qv.y, acc[u]);
+          acc[u] = fmaf(r[u].z, qv.z, acc[u]);
+          acc[u] = fmaf(r[u].w, qv.w, acc[u]);
+        }
       }
-      acc = warp_sum(acc);
-      if (lane == 0) {
-        score[i] = acc;
-        keys[i] = sel_key(acc, cand[i]);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) acc[u] = warp_sum(acc[u]);
+      if (lane < 4 && i0 + lane < n_cand) {
+        const float a = lane == 0 ? acc[0] : lane == 1 ? acc[1] : lane == 2 ? acc[2] : acc[3];
+        score[i0 + lane] = a;
+        keys[i0 + lane] = sel_key(a, cand[i0 + lane]);
       }
     }
     const int k = min(count_from_ppm(C[l], p.keep_ppm[l]), n_cand);
     __syncthreads();
     unsigned long long thr = 0ull;
-    if (k < n_cand) {
+    if (k < n_cand && n_cand <= 2 * kSelThreads) {
+      // rank of each candidate = number of larger keys (keys are distinct);
+      // the key of rank k - 1 is the k-th largest
+      for (int i = tid; i < n_cand; i += blockDim.x) {
+        const unsigned long long ki = keys[i];
+        int rank = 0;
+        for (int j = 0; j < n_cand; ++j) rank += keys[j] > ki;
+        if (rank == k - 1) s_thr = ki;
+      }
+      __syncthreads();
+      thr = s_thr;
+    } else if (k < n_cand) {
       int P = 1;
       while (P < n_cand) P <<= 1;
       for (int i = n_cand + tid; i < P; i += blockDim.x) keys[i] = 0ull;
