@@ -247,6 +247,20 @@ int validate_select(const mpc_select_args* a, SelectParams* p) {
   p->out_sel = a->out_sel;
   p->out_n_sel = a->out_n_sel;
   p->max_cand = P;
+  // rows staged in shared memory at once: the first round (the coarsest
+  // level plus the level below it) and each later round (the children of a
+  // level's kept clusters), capped by what shared memory holds
+  const int top = a->n_levels - 1;
+  long long need = (long long)p->pyr.cap[top] + (top > 0 ? p->pyr.cap[top - 1] : 0);
+  for (int l = top - 2; l >= 0; --l) {
+    long long r = (long long)p->pyr.fanout[l] * kmax[l + 1];
+    if (r > p->pyr.cap[l]) r = p->pyr.cap[l];
+    if (r > need) need = r;
+  }
+  const long long budget =
+      (kSmemOptin - 256 - (long long)select_smem_bytes(a->head_dim, P, 0)) / ((long long)a->head_dim * 4 + 4);
+  if (budget < 1) return fail(MPC_ERR_BAD_SHAPE, "%d candidates leave no shared memory to stage representatives", P);
+  p->row_buf = (int)(need < budget ? need : budget);
   return MPC_OK;
 }
 

@@ -17,6 +17,7 @@ typedef __nv_bfloat16 bf16;
 
 constexpr int kMaxRefs = MPC_MAX_REFS;
 constexpr int kMaxLevels = MPC_MAX_LEVELS;
+constexpr int kSmemOptin = 232448;  // shared memory per CTA on sm_103a (227 KB)
 
 constexpr float kPosInf = __builtin_huge_valf();
 constexpr float kNegInf = -__builtin_huge_valf();
@@ -132,6 +133,33 @@ static inline int take_status() {
   if (cudaMemcpyFromSymbol(&v, g_mpc_status, sizeof(int)) != cudaSuccess) return -1;
   if (cudaMemcpyToSymbol(g_mpc_status, &z, sizeof(int)) != cudaSuccess) return -1;
   return v;
+}
+
+// Programmatic dependent launch.  The per-step kernels are launched with
+// cudaLaunchAttributeProgrammaticStreamSerialization, so a kernel may become
+// resident while the previous kernel of the stream is still running.  Every
+// such kernel calls grid_dep_wait() before its first access to global memory
+// that an earlier launch may write; grid_dep_wait() returns once all earlier
+// grids have completed and their writes are visible (a no-op for a kernel
+// launched without the attribute).  grid_dep_launch() lets the next kernel of
+// the stream start its own launch early.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... P, typename... A>
+inline cudaError_t launch_pdl(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                              A&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<A>(args)...);
 }
 
 // Raises a kernel's dynamic shared-memory limit once per (kernel, device), so

@@ -368,6 +368,8 @@ __global__ void __launch_bounds__(128, 1) attn_bf16_persist_kernel(const __grid_
   int* s_pre = s_nt + B;                                           // exclusive prefix of s_nt (B + 1)
   int* s_n = s_pre + B + 1;                                        // cache rows before the append
   int* s_k1 = s_n + B;                                             // selected clusters
+  grid_dep_launch();
+  grid_dep_wait();
 
   // ---- per-sequence table
   if (warp == 0) {
@@ -848,6 +850,8 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const __grid_constant__ A
   constexpr int PER = D / 32;  // output channels per lane
   extern __shared__ __align__(128) uint8_t smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  grid_dep_launch();
+  grid_dep_wait();
   const Unit u = make_unit(p);
   const int s = p.pyr.s;
   const int G = p.G;
@@ -1036,8 +1040,7 @@ template <typename K>
 static cudaError_t launch_k(K kernel, dim3 grid, int smem, cudaStream_t st, const AttnParams& p) {
   cudaError_t e = ensure_dyn_smem((const void*)kernel, smem);
   if (e != cudaSuccess) return e;
-  kernel<<<grid, 128, smem, st>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(kernel, grid, dim3(128), smem, st, p);
 }
 
 // CTAs of the persistent grid: one per SM, at most kMaxPersistCtas.

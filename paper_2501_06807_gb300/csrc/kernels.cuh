@@ -51,6 +51,7 @@ struct SelectParams {
   int* out_sel;
   int* out_n_sel;
   int max_cand;  // power of two, capacity of the shared candidate arrays
+  int row_buf;   // representative rows staged in shared memory at once
 };
 
 struct StaticParams {
@@ -121,7 +122,7 @@ int attn_smem_bytes(int dtype, int D, int G);
 int attn_persist_ctas_max();
 int attn_persist_batch_max();
 cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cudaStream_t st);
-int select_smem_bytes(int D, int max_cand);
+int select_smem_bytes(int D, int max_cand, int row_buf);
 cudaError_t launch_clusters(const ClusterParams& p, int dtype, int D, int n_units, int groups_x,
                             bool any_leader, cudaStream_t st);
 cudaError_t launch_static(const StaticParams& p, int dtype, int D, int n_layer_span, cudaStream_t st);

@@ -3,217 +3,375 @@
 //
 // One CTA per (ref, sequence b, kv head h).  The GQA group's queries are
 // summed once (Eq. 3 is linear in q, so the sum scores the group), then the
-// levels are walked from the coarsest down: a warp per candidate computes
-// q_sum . rep over d channels (float4 loads of the fp32 representative), a
-// block bitonic sort of 64-bit keys (orderable score, inverted id) finds the
-// k-th key, and an order-preserving compaction keeps the candidates at or
-// above it, so the kept ids stay ascending.  The children of the kept
-// clusters are the next level's candidates.
+// levels are walked from the coarsest down.  Each candidate is held as one
+// 64-bit key (orderable score, inverted id: all keys distinct, larger score
+// first, then smaller id), so the key alone carries the id and the score.
+//
+// The walk is bounded by global-load latency, so the fp32 representatives
+// a level needs are staged in shared memory by 1-D bulk copies (contiguous
+// runs: the whole coarsest level, or the children of one kept cluster) on
+// one mbarrier, and scoring is batched into as few dependent rounds as the
+// pyramid allows.  The first round, requested before q and the token count
+// arrive, copies the coarsest level and, when they fit the staging buffer,
+// all clusters of the level below it, whose scores then need no round of
+// their own (a three-level pyramid takes two rounds).  Per level, with a
+// block barrier after each step:
+//   1. rank: a candidate is kept iff fewer than k keys are larger, counted
+//      by up to 32 threads per candidate over shared memory (a bitonic sort
+//      of a copy gives the k-th key instead above 1024 candidates);
+//   2. warp 0 compacts the kept positions in candidate order with ballots,
+//      so the kept ids stay ascending;
+//   3. the block writes the kept clusters' children as the next level's
+//      keys, with their scores when the first round computed them.
 #include "kernels.cuh"
 
 namespace mpc {
 
-
-constexpr int kSelThreads = 256;
+constexpr int kRankMax = 1024;  // candidates ranked by counting
+constexpr int kSelChunk = 8192; // bytes per bulk copy
 
 __device__ __forceinline__ unsigned long long sel_key(float score, int id) {
   return ((unsigned long long)orderable(score) << 32) | (unsigned long long)(0xffffffffu - (uint32_t)id);
 }
-
-// Exclusive prefix sum over the block (blockDim.x == kSelThreads).
-__device__ __forceinline__ int block_exclusive_scan(int v, int* warp_tot, int* total) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  int x = v;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, x, o);
-    if (lane >= o) x += y;
-  }
-  if (lane == 31) warp_tot[warp] = x;
-  __syncthreads();
-  if (warp == 0) {
-    int t = (lane < kSelThreads / 32) ? warp_tot[lane] : 0;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, t, o);
-      if (lane >= o) t += y;
-    }
-    if (lane < kSelThreads / 32) warp_tot[lane] = t;
-    if (lane == kSelThreads / 32 - 1) *total = t;
-  }
-  __syncthreads();
-  const int before = (warp > 0 ? warp_tot[warp - 1] : 0) + x - v;
-  __syncthreads();
-  return before;
+__device__ __forceinline__ int key_id(unsigned long long key) {
+  return (int)(0xffffffffu - (uint32_t)(key & 0xffffffffull));
 }
 
-template <typename T, int D>
-__global__ void __launch_bounds__(kSelThreads) select_kernel(const __grid_constant__ SelectParams p) {
-  extern __shared__ __align__(16) uint8_t smem[];
-  const int MC = p.max_cand;
-  float* qsum = reinterpret_cast<float*>(smem);
-  unsigned long long* keys = reinterpret_cast<unsigned long long*>(qsum + D);
-  int* cand = reinterpret_cast<int*>(keys + MC);
-  float* score = reinterpret_cast<float*>(cand + MC);
-  int* kept = reinterpret_cast<int*>(score + MC);
-  __shared__ int warp_tot[32];
-  __shared__ int s_total, s_ncand;
-  __shared__ unsigned long long s_thr;
+// Shared-memory layout of one select CTA (host and device).
+struct SelLayout {
+  size_t qsum, cs, keys, mark, kept, total;
+  __host__ __device__ SelLayout(int D, int MC, int RB) {
+    qsum = (size_t)RB * D * 4;             // staged rows first (16-byte aligned)
+    cs = qsum + (size_t)D * 4;              // scores of the first round's children
+    keys = (cs + (size_t)RB * 4 + 15) & ~(size_t)15;
+    mark = keys + (size_t)MC * 16;          // two key arrays
+    kept = mark + (size_t)MC * 4;
+    total = kept + (size_t)MC * 4;
+  }
+};
+
+// Warp-cooperative copy of nbytes (a multiple of 16) in chunks, lanes in
+// parallel, completing on bar.
+__device__ __forceinline__ void warp_copy(void* dst, const void* src, uint32_t nbytes, uint64_t* bar, int lane) {
+  for (uint32_t off = (uint32_t)lane * kSelChunk; off < nbytes; off += 32u * kSelChunk) {
+    const uint32_t nb = nbytes - off < (uint32_t)kSelChunk ? nbytes - off : (uint32_t)kSelChunk;
+    bulk_g2s(static_cast<uint8_t*>(dst) + off, static_cast<const uint8_t*>(src) + off, nb, bar);
+  }
+}
+
+template <typename T, int D, int NT>
+__global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ SelectParams p) {
+  constexpr int NW = NT / 32;
+  constexpr int LPR = D / 4;     // lanes per representative row (one float4 each)
+  constexpr int RPW = 32 / LPR;  // rows per warp-wide read
+  constexpr int U = 8;           // rows per lane per pass
+  constexpr uint32_t ROWB = D * 4;
+  extern __shared__ __align__(128) uint8_t smem[];
+  const int MC = p.max_cand, RB = p.row_buf;
+  const SelLayout L(D, MC, RB);
+  float* rows = reinterpret_cast<float*>(smem);
+  float* qsum = reinterpret_cast<float*>(smem + L.qsum);
+  float* cs = reinterpret_cast<float*>(smem + L.cs);
+  unsigned long long* keysA = reinterpret_cast<unsigned long long*>(smem + L.keys);
+  unsigned long long* keysB = keysA + MC;
+  int* mark = reinterpret_cast<int*>(smem + L.mark);
+  int* kept = reinterpret_cast<int*>(smem + L.kept);
+  __shared__ __align__(8) uint64_t s_bar;
+  __shared__ int s_C[kMaxLevels], s_k[kMaxLevels];
+  __shared__ int s_nk, s_next;
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int c4 = lane % LPR, sub = lane / LPR;
   const int unit = blockIdx.x;
   const int h = unit % p.Hkv, b = (unit / p.Hkv) % p.B, ri = unit / (p.Hkv * p.B);
   const int layer = p.refs.layer[ri], group = p.refs.group[ri];
   const int G = p.G;
+  const int top = p.pyr.n_levels - 1;
+  const float* rep0 = p.rep + ((int64_t)(group * p.B + b) * p.Hkv + h) * p.pyr.rows * D;
+  int* out = p.out_sel + ((int64_t)(group * p.B + b) * p.Hkv + h) * p.sel_cap;
+  uint32_t phase = 0;
+  bool timed_out = false;
+
+  // q_sum . (staged row r) for rows [0, nrows) of the buffer; put(r, score)
+  // runs on the first lane of each row.  Channel order is fixed: x, y, z, w
+  // per lane, then a butterfly over the row's lanes.
+  auto score_rows = [&](int nrows, auto&& put) {
+    const float4 qv = reinterpret_cast<const float4*>(qsum)[c4];
+    for (int r0 = warp * U * RPW; r0 < nrows; r0 += NW * U * RPW) {
+      float acc[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int r = r0 + u * RPW + sub;
+        const float4 v = r < nrows ? reinterpret_cast<const float4*>(rows + (size_t)r * D)[c4]
+                                   : make_float4(0.f, 0.f, 0.f, 0.f);
+        float a = 0.f;
+        a = fmaf(v.x, qv.x, a);
+        a = fmaf(v.y, qv.y, a);
+        a = fmaf(v.z, qv.z, a);
+        a = fmaf(v.w, qv.w, a);
+        acc[u] = a;
+      }
+#pragma unroll
+      for (int o = LPR / 2; o > 0; o >>= 1) {
+#pragma unroll
+        for (int u = 0; u < U; ++u) acc[u] += __shfl_xor_sync(0xffffffffu, acc[u], o);
+      }
+      if (c4 == 0) {
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          const int r = r0 + u * RPW + sub;
+          if (r < nrows) put(r, acc[u]);
+        }
+      }
+    }
+  };
+  auto wait_rows = [&]() {
+    if (!mbar_wait_bounded(&s_bar, phase)) timed_out = true;
+    phase ^= 1u;
+  };
+
+  if (tid == 0) {
+    mbar_init(&s_bar, 1);
+    fence_barrier_init();
+  }
+  grid_dep_launch();
+  grid_dep_wait();
+
+  // ---- first round, requested up front: rows [0, nT0) of the coarsest
+  // level at buffer row 0 and, when spec0, rows [0, capC) of the level
+  // below it at buffer row capT
+  const int capT = p.pyr.cap[top];
+  const int capC = top > 0 ? p.pyr.cap[top - 1] : 0;
+  const bool spec0 = top > 0 && capT + capC <= RB;
+  const int nT0 = capT < RB ? capT : RB;
+  const float* repT = rep0 + (int64_t)p.pyr.off[top] * D;
+  const float* repC = rep0 + (int64_t)(top > 0 ? p.pyr.off[top - 1] : 0) * D;
+  if (warp == 0) {
+    if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)(nT0 + (spec0 ? capC : 0)) * ROWB);
+    __syncwarp();
+    warp_copy(rows, repT, (uint32_t)nT0 * ROWB, &s_bar, lane);
+    if (spec0) warp_copy(rows + (size_t)capT * D, repC, (uint32_t)capC * ROWB, &s_bar, lane);
+  }
+  const int ntok = p.n_tok[b];
 
   // q_sum = sum over the group's query heads (fixed order)
   const T* qp = (const T*)p.q + layer * p.q_ls + ((int64_t)b * p.Hq + h * G) * D;
-  for (int c = tid; c < D; c += blockDim.x) {
+  for (int c = tid; c < D; c += NT) {
     float acc = 0.f;
     for (int g = 0; g < G; ++g) acc += to_float<T>(qp[g * D + c]);
     qsum[c] = acc;
   }
-
   int C[kMaxLevels];
-  level_counts(p.pyr, p.n_tok[b], C);
-  const int64_t ubase = ((int64_t)(group * p.B + b) * p.Hkv + h) * p.pyr.rows;
-  int* out = p.out_sel + ((int64_t)(group * p.B + b) * p.Hkv + h) * p.sel_cap;
-
-  const int top = p.pyr.n_levels - 1;
-  bool overflow = C[0] > p.pyr.cap[0];
-  if (tid == 0) s_ncand = min(C[top], MC);
-  if (C[top] > MC) overflow = true;
-  for (int i = tid; i < min(C[top], MC); i += blockDim.x) cand[i] = i;
+  level_counts(p.pyr, ntok, C);
+  if (tid < kMaxLevels) {
+    s_C[tid] = C[tid];
+    s_k[tid] = tid < p.pyr.n_levels ? count_from_ppm(C[tid], p.keep_ppm[tid]) : 0;
+  }
+  bool overflow = C[0] > p.pyr.cap[0] || C[top] > MC;
   __syncthreads();
+  wait_rows();
+
+  int n = overflow ? 0 : C[top];
+  {
+    const int nC = top > 0 ? C[top - 1] : 0;
+    const int own = n < nT0 ? n : nT0;
+    score_rows(spec0 ? capT + nC : own, [&](int r, float sc) {
+      if (r < own) keysA[r] = sel_key(sc, r);
+      else if (r >= capT) cs[r - capT] = sc;
+    });
+    __syncthreads();
+    // the rest of a coarsest level larger than the buffer
+    for (int x0 = nT0; x0 < n; x0 += RB) {
+      const int nb = min(RB, n - x0);
+      if (warp == 0) {
+        if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)nb * ROWB);
+        __syncwarp();
+        warp_copy(rows, repT + (int64_t)x0 * D, (uint32_t)nb * ROWB, &s_bar, lane);
+      }
+      wait_rows();
+      score_rows(nb, [&](int r, float sc) { keysA[x0 + r] = sel_key(sc, x0 + r); });
+      __syncthreads();
+    }
+  }
+  bool have_child = spec0;  // cs holds the scores of all children of keysA[0, n)
+  bool need_score = false;  // keysA holds ids only
 
   int nk = 0;
   for (int l = top; l >= 0 && !overflow; --l) {
-    const int n_cand = s_ncand;
-    // Eq. 3 similarity of every candidate: a warp takes 4 candidates at a
-    // time so that four independent row loads are in flight per lane
-    const float* rep = p.rep + (ubase + p.pyr.off[l]) * D;
-    for (int i0 = warp * 4; i0 < n_cand; i0 += (kSelThreads / 32) * 4) {
-      float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int c4 = lane; c4 < D / 4; c4 += 32) {
-        const float4 qv = *reinterpret_cast<const float4*>(qsum + 4 * c4);
-        float4 r[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-          r[u] = (i0 + u < n_cand) ? __ldg(reinterpret_cast<const float4*>(rep + (int64_t)cand[i0 + u] * D) + c4)
-                                   : make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          acc[u] = fmaf(r[u].x, qv.x, acc[u]);
-          acc[u] = fmaf(r[u].y, qv.y, acc[u]);
-          acc[u] = fmaf(r[u].z, qv.z, acc[u]);
-          acc[u] = fmaf(r[u].w, qv.w, acc[u]);
+    const int f = l > 0 ? p.pyr.fanout[l - 1] : 1;
+    const int nC = l > 0 ? s_C[l - 1] : 0;
+    if (need_score) {
+      // a round over the candidates' own rows, in batches of RB rows; the
+      // candidates are the children of the kept clusters of level l + 1, so
+      // every run of fl consecutive candidates is one run of rows
+      const int fl = p.pyr.fanout[l];
+      const float* repL = rep0 + (int64_t)p.pyr.off[l] * D;
+      for (int x0 = 0; x0 < n; x0 += RB) {
+        const int x1 = min(n, x0 + RB);
+        if (warp == 0) {
+          if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)(x1 - x0) * ROWB);
+          __syncwarp();
+          for (int kk = x0 / fl + lane; kk * fl < x1; kk += 32) {
+            const int s0 = max(x0, kk * fl), s1 = min(x1, kk * fl + fl);
+            bulk_g2s(rows + (size_t)(s0 - x0) * D, repL + (int64_t)key_id(keysA[s0]) * D, (uint32_t)(s1 - s0) * ROWB,
+                     &s_bar);
+          }
         }
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u) acc[u] = warp_sum(acc[u]);
-      if (lane < 4 && i0 + lane < n_cand) {
-        const float a = lane == 0 ? acc[0] : lane == 1 ? acc[1] : lane == 2 ? acc[2] : acc[3];
-        score[i0 + lane] = a;
-        keys[i0 + lane] = sel_key(a, cand[i0 + lane]);
+        wait_rows();
+        score_rows(x1 - x0, [&](int r, float sc) { keysA[x0 + r] = sel_key(sc, key_id(keysA[x0 + r])); });
+        __syncthreads();
       }
     }
-    const int k = min(count_from_ppm(C[l], p.keep_ppm[l]), n_cand);
-    __syncthreads();
-    unsigned long long thr = 0ull;
-    if (k < n_cand && n_cand <= 2 * kSelThreads) {
-      // rank of each candidate = number of larger keys (keys are distinct);
-      // the key of rank k - 1 is the k-th largest
-      for (int i = tid; i < n_cand; i += blockDim.x) {
-        const unsigned long long ki = keys[i];
+
+    // 1. mark[i] = candidate i is among the k largest keys
+    const int k = min(s_k[l], n);
+    if (k >= n) {
+      for (int i = tid; i < n; i += NT) mark[i] = 1;
+    } else if (n <= kRankMax) {
+      int ncp = 1, sh = 0;
+      while (ncp < n) ncp <<= 1;
+      int tpc = NT / ncp;  // threads per candidate, a power of two
+      tpc = tpc < 1 ? 1 : (tpc > 32 ? 32 : tpc);
+      while ((1 << sh) < tpc) ++sh;
+      const int work = n * tpc;
+      const int work32 = (work + 31) & ~31;  // whole warps, so the shuffles see every lane
+      for (int x = tid; x < work32; x += NT) {
+        const int i = x >> sh, t = x & (tpc - 1);
         int rank = 0;
-        for (int j = 0; j < n_cand; ++j) rank += keys[j] > ki;
-        if (rank == k - 1) s_thr = ki;
+        if (x < work) {
+          const unsigned long long ki = keysA[i];
+          int j = t;
+          for (; j + 3 * tpc < n; j += 4 * tpc) {
+            const unsigned long long a0 = keysA[j], a1 = keysA[j + tpc], a2 = keysA[j + 2 * tpc], a3 = keysA[j + 3 * tpc];
+            rank += (int)(a0 > ki) + (int)(a1 > ki) + (int)(a2 > ki) + (int)(a3 > ki);
+          }
+          for (; j < n; j += tpc) rank += keysA[j] > ki;
+        }
+        for (int o = tpc >> 1; o > 0; o >>= 1) rank += __shfl_xor_sync(0xffffffffu, rank, o);
+        if (x < work && t == 0) mark[i] = rank < k;
       }
-      __syncthreads();
-      thr = s_thr;
-    } else if (k < n_cand) {
+    } else {
+      // bitonic sort (descending) of a copy of the keys gives the k-th key
       int P = 1;
-      while (P < n_cand) P <<= 1;
-      for (int i = n_cand + tid; i < P; i += blockDim.x) keys[i] = 0ull;
+      while (P < n) P <<= 1;
+      for (int i = tid; i < P; i += NT) keysB[i] = i < n ? keysA[i] : 0ull;
       __syncthreads();
-      // bitonic sort, descending
       for (int kk = 2; kk <= P; kk <<= 1) {
         for (int j = kk >> 1; j > 0; j >>= 1) {
-          for (int i = tid; i < P; i += blockDim.x) {
+          for (int i = tid; i < P; i += NT) {
             const int ixj = i ^ j;
             if (ixj > i) {
-              const unsigned long long a = keys[i], bb = keys[ixj];
+              const unsigned long long a = keysB[i], bb = keysB[ixj];
               const bool desc = (i & kk) == 0;
               if (desc ? (a < bb) : (a > bb)) {
-                keys[i] = bb;
-                keys[ixj] = a;
+                keysB[i] = bb;
+                keysB[ixj] = a;
               }
             }
           }
           __syncthreads();
         }
       }
-      thr = keys[k - 1];
+      const unsigned long long thr = keysB[k - 1];
+      for (int i = tid; i < n; i += NT) mark[i] = keysA[i] >= thr;
     }
-    // order-preserving compaction of the kept candidates
-    const int per = (n_cand + kSelThreads - 1) / kSelThreads;
-    const int i0 = tid * per, i1 = min(n_cand, i0 + per);
-    int cnt = 0;
-    for (int i = i0; i < i1; ++i) cnt += (sel_key(score[i], cand[i]) >= thr);
-    const int off = block_exclusive_scan(cnt, warp_tot, &s_total);
-    for (int i = i0, o = off; i < i1; ++i)
-      if (sel_key(score[i], cand[i]) >= thr) kept[o++] = cand[i];
     __syncthreads();
-    nk = s_total;
+
+    // 2. order-preserving compaction of the kept positions (warp 0)
+    if (warp == 0) {
+      const unsigned lt = (1u << lane) - 1u;
+      int nkw = 0;
+      for (int i0 = 0; i0 < n; i0 += 128) {
+        bool fl4[4];
+        unsigned bal[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) fl4[c] = i0 + 32 * c + lane < n && mark[i0 + 32 * c + lane] != 0;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) bal[c] = __ballot_sync(0xffffffffu, fl4[c]);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          if (fl4[c]) {
+            const int pos = nkw + __popc(bal[c] & lt);
+            kept[pos] = i0 + 32 * c + lane;
+            if (l == 0 && pos < p.sel_cap) out[pos] = key_id(keysA[i0 + 32 * c + lane]);
+          }
+          nkw += __popc(bal[c]);
+        }
+      }
+      if (lane == 0) {
+        s_nk = nkw;
+        // children of the kept clusters: all full except possibly the last
+        // cluster of the level, which can only be the last kept one
+        int nxt = 0;
+        if (l > 0 && nkw > 0) {
+          const int last = key_id(keysA[kept[nkw - 1]]);
+          nxt = (nkw - 1) * f + min(f, nC - last * f);
+        }
+        s_next = nxt;
+      }
+    }
+    __syncthreads();
+    nk = s_nk;
     if (l == 0) break;
-    // children of the kept clusters become the next candidates
-    const int f = p.pyr.fanout[l - 1];
-    const int n_child = C[l - 1];
-    const int perk = (nk + kSelThreads - 1) / kSelThreads;
-    const int k0 = tid * perk, k1 = min(nk, k0 + perk);
-    int ccount = 0;
-    for (int i = k0; i < k1; ++i) ccount += min(f, n_child - kept[i] * f);
-    const int coff = block_exclusive_scan(ccount, warp_tot, &s_total);
-    if (s_total > MC) {
+
+    // 3. the next level's candidates: children of the kept clusters, in order
+    const int nn = s_next;
+    if (nn > MC) {
       overflow = true;
       break;
     }
-    for (int i = k0, o = coff; i < k1; ++i) {
-      const int c0 = kept[i] * f, c1 = min(c0 + f, n_child);
-      for (int c = c0; c < c1; ++c) cand[o++] = c;
+    for (int x = tid; x < nn; x += NT) {
+      const int kk = x / f, j = x - kk * f;
+      const int i = kept[kk];
+      const int id = key_id(keysA[i]) * f + j;
+      keysB[x] = have_child ? sel_key(cs[i * f + j], id) : sel_key(0.f, id);
     }
-    if (tid == 0) s_ncand = s_total;
+    need_score = !have_child;
+    have_child = false;
+    n = nn;
     __syncthreads();
+    unsigned long long* t = keysA;
+    keysA = keysB;
+    keysB = t;
   }
-  if (overflow || nk > p.sel_cap) {
+  if (overflow || timed_out || nk > p.sel_cap) {
     if (tid == 0) atomicOr(&g_mpc_status, 4);
     nk = 0;
   }
-  for (int i = tid; i < p.sel_cap; i += blockDim.x) out[i] = (i < nk) ? kept[i] : -1;
+  for (int i = tid; i < p.sel_cap; i += NT)
+    if (i >= nk) out[i] = -1;
   if (tid == 0 && h == 0 && ri == 0) p.out_n_sel[b] = nk;
 }
 
-int select_smem_bytes(int D, int max_cand) {
-  return D * 4 + max_cand * (8 + 4 + 4 + 4);
-}
+// Threads per CTA: 16 warps while the units fit one wave of SMs, else 8.
+static int select_threads(int units) { return units <= 152 ? 512 : 256; }
+
+int select_smem_bytes(int D, int max_cand, int row_buf) { return (int)SelLayout(D, max_cand, row_buf).total; }
 
 template <typename K>
-static cudaError_t launch_sel(K kernel, int units, int smem, cudaStream_t st, const SelectParams& p) {
+static cudaError_t launch_sel(K kernel, int units, int nt, int smem, cudaStream_t st, const SelectParams& p) {
   cudaError_t e = ensure_dyn_smem((const void*)kernel, smem);
   if (e != cudaSuccess) return e;
-  kernel<<<units, kSelThreads, smem, st>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(kernel, dim3(units), dim3(nt), smem, st, p);
 }
 
 cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cudaStream_t st) {
-  const int smem = select_smem_bytes(D, p.max_cand);
-  if (dtype == MPC_BF16) {
-    if (D == 64) return launch_sel(select_kernel<bf16, 64>, units, smem, st, p);
-    return launch_sel(select_kernel<bf16, 128>, units, smem, st, p);
+  const int smem = select_smem_bytes(D, p.max_cand, p.row_buf);
+  const int nt = select_threads(units);
+#define MPC_SEL(TT, DD)                                                                     \
+  if (D == DD) {                                                                            \
+    if (nt == 512) return launch_sel(select_kernel<TT, DD, 512>, units, nt, smem, st, p);  \
+    return launch_sel(select_kernel<TT, DD, 256>, units, nt, smem, st, p);                 \
   }
-  if (D == 64) return launch_sel(select_kernel<float, 64>, units, smem, st, p);
-  return launch_sel(select_kernel<float, 128>, units, smem, st, p);
+  if (dtype == MPC_BF16) {
+    MPC_SEL(bf16, 64)
+    MPC_SEL(bf16, 128)
+  } else {
+    MPC_SEL(float, 64)
+    MPC_SEL(float, 128)
+  }
+#undef MPC_SEL
+  return cudaErrorInvalidValue;
 }
 
 int take_status_select() { return take_status(); }
