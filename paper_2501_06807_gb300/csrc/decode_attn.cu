@@ -302,10 +302,12 @@ __device__ __forceinline__ void finish_grid(const AttnParams& p) {
 // movmatrix (an in-register 8x8 transpose).
 //
 // A unit finished inside one warp is written directly.  A unit split across
-// warps leaves partial (max, sum, o) records, two slots per warp (2 slot: the
-// warp's first piece when its unit began earlier, 2 slot + 1: its last piece
-// when the unit continues), and the warp that completes the unit's ticket
-// count merges them by log-sum-exp.
+// warps is merged by its owner, the warp holding its first piece: that piece
+// ends its warp's range, so it finishes last in time.  Every later piece is
+// the first piece of its warp, finished early; it writes a partial (max,
+// sum, o) record (one slot per warp) and signals the owner with a release
+// reduction on the unit's counter, without waiting.  The owner waits (bounded)
+// for the count, then folds the records into its registers by log-sum-exp.
 
 constexpr int kMaxPersistCtas = 152;
 
@@ -328,15 +330,18 @@ struct PSmem {
   static __host__ __device__ constexpr int stage(int G) { return 2 * TILEB + qbytes(G); }
   static __host__ __device__ constexpr int key_off(int G, int nst) { return kWarps * nst * stage(G); }
   static __host__ __device__ constexpr int sel_off(int G, int nst) { return key_off(G, nst) + kWarps * nst * 16; }
-  static __host__ __device__ constexpr int scr_off(int G, int nst) { return sel_off(G, nst) + kWarps * kSelSmem * 4; }
-  static __host__ __device__ constexpr int tab_off(int G, int nst) { return scr_off(G, nst) + kWarps * 96 * 4; }
+  static __host__ __device__ constexpr int tab_off(int G, int nst) { return sel_off(G, nst) + kWarps * kSelSmem * 4; }
   static __host__ __device__ constexpr int total(int G, int nst, int B) { return tab_off(G, nst) + (4 * B + 2) * 4; }
 };
 
-// Ring depth per warp for a head dimension and GQA group size (compile-time
-// for cp.async.wait_group): 5 stages (d 128, up to 8 heads), 4 (d 128, up
-// to 16 heads), 8 (d 64).
-inline int persist_stages(int D, int G) { return D == 64 ? 8 : (G <= 8 ? 5 : 4); }
+// Ring depth per warp (compile-time for cp.async.wait_group): d 64 takes 8
+// stages; d 128 takes 6 when they fit shared memory with the batch's tables
+// (up to 8 heads per group), else 5 (up to 8 heads) or 4 (up to 16).
+inline int persist_stages(int D, int G, int B) {
+  if (D == 64) return 8;
+  if (G <= 8 && PSmem<128>::total(G, 6, B) <= kSmemOptin) return 6;
+  return G <= 8 ? 5 : 4;
+}
 
 struct Cursor {
   int ri, b, h, lt;
@@ -363,7 +368,6 @@ __global__ void __launch_bounds__(128, 1) attn_bf16_persist_kernel(const __grid_
   uint8_t* ring = smem + warp * NST * STAGE;
   int8_t* keys = reinterpret_cast<int8_t*>(smem + S::key_off(G, NST)) + warp * NST * 16;
   int* sel_s = reinterpret_cast<int*>(smem + S::sel_off(G, NST)) + warp * kSelSmem;
-  float* scr = reinterpret_cast<float*>(smem + S::scr_off(G, NST)) + warp * 96;  // merge scratch
   int* s_nt = reinterpret_cast<int*>(smem + S::tab_off(G, NST));  // tiles per unit of sequence b
   int* s_pre = s_nt + B;                                           // exclusive prefix of s_nt (B + 1)
   int* s_n = s_pre + B + 1;                                        // cache rows before the append
@@ -572,24 +576,11 @@ __global__ void __launch_bounds__(128, 1) attn_bf16_persist_kernel(const __grid_
     const int64_t uend = ustart + s_nt[u.b];
     const bool before = ustart < x0, after = uend > x1;
     float* outp = p.out + u.layer * p.out_ls + ((int64_t)u.b * p.Hq + u.h * G) * D;
-    if (!before && !after) {
-#pragma unroll
-      for (int hn = 0; hn < HN; ++hn)
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const int g = hn * 8 + h_off + e;
-          if (g < G) {
-            const float inv = 1.f / lq[hn][e];
-#pragma unroll
-            for (int mt = 0; mt < KS; ++mt) {
-              outp[g * D + mt * 16 + r_tok] = o[mt][hn][e] * inv;
-              outp[g * D + mt * 16 + r_tok + 8] = o[mt][hn][2 + e] * inv;
-            }
-          }
-        }
-    } else {
-      const int rec = 2 * gw + (before ? 0 : 1);
-      float* dst = p.part + (int64_t)rec * G * (D + 4);
+    const int64_t unit_id = ((int64_t)u_ri * B + u.b) * Hkv + u.h;
+    if (before) {
+      // a later piece of a unit that began in an earlier warp: publish the
+      // (max, sum, o) record and signal the unit's owner, without waiting
+      float* dst = p.part + (int64_t)gw * G * (D + 4);
 #pragma unroll
       for (int hn = 0; hn < HN; ++hn)
 #pragma unroll
@@ -607,82 +598,65 @@ __global__ void __launch_bounds__(128, 1) attn_bf16_persist_kernel(const __grid_
             }
           }
         }
-      __threadfence();
       __syncwarp();
-      const int wa = warp_of(ustart), wb = warp_of(uend - 1);
-      const int64_t unit_id = ((int64_t)u_ri * B + u.b) * Hkv + u.h;
-      int ticket = 0;
-      if (lane == 0) ticket = atomicAdd(&p.unit_counter[unit_id], 1);
-      ticket = __shfl_sync(0xffffffffu, ticket, 0);
-      if (ticket == wb - wa) {
-        __threadfence();
-        const int nrec = wb - wa + 1;
-        auto rec_ptr = [&](int k, int g) {
-          const int r2 = k == 0 ? 2 * wa + 1 : 2 * (wa + k);
-          return p.part + ((int64_t)r2 * G + g) * (D + 4);
-        };
-        if (nrec * G <= 32 && nrec <= 8) {
-          // (max, sum) of every (record, head) in parallel, one pair per lane
-          const int pk = lane / G, pg = lane % G;
-          float mk = kNegInf, lk = 0.f;
-          if (lane < nrec * G) {
-            mk = __ldcg(rec_ptr(pk, pg));
-            lk = __ldcg(rec_ptr(pk, pg) + 1);
+      if (lane == 0) red_release_add(&p.unit_counter[unit_id], 1);
+    } else {
+      if (after) {
+        // this warp holds the unit's first piece, which ends last in time:
+        // wait for the later pieces' records and merge them into registers
+        const int nother = warp_of(uend - 1) - gw;
+        if (lane == 0) {
+          if (ld_acquire(&p.unit_counter[unit_id]) < nother) {
+            const uint64_t t0 = global_timer_ns();
+            while (ld_acquire(&p.unit_counter[unit_id]) < nother) {
+              if (global_timer_ns() - t0 > 1000000000ull) {
+                atomicOr(&g_mpc_status, kStatusWaitTimeout);
+                break;
+              }
+              __nanosleep(64);
+            }
           }
-          scr[lane] = mk;
-          __syncwarp();
-          float M = kNegInf;
-          for (int k = 0; k < nrec; ++k) M = fmaxf(M, scr[k * G + pg]);
-          const float wk = (lane < nrec * G && mk != kNegInf) ? fast_exp2(mk - M) : 0.f;
-          scr[32 + lane] = wk;
-          scr[64 + lane] = wk * lk;
-          __syncwarp();
-          for (int g = 0; g < G; ++g) {
-            float v[8][D / 32];
+          p.unit_counter[unit_id] = 0;
+        }
+        __syncwarp();
+        for (int k = 1; k <= nother; ++k) {
+          const float* rec = p.part + (int64_t)(gw + k) * G * (D + 4);
 #pragma unroll
-            for (int k = 0; k < 8; ++k)
+          for (int hn = 0; hn < HN; ++hn)
 #pragma unroll
-              for (int t = 0; t < D / 32; ++t) v[k][t] = (k < nrec) ? __ldcg(rec_ptr(k, g) + 4 + lane + 32 * t) : 0.f;
-            float L = 0.f, acc[D / 32];
+            for (int e = 0; e < 2; ++e) {
+              const int g = hn * 8 + h_off + e;
+              if (g < G) {
+                const float* rg = rec + g * (D + 4);
+                const float mk = __ldcg(rg), lk = __ldcg(rg + 1);
+                const float M = fmaxf(m_run[hn][e], mk);
+                const float wa = (m_run[hn][e] == kNegInf) ? 0.f : fast_exp2(m_run[hn][e] - M);
+                const float wb = (mk == kNegInf) ? 0.f : fast_exp2(mk - M);
+                m_run[hn][e] = M;
+                lq[hn][e] = lq[hn][e] * wa + lk * wb;
 #pragma unroll
-            for (int t = 0; t < D / 32; ++t) acc[t] = 0.f;
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              if (k < nrec) {
-                const float wgt = scr[32 + k * G + g];
-                L += scr[64 + k * G + g];
-#pragma unroll
-                for (int t = 0; t < D / 32; ++t) acc[t] = fmaf(wgt, v[k][t], acc[t]);
+                for (int mt = 0; mt < KS; ++mt) {
+                  o[mt][hn][e] = o[mt][hn][e] * wa + wb * __ldcg(rg + 4 + mt * 16 + r_tok);
+                  o[mt][hn][2 + e] = o[mt][hn][2 + e] * wa + wb * __ldcg(rg + 4 + mt * 16 + r_tok + 8);
+                }
               }
             }
-            const float inv = 1.f / L;
+        }
+      }
 #pragma unroll
-            for (int t = 0; t < D / 32; ++t) outp[g * D + lane + 32 * t] = acc[t] * inv;
-          }
-          __syncwarp();
-        } else {
-          for (int g = 0; g < G; ++g) {
-            float M = kNegInf;
-            for (int k = 0; k < nrec; ++k) M = fmaxf(M, __ldcg(rec_ptr(k, g)));
-            float L = 0.f;
-            float acc[D / 32];
+      for (int hn = 0; hn < HN; ++hn)
 #pragma unroll
-            for (int t = 0; t < D / 32; ++t) acc[t] = 0.f;
-            for (int k = 0; k < nrec; ++k) {
-              const float* rp = rec_ptr(k, g);
-              const float mm = __ldcg(rp);
-              const float f = (mm == kNegInf) ? 0.f : fast_exp2(mm - M);
-              L += f * __ldcg(rp + 1);
+        for (int e = 0; e < 2; ++e) {
+          const int g = hn * 8 + h_off + e;
+          if (g < G) {
+            const float inv = 1.f / lq[hn][e];
 #pragma unroll
-              for (int t = 0; t < D / 32; ++t) acc[t] += f * __ldcg(rp + 4 + lane + 32 * t);
+            for (int mt = 0; mt < KS; ++mt) {
+              outp[g * D + mt * 16 + r_tok] = o[mt][hn][e] * inv;
+              outp[g * D + mt * 16 + r_tok + 8] = o[mt][hn][2 + e] * inv;
             }
-            const float inv = 1.f / L;
-#pragma unroll
-            for (int t = 0; t < D / 32; ++t) outp[g * D + lane + 32 * t] = acc[t] * inv;
           }
         }
-        if (lane == 0) p.unit_counter[unit_id] = 0;
-      }
     }
     // the piece that holds the appended row seals a full tail
     if (uend <= x1) seal_tail<bf16, D>(p, u, reinterpret_cast<const bf16*>(kv_base(u, 0)));
@@ -1025,10 +999,10 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const __grid_constant__ A
 
 // ------------------------------------------------------------- launch ----
 
-int attn_smem_bytes(int dtype, int D, int G) {
+int attn_smem_bytes(int dtype, int D, int G, int B) {
   if (dtype == MPC_BF16) {
-    const int nst = persist_stages(D, G);
-    return D == 64 ? PSmem<64>::total(G, nst, kMaxBatchPersist) : PSmem<128>::total(G, nst, kMaxBatchPersist);
+    const int nst = persist_stages(D, G, B);
+    return D == 64 ? PSmem<64>::total(G, nst, B) : PSmem<128>::total(G, nst, B);
   }
   return D == 64 ? Smem<64, 4>::total(G) : Smem<128, 4>::total(G);
 }
@@ -1062,18 +1036,19 @@ static int persist_ctas() {
 cudaError_t launch_attn(const AttnParams& p0, int dtype, int D, int n_units, cudaStream_t st) {
   AttnParams p = p0;
   if (dtype == MPC_BF16) {
-    p.n_stages = persist_stages(D, p.G);
-    const int smem = attn_smem_bytes(dtype, D, p.G);
+    p.n_stages = persist_stages(D, p.G, p.B);
+    const int smem = attn_smem_bytes(dtype, D, p.G, p.B);
     const dim3 grid(persist_ctas());
     if (p.G <= 8) {
       if (D == 64) return launch_k(attn_bf16_persist_kernel<64, 1, 8>, grid, smem, st, p);
+      if (p.n_stages == 6) return launch_k(attn_bf16_persist_kernel<128, 1, 6>, grid, smem, st, p);
       return launch_k(attn_bf16_persist_kernel<128, 1, 5>, grid, smem, st, p);
     }
     if (D == 64) return launch_k(attn_bf16_persist_kernel<64, 2, 8>, grid, smem, st, p);
     return launch_k(attn_bf16_persist_kernel<128, 2, 4>, grid, smem, st, p);
   }
   const dim3 grid(p.n_split, n_units);
-  const int smem = attn_smem_bytes(dtype, D, p.G);
+  const int smem = attn_smem_bytes(dtype, D, p.G, p.B);
   const int G = p.G;
 #define MPC_F32_CASE(DD, GG) \
   if (D == DD && G <= GG) return launch_k(attn_f32_kernel<DD, GG>, grid, smem, st, p);

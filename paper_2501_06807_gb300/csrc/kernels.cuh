@@ -118,7 +118,7 @@ struct ClusterParams {
 };
 
 cudaError_t launch_attn(const AttnParams& p, int dtype, int D, int n_units, cudaStream_t st);
-int attn_smem_bytes(int dtype, int D, int G);
+int attn_smem_bytes(int dtype, int D, int G, int B);
 int attn_persist_ctas_max();
 int attn_persist_batch_max();
 cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cudaStream_t st);
