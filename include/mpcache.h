@@ -24,7 +24,8 @@
  *   library never allocates, frees or retains them past the call.  Scratch
  *   space is the caller's too: `*_workspace_size` reports how many bytes a
  *   call needs and the call receives them as `workspace`.  A workspace must
- *   be zero-filled once before its first use; calls leave it zero-filled.
+ *   be 16-byte aligned and zero-filled once before its first use; the calls
+ *   that keep counters in it leave them zero, so it can be reused as is.
  * - Every call is asynchronous on `stream` (a cudaStream_t; NULL = legacy
  *   default stream) and returns once its kernels are queued.  Arguments are
  *   validated on the host before anything is launched.

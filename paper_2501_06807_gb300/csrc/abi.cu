@@ -159,7 +159,12 @@ int validate_static(const mpc_static_args* a, StaticParams* p) {
 }
 
 // Row statistics (m, 1/l) of every window row.
-size_t static_ws(const StaticParams& p) { return (size_t)p.n_refs * p.B * p.Hq * p.win_rows * sizeof(float2); }
+// Row statistics of the window: per (ref, b, query head) the arrays -m and
+// 1 / l, each padded to a multiple of 128 rows (one TMA copy per row tile).
+int stats_ld_of(int win_rows) { return (win_rows + 127) / 128 * 128; }
+size_t static_ws(const StaticParams& p) {
+  return (size_t)p.n_refs * p.B * p.Hq * 2 * stats_ld_of(p.win_rows) * sizeof(float);
+}
 
 // ------------------------------------------------------------ clusters ----
 int validate_clusters(const mpc_cluster_args* a, ClusterParams* p) {
@@ -422,7 +427,9 @@ MPC_API int mpc_static_evict(const mpc_static_args* args, void* workspace, size_
   const size_t need = static_ws(p);
   if (workspace == nullptr || workspace_bytes < need)
     return fail(MPC_ERR_WORKSPACE, "workspace of %zu bytes needed", need);
-  p.stats = static_cast<float2*>(workspace);
+  if (!aligned16(workspace)) return fail(MPC_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
+  p.stats = static_cast<float*>(workspace);
+  p.stats_ld = stats_ld_of(p.win_rows);
   int span = 0;
   for (int i = 0; i < args->n_refs; ++i) span = args->refs[i].layer + 1 > span ? args->refs[i].layer + 1 : span;
   const cudaError_t e = launch_static(p, args->dtype, args->head_dim, span, static_cast<cudaStream_t>(stream));

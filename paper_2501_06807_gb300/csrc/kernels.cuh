@@ -71,7 +71,8 @@ struct StaticParams {
   float* scores;      // [group][b][Hkv][t_max]
   int* kept;          // [group][b][Hkv][keep_cap]
   int* n_keep;        // [b]
-  float2* stats;      // [ref][b][Hq][win_rows]: (m, 1 / l)
+  float* stats;       // [ref][b][Hq][2][stats_ld]: -m, then 1 / l, per window row
+  int stats_ld;       // win_rows rounded up to 128
 };
 
 // Window scoring on tcgen05 (bf16 queries and dense keys).
@@ -88,7 +89,8 @@ struct ScoreTcParams {
   int window_ppm, long_window_ppm, long_threshold;
   float scale_log2;
   float* scores;
-  float2* stats;
+  float* stats;  // as StaticParams::stats
+  int stats_ld;
 };
 
 struct KvSrc {

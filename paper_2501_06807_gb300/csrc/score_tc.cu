@@ -12,14 +12,21 @@
 //     A = the 128 key rows (fixed), B = 128-row tiles of window queries of
 //     every query head of the GQA group.  S^T = A B^T puts one key per TMEM
 //     lane, so each thread sums 2^(s_ij - m_i) / l_i over the rows i in its
-//     own registers, in a fixed order (deterministic scores).
+//     own registers, in a fixed order (deterministic scores).  The rows'
+//     (-m, 1/l) arrive by bulk copy with each query tile; rows past the
+//     window carry -m = -inf, so they add exact zeros.
 //
 // Roles: warp 0 issues TMA tile loads (128B-swizzled, K-major boxes of
 // 128 rows x 64 channels), warp 1 allocates TMEM and issues tcgen05.mma
 // (M = N = 128, K = 16, bf16 in, fp32 accumulate) into one of two 128-column
-// accumulators, warps 2-5 drain the other accumulator with tcgen05.ld.
-// Every wait is bounded; a timeout sets the device status word and an abort
-// flag that stops the other roles, and TMEM is always released.
+// accumulators, and eight epilogue warps drain the other accumulator with
+// tcgen05.ld: two warps per 32-lane quarter, each taking half of the 128
+// columns, combined through shared memory at the end.  The epilogue is the
+// bound (one ex2 per score), so its inner loops use packed f32x2 FMA / add
+// and a three-input max, and compare keys against rows only on the tiles
+// that cross the causal diagonal.  Every wait is bounded; a timeout sets
+// the device status word and an abort flag that stops the other roles, and
+// TMEM is always released.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -30,7 +37,9 @@
 namespace mpc {
 namespace {
 
-constexpr int kTcThreads = 192;
+constexpr int kTcEpiWarps = 8;
+constexpr int kTcEpiThreads = 32 * kTcEpiWarps;
+constexpr int kTcThreads = 64 + kTcEpiThreads;
 constexpr int kStagesTc = 2;
 constexpr int kBoxBytes = 128 * 128;  // 128 rows x 64 bf16 channels
 
@@ -41,24 +50,61 @@ struct TcSmem {
   static constexpr int A_OFF = 0;
   static constexpr int B_OFF = TILE;
   static constexpr int STAGE = TILE;                // one streamed B tile
-  static constexpr int STATS_OFF = B_OFF + kStagesTc * STAGE;  // 2 x 128 row stats (pass 1)
-  static constexpr int BAR_OFF = STATS_OFF + 2 * 128 * 8;
+  static constexpr int STATS_OFF = B_OFF + kStagesTc * STAGE;  // pass 1: 2 slots x (128 -m, 128 1/l)
+  static constexpr int XCH_OFF = STATS_OFF + 2 * 256 * 4;      // halves' partials, 128 x float2
+  static constexpr int BAR_OFF = XCH_OFF + 128 * 8;
   static constexpr int USED = BAR_OFF + 256 + 1024;  // + alignment slack
   // at least 80 KB so that at most two CTAs (2 x 256 TMEM columns) share an SM
   static constexpr int TOTAL = USED > 80 * 1024 ? USED : 80 * 1024;
 };
 
-// Barrier of the 128 epilogue threads that also ANDs a flag over them, so
-// all four warps take the same branch after it.
+// Barrier of the epilogue threads that also ANDs a flag over them, so all
+// epilogue warps take the same branch after it.
 __device__ __forceinline__ bool epilogue_all(bool v) {
   uint32_t r;
   asm volatile(
-      "{\n .reg .pred pi, po;\n setp.ne.u32 pi, %1, 0;\n bar.red.and.pred po, 1, 128, pi;\n"
+      "{\n .reg .pred pi, po;\n setp.ne.u32 pi, %1, 0;\n bar.red.and.pred po, 1, %2, pi;\n"
       " selp.u32 %0, 1, 0, po;\n}"
       : "=r"(r)
-      : "r"((uint32_t)v)
+      : "r"((uint32_t)v), "n"(kTcEpiThreads)
       : "memory");
   return r != 0;
+}
+__device__ __forceinline__ void epilogue_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kTcEpiThreads) : "memory"); }
+
+// Packed pairs of fp32 (one 64-bit register pair) and the sm_100 f32x2 ops.
+__device__ __forceinline__ uint64_t pk2(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+__device__ __forceinline__ void upk2(uint64_t r, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(r));
+}
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.ftz.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.ftz.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+// max of 32 values, two independent chains of three-input max
+__device__ __forceinline__ float max32(const float* v) {
+  float a = fmax3(v[0], v[1], v[2]), b = fmax3(v[3], v[4], v[5]);
+#pragma unroll
+  for (int k = 6; k < 30; k += 4) {
+    a = fmax3(a, v[k], v[k + 1]);
+    b = fmax3(b, v[k + 2], v[k + 3]);
+  }
+  return fmax3(a, b, fmaxf(v[30], v[31]));
 }
 
 // ----------------------------------------------------------------- PTX ----
@@ -157,7 +203,7 @@ __device__ __forceinline__ int win_rows_of(const ScoreTcParams& p, int T) {
 }
 
 template <int PASS, int D>
-__global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(const __grid_constant__ ScoreTcParams p) {
+__global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_constant__ ScoreTcParams p) {
   using S = TcSmem<D>;
   constexpr int KH = S::KH;
   extern __shared__ uint8_t smem_raw[];
@@ -167,8 +213,10 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(const __grid_co
   uint64_t* a_full = empty + kStagesTc;
   uint64_t* acc_full = a_full + 1;
   uint64_t* acc_empty = acc_full + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(acc_empty + 2);
+  uint64_t* stats_full = acc_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(stats_full + 2);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  float* stats_s = reinterpret_cast<float*>(smem + S::STATS_OFF);  // [slot][-m 128 | 1/l 128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // ---- work unit
@@ -208,7 +256,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(const __grid_co
     mbar_init(a_full, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(&acc_full[i], 1);
-      mbar_init(&acc_empty[i], 4);
+      mbar_init(&acc_empty[i], kTcEpiWarps);
+      mbar_init(&stats_full[i], 1);
     }
     *abort = 0;
     fence_barrier_init();
@@ -224,7 +273,7 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(const __grid_co
 
   if (warp == 0 && lane == 0 && n_tiles > 0) {
     // ---------------------------------------------------- TMA producer
-    int n_issued = 0;
+    int n_issued = 0, n_stats = 0;
     const int qrow0 = (b * p.Hq) * p.win_rows + qoff;       // + hq * win_rows + i
     const int krow0 = (b * p.Hkv) * p.t_max;                 // + hk * t_max + j
     mbar_arrive_expect_tx(a_full, S::TILE);
@@ -249,13 +298,28 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(const __grid_co
         mbar_arrive_expect_tx(&full[s], S::TILE);
         for (int kh = 0; kh < KH; ++kh)
           tma_load_3d(st + kh * kBoxBytes, &p.map_q, kh * 64, qrow0 + hq * p.win_rows + it, layer, &full[s]);
+        n_issued = t + 1;
+        // the rows' (-m, 1/l) into the slot of this tile's accumulator, once
+        // the epilogue has finished the tile that used it before
+        const int sb = t & 1;
+        if (t >= 2 && !wait_or_abort(&acc_empty[sb], ((t >> 1) - 1) & 1, abort)) break;
+        const float* src = p.stats + (((int64_t)ri * p.B + b) * p.Hq + hq) * 2 * p.stats_ld + it;
+        float* dst = stats_s + sb * 256;
+        mbar_arrive_expect_tx(&stats_full[sb], 1024);
+        bulk_g2s(dst, src, 512, &stats_full[sb]);
+        bulk_g2s(dst + 128, src + p.stats_ld, 512, &stats_full[sb]);
+        n_stats = t + 1;
       }
       n_issued = t + 1;
     }
-    // leave no copy in flight: wait (bounded) for the last stages issued
+    // leave no copy in flight: wait (bounded) for the last copies issued
     for (int t = n_issued > kStagesTc ? n_issued - kStagesTc : 0; t < n_issued; ++t) {
       int never = 0;
       wait_or_abort(&full[t % kStagesTc], (t / kStagesTc) & 1, &never);
+    }
+    for (int t = n_stats > 2 ? n_stats - 2 : 0; t < n_stats; ++t) {
+      int never = 0;
+      wait_or_abort(&stats_full[t & 1], (t >> 1) & 1, &never);
     }
   } else if (warp == 1 && lane == 0 && n_tiles > 0) {
     // ---------------------------------------------------- MMA issuer
@@ -286,90 +350,105 @@ __global__ void __launch_bounds__(kTcThreads, 1) score_tc_kernel(const __grid_co
   } else if (warp >= 2) {
     // ---------------------------------------------------- epilogue
     const int quarter = warp & 3;               // TMEM lanes 32*quarter ..
+    const int half = (warp - 2) >> 2;           // columns 64*half .. +63
+    const int col0 = half * 64;
     const int r = quarter * 32 + lane;          // this thread's TMEM lane
-    const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
+    const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16) + col0;
+    const uint64_t sc2 = pk2(p.scale_log2, p.scale_log2);
     float m = kNegInf, l = 0.f, acc = 0.f;
     const int i_row = i0 + r;                   // pass 0: window row
     const int pos_row = base + i_row;
     const int j_key = j0 + r;                   // pass 1: key
-    float2* stats_s = reinterpret_cast<float2*>(smem + S::STATS_OFF);
-    // pass 1: (m, 1/l) of the 128 window rows of a tile; thread r fetches row
-    // r of the next tile while the current one is processed
-    auto row_stats = [&](int t) -> float2 {
-      const int g = t / tiles_per_g, it = i_start + (t % tiles_per_g) * 128;
-      if (it + r >= w) return make_float2(0.f, 0.f);
-      return p.stats[(((int64_t)ri * p.B + b) * p.Hq + head * p.G + g) * p.win_rows + it + r];
-    };
-    float2 next_stats = make_float2(0.f, 0.f);
-    if (PASS == 1 && n_tiles > 0) next_stats = row_stats(0);
-    for (int t = 0; t < n_tiles; ++t) {
+    int t = 0;
+    for (; t < n_tiles; ++t) {
       const int buf = t & 1;
-      if (PASS == 1) {
-        stats_s[buf * 128 + r] = next_stats;
-        if (t + 1 < n_tiles) next_stats = row_stats(t + 1);
-      }
-      const bool ok = wait_or_abort(&acc_full[buf], (t >> 1) & 1, abort);
+      bool ok = wait_or_abort(&acc_full[buf], (t >> 1) & 1, abort);
+      if (PASS == 1 && ok) ok = wait_or_abort(&stats_full[buf], (t >> 1) & 1, abort);
       if (!epilogue_all(ok)) break;
       tc_fence_after();
       if (PASS == 0) {
-        const int kj = t * 128;
-        const bool need_mask = kj + 127 > base + i0;
+        const int kj = t * 128 + col0;                  // first key of this thread's columns
+        const bool need_mask = kj + 63 > base + i0;     // crosses some row's diagonal
 #pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
+        for (int c = 0; c < 2; ++c) {
           float v[32];
           tmem_ld32(lane_addr + buf * 128 + c * 32, v);
-          float mx = kNegInf;
+          if (need_mask) {
 #pragma unroll
-          for (int k = 0; k < 32; ++k) {
-            if (need_mask && kj + c * 32 + k > pos_row) v[k] = kNegInf;
-            mx = fmaxf(mx, v[k]);
+            for (int k = 0; k < 32; ++k)
+              if (kj + c * 32 + k > pos_row) v[k] = kNegInf;
           }
-          const float mnew = fmaxf(m, mx * p.scale_log2);
+          const float mnew = fmaxf(m, max32(v) * p.scale_log2);
           if (mnew != kNegInf) {
-            float sum = 0.f;
+            const uint64_t nm2 = pk2(-mnew, -mnew);
+            uint64_t s2 = pk2(0.f, 0.f);
 #pragma unroll
-            for (int k = 0; k < 32; ++k) sum += fast_exp2(fmaf(v[k], p.scale_log2, -mnew));
+            for (int k = 0; k < 32; k += 2) {
+              float x0, x1;
+              upk2(ffma2(pk2(v[k], v[k + 1]), sc2, nm2), x0, x1);
+              s2 = fadd2(s2, pk2(fast_exp2(x0), fast_exp2(x1)));
+            }
+            float s0, s1;
+            upk2(s2, s0, s1);
+            const float sum = s0 + s1;
             l = (m == kNegInf) ? sum : l * fast_exp2(m - mnew) + sum;
             m = mnew;
           }
         }
       } else {
-        const int it = i_start + (t % tiles_per_g) * 128;
-        const float2* st = stats_s + buf * 128;
-        // rows it .. it+127; row i sees key j when j <= base + i and i < w
-        const bool need_mask = (j0 + 127 > base + it) || (it + 127 >= w);
-        float tsum = 0.f;
+        const int it = i_start + (t % tiles_per_g) * 128 + col0;  // first row of this thread's columns
+        const float* nm_s = stats_s + buf * 256 + col0;
+        const float* il_s = nm_s + 128;
+        // row i sees key j when j <= base + i; rows past the window have -m = -inf
+        const bool need_mask = j0 + 127 > base + it;
+        uint64_t s2 = pk2(0.f, 0.f);
 #pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
+        for (int c = 0; c < 2; ++c) {
           float v[32];
           tmem_ld32(lane_addr + buf * 128 + c * 32, v);
+          if (need_mask) {
 #pragma unroll
-          for (int k = 0; k < 32; k += 2) {
-            const float4 ml = *reinterpret_cast<const float4*>(st + c * 32 + k);
-            float e0 = fast_exp2(fmaf(v[k], p.scale_log2, -ml.x)) * ml.y;
-            float e1 = fast_exp2(fmaf(v[k + 1], p.scale_log2, -ml.z)) * ml.w;
-            if (need_mask) {
-              const int ia = it + c * 32 + k;
-              if (ia >= w || j_key > base + ia) e0 = 0.f;
-              if (ia + 1 >= w || j_key > base + ia + 1) e1 = 0.f;
-            }
-            tsum += e0;
-            tsum += e1;
+            for (int k = 0; k < 32; ++k)
+              if (j_key > base + it + c * 32 + k) v[k] = kNegInf;
+          }
+#pragma unroll
+          for (int k = 0; k < 32; k += 4) {
+            const float4 nm4 = *reinterpret_cast<const float4*>(nm_s + c * 32 + k);
+            const float4 il4 = *reinterpret_cast<const float4*>(il_s + c * 32 + k);
+            float x0, x1, x2, x3;
+            upk2(ffma2(pk2(v[k], v[k + 1]), sc2, pk2(nm4.x, nm4.y)), x0, x1);
+            upk2(ffma2(pk2(v[k + 2], v[k + 3]), sc2, pk2(nm4.z, nm4.w)), x2, x3);
+            s2 = ffma2(pk2(fast_exp2(x0), fast_exp2(x1)), pk2(il4.x, il4.y), s2);
+            s2 = ffma2(pk2(fast_exp2(x2), fast_exp2(x3)), pk2(il4.z, il4.w), s2);
           }
         }
-        acc += tsum;
+        float s0, s1;
+        upk2(s2, s0, s1);
+        acc += s0 + s1;
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&acc_empty[buf]);
     }
-    if (!*abort) {
+    // combine the two column halves of every lane (fixed order: half 0 + half 1)
+    float2* xch = reinterpret_cast<float2*>(smem + S::XCH_OFF);
+    if (half == 1) xch[r] = PASS == 0 ? make_float2(m, l) : make_float2(acc, 0.f);
+    epilogue_sync();
+    if (half == 0 && !*abort && t == n_tiles && n_tiles > 0) {
+      const float2 o = xch[r];
       if (PASS == 0) {
-        if (i_row < w && n_tiles > 0)
-          p.stats[(((int64_t)ri * p.B + b) * p.Hq + head) * p.win_rows + i_row] = make_float2(m, 1.f / l);
-      } else {
-        if (n_tiles > 0 && j_key < T_b)
-          p.scores[((int64_t)(group * p.B + b) * p.Hkv + head) * p.t_max + j_key] = acc;
+        const float M = fmaxf(m, o.x);
+        const float L = (m == kNegInf ? 0.f : l * fast_exp2(m - M)) + (o.x == kNegInf ? 0.f : o.y * fast_exp2(o.x - M));
+        float* st = p.stats + (((int64_t)ri * p.B + b) * p.Hq + head) * 2 * p.stats_ld;
+        if (i_row < w) {
+          st[i_row] = -M;
+          st[p.stats_ld + i_row] = 1.f / L;
+        } else if (i_row < (w + 127) / 128 * 128) {
+          st[i_row] = kNegInf;  // past the window: contributes nothing in pass 1
+          st[p.stats_ld + i_row] = 0.f;
+        }
+      } else if (j_key < T_b) {
+        p.scores[((int64_t)(group * p.B + b) * p.Hkv + head) * p.t_max + j_key] = acc + o.x;
       }
     }
   }

@@ -126,8 +126,11 @@ __global__ void __launch_bounds__(256) rowstats_kernel(const __grid_constant__ S
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
       const int i = row0 + ty * 4 + r;
-      if (i < w)
-        p.stats[(((int64_t)ri * p.B + b) * p.Hq + hq) * p.win_rows + i] = make_float2(m[r], 1.f / l[r]);
+      if (i < w) {
+        float* st = p.stats + (((int64_t)ri * p.B + b) * p.Hq + hq) * 2 * p.stats_ld;
+        st[i] = -m[r];
+        st[p.stats_ld + i] = 1.f / l[r];
+      }
     }
   }
 }
@@ -156,12 +159,12 @@ __global__ void __launch_bounds__(256) colsum_kernel(const __grid_constant__ Sta
   for (int g = 0; g < p.G; ++g) {
     const int hq = hk * p.G + g;
     const T* qbase = (const T*)p.q_win + layer * p.qw_ls + ((int64_t)b * p.Hq + hq) * p.win_rows * D;
-    const float2* stats = p.stats + (((int64_t)ri * p.B + b) * p.Hq + hq) * p.win_rows;
+    const float* stats = p.stats + (((int64_t)ri * p.B + b) * p.Hq + hq) * 2 * p.stats_ld;
     for (int i0 = i_start; i0 < w; i0 += kTile) {
       __syncthreads();
       load_tile_t<T, D>(Qs, w, i0, [&](int i) { return qbase + (int64_t)(qoff + i) * D; });
       for (int i = threadIdx.x; i < kTile; i += blockDim.x)
-        st[i] = (i0 + i < w) ? stats[i0 + i] : make_float2(0.f, 0.f);
+        st[i] = (i0 + i < w) ? make_float2(stats[i0 + i], stats[p.stats_ld + i0 + i]) : make_float2(0.f, 0.f);
       __syncthreads();
       float acc[4][4] = {};
 #pragma unroll 8
@@ -183,7 +186,7 @@ __global__ void __launch_bounds__(256) colsum_kernel(const __grid_constant__ Sta
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
           const int j = j0 + ty * 4 + q;
-          if (i < w && j <= pos) tile[q] += fast_exp2(acc[q][r] * p.scale_log2 - ml.x) * ml.y;
+          if (i < w && j <= pos) tile[q] += fast_exp2(acc[q][r] * p.scale_log2 + ml.x) * ml.y;
         }
       }
 #pragma unroll
@@ -328,6 +331,7 @@ cudaError_t launch_static(const StaticParams& p, int dtype, int D, int n_layer_s
     t.scale_log2 = p.scale_log2;
     t.scores = p.scores;
     t.stats = p.stats;
+    t.stats_ld = p.stats_ld;
     if ((e = launch_score_tc(t, D, n_layer_span, st)) != cudaSuccess) return e;
   } else {
     const int smem = static_tile_smem(D);
