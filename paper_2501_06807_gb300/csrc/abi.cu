@@ -159,11 +159,11 @@ int validate_static(const mpc_static_args* a, StaticParams* p) {
 }
 
 // Row statistics (m, 1/l) of every window row.
-// Row statistics of the window: per (ref, b, query head) the arrays -m and
-// 1 / l, each padded to a multiple of 128 rows (one TMA copy per row tile).
+// Row statistics of the window: per (ref, b, query head) one array of
+// -(m + log2 l), padded to a multiple of 128 rows (one bulk copy per row tile).
 int stats_ld_of(int win_rows) { return (win_rows + 127) / 128 * 128; }
 size_t static_ws(const StaticParams& p) {
-  return (size_t)p.n_refs * p.B * p.Hq * 2 * stats_ld_of(p.win_rows) * sizeof(float);
+  return (size_t)p.n_refs * p.B * p.Hq * stats_ld_of(p.win_rows) * sizeof(float);
 }
 
 // ------------------------------------------------------------ clusters ----

@@ -71,7 +71,7 @@ struct StaticParams {
   float* scores;      // [group][b][Hkv][t_max]
   int* kept;          // [group][b][Hkv][keep_cap]
   int* n_keep;        // [b]
-  float* stats;       // [ref][b][Hq][2][stats_ld]: -m, then 1 / l, per window row
+  float* stats;       // [ref][b][Hq][stats_ld]: -(m + log2 l) per window row
   int stats_ld;       // win_rows rounded up to 128
 };
 

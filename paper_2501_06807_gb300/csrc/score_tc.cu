@@ -12,9 +12,10 @@
 //     A = the 128 key rows (fixed), B = 128-row tiles of window queries of
 //     every query head of the GQA group.  S^T = A B^T puts one key per TMEM
 //     lane, so each thread sums 2^(s_ij - m_i) / l_i over the rows i in its
-//     own registers, in a fixed order (deterministic scores).  The rows'
-//     (-m, 1/l) arrive by bulk copy with each query tile; rows past the
-//     window carry -m = -inf, so they add exact zeros.
+//     own registers, in a fixed order (deterministic scores).  Each row's
+//     statistic arrives as -(m_i + log2 l_i) by bulk copy with its query
+//     tile, so a score costs one FMA, one ex2 and one add; rows past the
+//     window carry -inf, so they add exact zeros.
 //
 // Roles: warp 0 issues TMA tile loads (128B-swizzled, K-major boxes of
 // 128 rows x 64 channels), warp 1 allocates TMEM and issues tcgen05.mma
@@ -41,6 +42,7 @@ constexpr int kTcEpiWarps = 8;
 constexpr int kTcEpiThreads = 32 * kTcEpiWarps;
 constexpr int kTcThreads = 64 + kTcEpiThreads;
 constexpr int kStagesTc = 2;
+constexpr int kStatSlots = 4;  // row-statistics ring of pass 1 (tiles in flight ahead of the epilogue)
 constexpr int kBoxBytes = 128 * 128;  // 128 rows x 64 bf16 channels
 
 template <int D>
@@ -50,8 +52,8 @@ struct TcSmem {
   static constexpr int A_OFF = 0;
   static constexpr int B_OFF = TILE;
   static constexpr int STAGE = TILE;                // one streamed B tile
-  static constexpr int STATS_OFF = B_OFF + kStagesTc * STAGE;  // pass 1: 2 slots x (128 -m, 128 1/l)
-  static constexpr int XCH_OFF = STATS_OFF + 2 * 256 * 4;      // halves' partials, 128 x float2
+  static constexpr int STATS_OFF = B_OFF + kStagesTc * STAGE;  // pass 1: kStatSlots x 128 -(m + log2 l)
+  static constexpr int XCH_OFF = STATS_OFF + kStatSlots * 128 * 4;  // halves' partials, 128 x float2
   static constexpr int BAR_OFF = XCH_OFF + 128 * 8;
   static constexpr int USED = BAR_OFF + 256 + 1024;  // + alignment slack
   // at least 80 KB so that at most two CTAs (2 x 256 TMEM columns) share an SM
@@ -96,6 +98,13 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
   asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
   return d;
 }
+// two ex2.approx (MUFU)
+__device__ __forceinline__ uint64_t exp2_mufu2(uint64_t x2) {
+  float x0, x1;
+  upk2(x2, x0, x1);
+  return pk2(fast_exp2(x0), fast_exp2(x1));
+}
+
 // max of 32 values, two independent chains of three-input max
 __device__ __forceinline__ float max32(const float* v) {
   float a = fmax3(v[0], v[1], v[2]), b = fmax3(v[3], v[4], v[5]);
@@ -214,9 +223,10 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
   uint64_t* acc_full = a_full + 1;
   uint64_t* acc_empty = acc_full + 2;
   uint64_t* stats_full = acc_empty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(stats_full + 2);
+  uint64_t* stats_empty = stats_full + kStatSlots;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(stats_empty + kStatSlots);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  float* stats_s = reinterpret_cast<float*>(smem + S::STATS_OFF);  // [slot][-m 128 | 1/l 128]
+  float* stats_s = reinterpret_cast<float*>(smem + S::STATS_OFF);  // [slot][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // ---- work unit
@@ -257,7 +267,10 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
     for (int i = 0; i < 2; ++i) {
       mbar_init(&acc_full[i], 1);
       mbar_init(&acc_empty[i], kTcEpiWarps);
+    }
+    for (int i = 0; i < kStatSlots; ++i) {
       mbar_init(&stats_full[i], 1);
+      mbar_init(&stats_empty[i], kTcEpiWarps);
     }
     *abort = 0;
     fence_barrier_init();
@@ -299,15 +312,13 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
         for (int kh = 0; kh < KH; ++kh)
           tma_load_3d(st + kh * kBoxBytes, &p.map_q, kh * 64, qrow0 + hq * p.win_rows + it, layer, &full[s]);
         n_issued = t + 1;
-        // the rows' (-m, 1/l) into the slot of this tile's accumulator, once
-        // the epilogue has finished the tile that used it before
-        const int sb = t & 1;
-        if (t >= 2 && !wait_or_abort(&acc_empty[sb], ((t >> 1) - 1) & 1, abort)) break;
-        const float* src = p.stats + (((int64_t)ri * p.B + b) * p.Hq + hq) * 2 * p.stats_ld + it;
-        float* dst = stats_s + sb * 256;
-        mbar_arrive_expect_tx(&stats_full[sb], 1024);
-        bulk_g2s(dst, src, 512, &stats_full[sb]);
-        bulk_g2s(dst + 128, src + p.stats_ld, 512, &stats_full[sb]);
+        // the rows' -(m + log2 l) into their ring slot, once the epilogue
+        // has finished the tile that used the slot before
+        const int sb = t % kStatSlots;
+        if (t >= kStatSlots && !wait_or_abort(&stats_empty[sb], ((t / kStatSlots) - 1) & 1, abort)) break;
+        const float* src = p.stats + (((int64_t)ri * p.B + b) * p.Hq + hq) * p.stats_ld + it;
+        mbar_arrive_expect_tx(&stats_full[sb], 512);
+        bulk_g2s(stats_s + sb * 128, src, 512, &stats_full[sb]);
         n_stats = t + 1;
       }
       n_issued = t + 1;
@@ -317,9 +328,9 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
       int never = 0;
       wait_or_abort(&full[t % kStagesTc], (t / kStagesTc) & 1, &never);
     }
-    for (int t = n_stats > 2 ? n_stats - 2 : 0; t < n_stats; ++t) {
+    for (int t = n_stats > kStatSlots ? n_stats - kStatSlots : 0; t < n_stats; ++t) {
       int never = 0;
-      wait_or_abort(&stats_full[t & 1], (t >> 1) & 1, &never);
+      wait_or_abort(&stats_full[t % kStatSlots], (t / kStatSlots) & 1, &never);
     }
   } else if (warp == 1 && lane == 0 && n_tiles > 0) {
     // ---------------------------------------------------- MMA issuer
@@ -363,7 +374,7 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
     for (; t < n_tiles; ++t) {
       const int buf = t & 1;
       bool ok = wait_or_abort(&acc_full[buf], (t >> 1) & 1, abort);
-      if (PASS == 1 && ok) ok = wait_or_abort(&stats_full[buf], (t >> 1) & 1, abort);
+      if (PASS == 1 && ok) ok = wait_or_abort(&stats_full[t % kStatSlots], (t / kStatSlots) & 1, abort);
       if (!epilogue_all(ok)) break;
       tc_fence_after();
       if (PASS == 0) {
@@ -384,9 +395,8 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
             uint64_t s2 = pk2(0.f, 0.f);
 #pragma unroll
             for (int k = 0; k < 32; k += 2) {
-              float x0, x1;
-              upk2(ffma2(pk2(v[k], v[k + 1]), sc2, nm2), x0, x1);
-              s2 = fadd2(s2, pk2(fast_exp2(x0), fast_exp2(x1)));
+              const uint64_t x2 = ffma2(pk2(v[k], v[k + 1]), sc2, nm2);
+              s2 = fadd2(s2, exp2_mufu2(x2));
             }
             float s0, s1;
             upk2(s2, s0, s1);
@@ -397,8 +407,7 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
         }
       } else {
         const int it = i_start + (t % tiles_per_g) * 128 + col0;  // first row of this thread's columns
-        const float* nm_s = stats_s + buf * 256 + col0;
-        const float* il_s = nm_s + 128;
+        const float* nm_s = stats_s + (t % kStatSlots) * 128 + col0;
         // row i sees key j when j <= base + i; rows past the window have -m = -inf
         const bool need_mask = j0 + 127 > base + it;
         uint64_t s2 = pk2(0.f, 0.f);
@@ -414,12 +423,8 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
 #pragma unroll
           for (int k = 0; k < 32; k += 4) {
             const float4 nm4 = *reinterpret_cast<const float4*>(nm_s + c * 32 + k);
-            const float4 il4 = *reinterpret_cast<const float4*>(il_s + c * 32 + k);
-            float x0, x1, x2, x3;
-            upk2(ffma2(pk2(v[k], v[k + 1]), sc2, pk2(nm4.x, nm4.y)), x0, x1);
-            upk2(ffma2(pk2(v[k + 2], v[k + 3]), sc2, pk2(nm4.z, nm4.w)), x2, x3);
-            s2 = ffma2(pk2(fast_exp2(x0), fast_exp2(x1)), pk2(il4.x, il4.y), s2);
-            s2 = ffma2(pk2(fast_exp2(x2), fast_exp2(x3)), pk2(il4.z, il4.w), s2);
+            s2 = fadd2(s2, exp2_mufu2(ffma2(pk2(v[k], v[k + 1]), sc2, pk2(nm4.x, nm4.y))));
+            s2 = fadd2(s2, exp2_mufu2(ffma2(pk2(v[k + 2], v[k + 3]), sc2, pk2(nm4.z, nm4.w))));
           }
         }
         float s0, s1;
@@ -428,7 +433,10 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&acc_empty[buf]);
+      if (lane == 0) {
+        mbar_arrive(&acc_empty[buf]);
+        if (PASS == 1) mbar_arrive(&stats_empty[t % kStatSlots]);
+      }
     }
     // combine the two column halves of every lane (fixed order: half 0 + half 1)
     float2* xch = reinterpret_cast<float2*>(smem + S::XCH_OFF);
@@ -439,14 +447,11 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
       if (PASS == 0) {
         const float M = fmaxf(m, o.x);
         const float L = (m == kNegInf ? 0.f : l * fast_exp2(m - M)) + (o.x == kNegInf ? 0.f : o.y * fast_exp2(o.x - M));
-        float* st = p.stats + (((int64_t)ri * p.B + b) * p.Hq + head) * 2 * p.stats_ld;
-        if (i_row < w) {
-          st[i_row] = -M;
-          st[p.stats_ld + i_row] = 1.f / L;
-        } else if (i_row < (w + 127) / 128 * 128) {
+        float* st = p.stats + (((int64_t)ri * p.B + b) * p.Hq + head) * p.stats_ld;
+        if (i_row < w)
+          st[i_row] = -(M + log2f(L));
+        else if (i_row < (w + 127) / 128 * 128)
           st[i_row] = kNegInf;  // past the window: contributes nothing in pass 1
-          st[p.stats_ld + i_row] = 0.f;
-        }
       } else if (j_key < T_b) {
         p.scores[((int64_t)(group * p.B + b) * p.Hkv + head) * p.t_max + j_key] = acc + o.x;
       }

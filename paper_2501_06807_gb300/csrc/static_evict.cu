@@ -8,7 +8,9 @@
 //                    (online, one key tile at a time);
 //   colsum_kernel    per (ref, b, kv head, 64-key block): recomputes s_ij for
 //                    every window row of every query head of the group and
-//                    sums 2^(s_ij - m_i) / l_i per key in registers;
+//                    sums 2^(s_ij - m_i) / l_i = 2^(s_ij - (m_i + log2 l_i))
+//                    per key in registers (the row statistic is stored as
+//                    the single value -(m_i + log2 l_i));
 //   budget_kernel    per (ref, b, kv head): exact top-n_keep of the scores by
 //                    a 4-pass 8-bit radix select on orderable fp32 keys, ties
 //                    to the lower position, then an order-preserving
@@ -126,11 +128,7 @@ __global__ void __launch_bounds__(256) rowstats_kernel(const __grid_constant__ S
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
       const int i = row0 + ty * 4 + r;
-      if (i < w) {
-        float* st = p.stats + (((int64_t)ri * p.B + b) * p.Hq + hq) * 2 * p.stats_ld;
-        st[i] = -m[r];
-        st[p.stats_ld + i] = 1.f / l[r];
-      }
+      if (i < w) p.stats[(((int64_t)ri * p.B + b) * p.Hq + hq) * p.stats_ld + i] = -(m[r] + log2f(l[r]));
     }
   }
 }
@@ -140,7 +138,7 @@ __global__ void __launch_bounds__(256) colsum_kernel(const __grid_constant__ Sta
   extern __shared__ __align__(16) float sm[];
   float* Ks = sm;
   float* Qs = sm + D * kPad;
-  float2* st = reinterpret_cast<float2*>(Qs + D * kPad);
+  float* st = Qs + D * kPad;  // -(m + log2 l) of the tile's rows
   const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;  // ty: keys, tx: rows
   const int unit = blockIdx.y;
   const int hk = unit % p.Hkv, b = (unit / p.Hkv) % p.B, ri = unit / (p.Hkv * p.B);
@@ -159,12 +157,12 @@ __global__ void __launch_bounds__(256) colsum_kernel(const __grid_constant__ Sta
   for (int g = 0; g < p.G; ++g) {
     const int hq = hk * p.G + g;
     const T* qbase = (const T*)p.q_win + layer * p.qw_ls + ((int64_t)b * p.Hq + hq) * p.win_rows * D;
-    const float* stats = p.stats + (((int64_t)ri * p.B + b) * p.Hq + hq) * 2 * p.stats_ld;
+    const float* stats = p.stats + (((int64_t)ri * p.B + b) * p.Hq + hq) * p.stats_ld;
     for (int i0 = i_start; i0 < w; i0 += kTile) {
       __syncthreads();
       load_tile_t<T, D>(Qs, w, i0, [&](int i) { return qbase + (int64_t)(qoff + i) * D; });
       for (int i = threadIdx.x; i < kTile; i += blockDim.x)
-        st[i] = (i0 + i < w) ? make_float2(stats[i0 + i], stats[p.stats_ld + i0 + i]) : make_float2(0.f, 0.f);
+        st[i] = (i0 + i < w) ? stats[i0 + i] : kNegInf;
       __syncthreads();
       float acc[4][4] = {};
 #pragma unroll 8
@@ -182,11 +180,11 @@ __global__ void __launch_bounds__(256) colsum_kernel(const __grid_constant__ Sta
       for (int r = 0; r < 4; ++r) {
         const int i = i0 + tx * 4 + r;
         const int pos = T_b - w + i;
-        const float2 ml = st[tx * 4 + r];
+        const float nml = st[tx * 4 + r];
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
           const int j = j0 + ty * 4 + q;
-          if (i < w && j <= pos) tile[q] += fast_exp2(acc[q][r] * p.scale_log2 + ml.x) * ml.y;
+          if (i < w && j <= pos) tile[q] += fast_exp2(acc[q][r] * p.scale_log2 + nml);
         }
       }
 #pragma unroll

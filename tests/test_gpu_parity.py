@@ -36,11 +36,14 @@ def _tol(dtype):
 
 def static_band(qw, K, scale, w, G):
     """Relative error bound of the GPU's accumulated scores: fp32 dot products
-    over d channels (|error| <= d u sum|q k|), the log2 rescale, two ex2.approx
-    per probability and the row / column sums."""
+    over d channels (|error| <= d u sum|q k|), the log2 rescale and the row
+    statistic -(m + log2 l) folded into the exponent (four roundings of
+    magnitude up to scale log2(e) A, and log2 l <= log2 T), two ex2.approx per
+    probability and the row / column sums."""
     A = (np.abs(qw.reshape(-1, qw.shape[-1])) @ np.abs(K).T).max()
     d, T = K.shape[1], K.shape[0]
-    return 2 * scale * d * U * A + 3 * U * scale * 1.4427 * A + 4 * 2.0 ** -22 + (T / 64 + w * G / 64 + 64) * U
+    return (2 * scale * d * U * A + 4 * U * scale * 1.4427 * A + 3 * U * math.log2(T) + 4 * 2.0 ** -22
+            + (T / 64 + w * G / 64 + 64) * U)
 
 
 def select_band(q_group, levels):
