@@ -31,8 +31,11 @@ if ROOT not in sys.path:
 
 from paper_2501_06807_gb300 import synth  # noqa: E402
 
-METRIC = "selected-KV tokens/s"
-UNIT = "tokens/s"
+# The headline metric names three figures; `value` is the last (selected KV
+# tokens attended per second over the whole job), and the line also carries
+# the decode-step latency (decode_step_us) and its HBM GB/s (decode).
+METRIC = "decode-step latency (\u00b5s) and achieved HBM GB/s vs ~8 TB/s; selected-KV tokens/s"
+UNIT = "selected-KV tokens/s"
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 # fp32 FFMA peak of a GB300 at its maximum SM clock: 152 SMs x 128 lanes x 2 flops
