@@ -28,6 +28,7 @@
 namespace mpc {
 
 constexpr int kRankMax = 1024;  // candidates ranked by counting
+
 constexpr int kSelChunk = 8192; // bytes per bulk copy
 
 __device__ __forceinline__ unsigned long long sel_key(float score, int id) {
@@ -60,12 +61,13 @@ __device__ __forceinline__ void warp_copy(void* dst, const void* src, uint32_t n
 }
 
 template <typename T, int D, int NT>
-__global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ SelectParams p) {
+__global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ SelectParams p) {
   constexpr int NW = NT / 32;
   constexpr int LPR = D / 4;     // lanes per representative row (one float4 each)
   constexpr int RPW = 32 / LPR;  // rows per warp-wide read
   constexpr int U = 8;           // rows per lane per pass
   constexpr uint32_t ROWB = D * 4;
+  constexpr int kFastMax = 16 * NW;  // candidates ranked from registers (NW / 2 keys per lane)
   extern __shared__ __align__(128) uint8_t smem[];
   const int MC = p.max_cand, RB = p.row_buf;
   const SelLayout L(D, MC, RB);
@@ -79,6 +81,7 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   __shared__ __align__(8) uint64_t s_bar;
   __shared__ int s_C[kMaxLevels], s_k[kMaxLevels];
   __shared__ int s_nk, s_next;
+  __shared__ uint32_t s_wmask[NW];
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int c4 = lane % LPR, sub = lane / LPR;
@@ -223,8 +226,78 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
       }
     }
 
-    // 1. mark[i] = candidate i is among the k largest keys
     const int k = min(s_k[l], n);
+    if (n <= kFastMax) {
+      // rank, compact and expand in two barriers: every lane holds its
+      // share of the keys; warp w ranks candidates [w C, w C + C) with one
+      // warp-wide reduction each and records the kept ones in a bit mask;
+      // after a barrier each warp places its kept clusters (and their
+      // children) at the offset given by the masks of the warps before it
+      constexpr int MJ = kFastMax / 32;  // keys per lane
+      const int C = (n + NW - 1) / NW;
+      const int c0 = warp * C;
+      unsigned long long kj[MJ];
+#pragma unroll
+      for (int m = 0; m < MJ; ++m) kj[m] = lane + 32 * m < n ? keysA[lane + 32 * m] : 0ull;  // 0 is below every key
+      uint32_t wmask = 0;
+      for (int c = 0; c < C && c0 + c < n; ++c) {
+        const unsigned long long ki = keysA[c0 + c];
+        int cnt = 0;
+#pragma unroll
+        for (int m = 0; m < MJ; ++m) cnt += (int)(kj[m] > ki);
+        if (k >= n || __reduce_add_sync(0xffffffffu, cnt) < k) wmask |= 1u << c;
+      }
+      if (lane == 0) s_wmask[warp] = wmask;
+      __syncthreads();
+      // kept before this warp, kept in total, and the last kept candidate
+      const int cw = lane < NW ? __popc(s_wmask[lane]) : 0;
+      int incl = cw;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      const int before = __shfl_sync(0xffffffffu, incl - cw, warp);
+      const int total = __shfl_sync(0xffffffffu, incl, 31);
+      const unsigned has = __ballot_sync(0xffffffffu, cw > 0);
+      int nn = 0;
+      if (l > 0 && total > 0) {
+        const int wl = 31 - __clz(has);
+        const int last = key_id(keysA[wl * C + 31 - __clz(s_wmask[wl])]);
+        nn = (total - 1) * f + min(f, nC - last * f);
+      }
+      const bool fits = l == 0 || nn <= MC;
+      for (uint32_t mk = wmask; mk != 0 && fits; mk &= mk - 1) {
+        const int c = __ffs(mk) - 1;
+        const int pos = before + __popc(wmask & ((1u << c) - 1u));
+        const int i = c0 + c;
+        const int id = key_id(keysA[i]);
+        if (l == 0) {
+          if (lane == 0 && pos < p.sel_cap) out[pos] = id;
+        } else {
+          for (int j = lane; j < f; j += 32) {
+            const int cid = id * f + j;
+            if (cid < nC) keysB[pos * f + j] = have_child ? sel_key(cs[i * f + j], cid) : sel_key(0.f, cid);
+          }
+        }
+      }
+      nk = total;
+      if (l == 0) break;
+      if (!fits) {
+        overflow = true;
+        break;
+      }
+      need_score = !have_child;
+      have_child = false;
+      n = nn;
+      __syncthreads();
+      unsigned long long* t = keysA;
+      keysA = keysB;
+      keysB = t;
+      continue;
+    }
+
+    // 1. mark[i] = candidate i is among the k largest keys
     if (k >= n) {
       for (int i = tid; i < n; i += NT) mark[i] = 1;
     } else if (n <= kRankMax) {
@@ -298,6 +371,7 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
           nkw += __popc(bal[c]);
         }
       }
+      __syncwarp();
       if (lane == 0) {
         s_nk = nkw;
         // children of the kept clusters: all full except possibly the last
@@ -343,8 +417,9 @@ __global__ void __launch_bounds__(NT) select_kernel(const __grid_constant__ Sele
   if (tid == 0 && h == 0 && ri == 0) p.out_n_sel[b] = nk;
 }
 
-// Threads per CTA: 16 warps while the units fit one wave of SMs, else 8.
-static int select_threads(int units) { return units <= 152 ? 512 : 256; }
+// Threads per CTA: 16 warps while the units fit one wave of SMs, 8 while
+// they fit two CTAs per SM, else 4 (up to five CTAs per SM).
+static int select_threads(int units) { return units <= 152 ? 512 : (units <= 304 ? 256 : 128); }
 
 int select_smem_bytes(int D, int max_cand, int row_buf) { return (int)SelLayout(D, max_cand, row_buf).total; }
 
@@ -361,7 +436,8 @@ cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cu
 #define MPC_SEL(TT, DD)                                                                     \
   if (D == DD) {                                                                            \
     if (nt == 512) return launch_sel(select_kernel<TT, DD, 512>, units, nt, smem, st, p);  \
-    return launch_sel(select_kernel<TT, DD, 256>, units, nt, smem, st, p);                 \
+    if (nt == 256) return launch_sel(select_kernel<TT, DD, 256>, units, nt, smem, st, p);  \
+    return launch_sel(select_kernel<TT, DD, 128>, units, nt, smem, st, p);                 \
   }
   if (dtype == MPC_BF16) {
     MPC_SEL(bf16, 64)
