@@ -72,6 +72,23 @@ def rules(w):
     return R, leaders
 
 
+def select_rows(w, n_tok):
+    """Representative rows the hierarchical selection of one (leader, b, kv
+    head) scores for a cache of n_tok rows: every cluster of the coarsest
+    level, then the children of each level's kept clusters."""
+    from paper_2501_06807_gb300 import mpcache
+    C = [n_tok // w.cluster_size]
+    for f in w.fanouts:
+        C.append(-(-C[-1] // f))
+    rows, cand = 0, C[-1]
+    for l in range(len(C) - 1, -1, -1):
+        rows += cand
+        k = min(mpcache.ppm_count(C[l], w.level_keep_ppm[l]), cand)
+        if l > 0:
+            cand = min(C[l - 1], k * w.fanouts[l - 1])
+    return rows
+
+
 def static_flops(w, lens, n_leaders):
     """Algorithmic FLOPs of the two score passes: every (window row, causal
     key) pair of every leader layer and query head, 2 d flops per pass."""
@@ -165,12 +182,14 @@ def run_ours(args, rank, world, dist):
     attended = 0
     n_keep = eng.n_keep.cpu().tolist()
     s = w.cluster_size
+    rep_rows = 0
     for e in range(E):
         eng.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=out_all[e])
         n_sel = eng.n_sel.cpu().tolist()
         for b in range(w.batch):
             n_tok = n_keep[b] + e
             attended += (n_sel[b] * s + n_tok % s + 1) * w.n_layers * w.n_kv_heads
+            rep_rows += select_rows(w, n_tok) * len(leaders) * w.n_kv_heads
     status = mpcache.device_status()
     if status != 0:
         raise RuntimeError(f"device status {status} after the eager pass")
@@ -261,14 +280,16 @@ def run_ours(args, rank, world, dist):
     flops = static_flops(w, [int(t) for t in x.prompt_lens], n_lead)
     static_tflops = flops / (static_ms / 1e3) / 1e12
     esz = 2 if w.dtype == "bf16" else 4
-    # decode bytes: attended K and V rows, the leaders' summaries read by the
-    # selection (upper bound: every level's candidates), q, k_new, v_new, o
+    # decode bytes: attended K and V rows, the fp32 representatives the
+    # selection scores (each level's candidates), q, k_new, v_new, o
     kv_bytes = attended * w.head_dim * 2 * esz
+    rep_bytes = rep_rows * w.head_dim * 4
     io_bytes = E * w.n_layers * w.batch * (w.n_q_heads * w.head_dim * (esz + 4) + 2 * w.n_kv_heads * w.head_dim * esz)
-    dec_bytes = kv_bytes + io_bytes
+    dec_bytes = kv_bytes + rep_bytes + io_bytes
     decode_gbs = dec_bytes / (decode_ms / 1e3) / 1e9
     dominant_static = static_ms >= decode_ms
-    tensor_path = w.dtype == "bf16" and not w.paged
+    # bf16 keys score on tcgen05, dense or in pages of 8..128 rows dividing 128
+    tensor_path = w.dtype == "bf16" and (not w.paged or (w.page_size >= 8 and 128 % w.page_size == 0))
     if dominant_static and tensor_path:
         # tcgen05 score passes; the kernel runs inside a long step, so the
         # sustained bf16 figure is the denominator

@@ -78,7 +78,11 @@ struct StaticParams {
 // Window scoring on tcgen05 (bf16 queries and dense keys).
 struct ScoreTcParams {
   CUtensorMap map_q;  // [layer][B*Hq*win_rows][d], 128 x 64 boxes, 128B swizzle
-  CUtensorMap map_k;  // [layer][B*Hkv*t_max][d]
+  CUtensorMap map_k;  // dense [layer][B*Hkv*t_max][d] (128-row boxes) or the
+                      // page pool [layer][pages*Hkv*page_size][d] (page-row boxes)
+  const int* page_table;  // null for dense keys
+  int page_size, max_pages;
+  int64_t pool_pages;     // pages per layer of the pool
   RefTable refs;
   int n_refs, B, Hq, Hkv, G, t_max, win_rows;
   const int* lens;

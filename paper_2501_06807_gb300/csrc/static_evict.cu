@@ -306,8 +306,11 @@ static cudaError_t set_smem(K kernel, int bytes) {
 
 cudaError_t launch_static(const StaticParams& p, int dtype, int D, int n_layer_span, cudaStream_t st) {
   cudaError_t e = cudaSuccess;
-  if (dtype == MPC_BF16 && p.page_table == nullptr) {
-    // both score passes on the tensor cores
+  const bool tc_pages = p.page_table == nullptr ||
+                        (p.page_size >= 8 && p.page_size <= 128 && 128 % p.page_size == 0 && p.k_ls > 0);
+  if (dtype == MPC_BF16 && tc_pages) {
+    // both score passes on the tensor cores (dense keys, or pages of 8 to
+    // 128 rows that tile a 128-key block)
     ScoreTcParams t;
     memset(&t, 0, sizeof(t));
     t.refs = p.refs;
@@ -330,6 +333,9 @@ cudaError_t launch_static(const StaticParams& p, int dtype, int D, int n_layer_s
     t.scores = p.scores;
     t.stats = p.stats;
     t.stats_ld = p.stats_ld;
+    t.page_table = p.page_table;
+    t.page_size = p.page_size;
+    t.max_pages = p.max_pages;
     if ((e = launch_score_tc(t, D, n_layer_span, st)) != cudaSuccess) return e;
   } else {
     const int smem = static_tile_smem(D);
