@@ -253,11 +253,14 @@ int validate_select(const mpc_select_args* a, SelectParams* p) {
   p->out_n_sel = a->out_n_sel;
   p->max_cand = P;
   // rows staged in shared memory at once: the first round (the coarsest
-  // level plus the level below it) and each later round (the children of a
-  // level's kept clusters), capped by what shared memory holds
+  // level, plus the level below it when the units are few) and each later
+  // round (the children of a level's kept clusters), capped by what shared
+  // memory holds
   const int top = a->n_levels - 1;
-  long long need = (long long)p->pyr.cap[top] + (top > 0 ? p->pyr.cap[top - 1] : 0);
-  for (int l = top - 2; l >= 0; --l) {
+  p->spec_first = select_spec_first(a->n_refs * a->batch * a->n_kv_heads);
+  const bool spec = p->spec_first && top > 0;
+  long long need = (long long)p->pyr.cap[top] + (spec ? p->pyr.cap[top - 1] : 0);
+  for (int l = spec ? top - 2 : top - 1; l >= 0; --l) {
     long long r = (long long)p->pyr.fanout[l] * kmax[l + 1];
     if (r > p->pyr.cap[l]) r = p->pyr.cap[l];
     if (r > need) need = r;

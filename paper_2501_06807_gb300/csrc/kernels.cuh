@@ -52,6 +52,7 @@ struct SelectParams {
   int* out_n_sel;
   int max_cand;  // power of two, capacity of the shared candidate arrays
   int row_buf;   // representative rows staged in shared memory at once
+  int spec_first;  // the first round also scores the whole level below the coarsest
 };
 
 struct StaticParams {
@@ -129,6 +130,7 @@ int attn_persist_ctas_max();
 int attn_persist_batch_max();
 cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cudaStream_t st);
 int select_smem_bytes(int D, int max_cand, int row_buf);
+int select_spec_first(int units);
 cudaError_t launch_clusters(const ClusterParams& p, int dtype, int D, int n_units, int groups_x,
                             bool any_leader, cudaStream_t st);
 cudaError_t launch_static(const StaticParams& p, int dtype, int D, int n_layer_span, cudaStream_t st);

@@ -11,10 +11,11 @@
 // a level needs are staged in shared memory by 1-D bulk copies (contiguous
 // runs: the whole coarsest level, or the children of one kept cluster) on
 // one mbarrier, and scoring is batched into as few dependent rounds as the
-// pyramid allows.  The first round, requested before q and the token count
-// arrive, copies the coarsest level and, when they fit the staging buffer,
-// all clusters of the level below it, whose scores then need no round of
-// their own (a three-level pyramid takes two rounds).  Per level, with a
+// pyramid allows.  The first round, requested as soon as the token count
+// arrives (while q is still loading), copies the coarsest level and, while
+// the units are few enough to be latency-bound and both fit the staging
+// buffer, all clusters of the level below it, whose scores then need no
+// round of their own (a three-level pyramid takes two rounds).  Per level, with a
 // block barrier after each step:
 //   1. rank: a candidate is kept iff fewer than k keys are larger, counted
 //      by up to 32 threads per candidate over shared memory (a bitonic sort
@@ -140,22 +141,26 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   grid_dep_launch();
   grid_dep_wait();
 
-  // ---- first round, requested up front: rows [0, nT0) of the coarsest
-  // level at buffer row 0 and, when spec0, rows [0, capC) of the level
-  // below it at buffer row capT
+  // ---- first round, requested as soon as the token count is known: the
+  // clusters [0, nT) of the coarsest level at buffer row 0 and, when spec0,
+  // all clusters of the level below it at buffer row capT
   const int capT = p.pyr.cap[top];
   const int capC = top > 0 ? p.pyr.cap[top - 1] : 0;
-  const bool spec0 = top > 0 && capT + capC <= RB;
+  const bool spec0 = p.spec_first && top > 0 && capT + capC <= RB;
   const int nT0 = capT < RB ? capT : RB;
   const float* repT = rep0 + (int64_t)p.pyr.off[top] * D;
   const float* repC = rep0 + (int64_t)(top > 0 ? p.pyr.off[top - 1] : 0) * D;
-  if (warp == 0) {
-    if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)(nT0 + (spec0 ? capC : 0)) * ROWB);
-    __syncwarp();
-    warp_copy(rows, repT, (uint32_t)nT0 * ROWB, &s_bar, lane);
-    if (spec0) warp_copy(rows + (size_t)capT * D, repC, (uint32_t)capC * ROWB, &s_bar, lane);
-  }
   const int ntok = p.n_tok[b];
+  int C[kMaxLevels];
+  level_counts(p.pyr, ntok, C);
+  if (warp == 0) {
+    const int nT = max(0, min(C[top], nT0));
+    const int nCc = spec0 ? max(0, min(C[top - 1], capC)) : 0;
+    if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)(nT + nCc) * ROWB);
+    __syncwarp();
+    warp_copy(rows, repT, (uint32_t)nT * ROWB, &s_bar, lane);
+    if (nCc > 0) warp_copy(rows + (size_t)capT * D, repC, (uint32_t)nCc * ROWB, &s_bar, lane);
+  }
 
   // q_sum = sum over the group's query heads (fixed order)
   const T* qp = (const T*)p.q + layer * p.q_ls + ((int64_t)b * p.Hq + h * G) * D;
@@ -164,8 +169,6 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
     for (int g = 0; g < G; ++g) acc += to_float<T>(qp[g * D + c]);
     qsum[c] = acc;
   }
-  int C[kMaxLevels];
-  level_counts(p.pyr, ntok, C);
   if (tid < kMaxLevels) {
     s_C[tid] = C[tid];
     s_k[tid] = tid < p.pyr.n_levels ? count_from_ppm(C[tid], p.keep_ppm[tid]) : 0;
@@ -422,6 +425,11 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
 static int select_threads(int units) { return units <= 152 ? 512 : (units <= 304 ? 256 : 128); }
 
 int select_smem_bytes(int D, int max_cand, int row_buf) { return (int)SelLayout(D, max_cand, row_buf).total; }
+
+// Scoring the whole level below the coarsest in the first round saves a
+// dependent round but reads the children of unkept clusters too: worth it
+// while the units fit two CTAs per SM (latency-bound), not beyond.
+int select_spec_first(int units) { return units <= 2 * 152 ? 1 : 0; }
 
 template <typename K>
 static cudaError_t launch_sel(K kernel, int units, int nt, int smem, cudaStream_t st, const SelectParams& p) {
