@@ -180,21 +180,24 @@ def _off(eng, level):
 # ------------------------------------------------- selection in isolation ----
 
 SELECT_CASES = [
-    # dtype, d, Hq, Hkv, s, fanouts, keep ppm (finest first), n_tok
-    (torch.float32, 64, 3, 3, 16, (), (250_000,), 16 * 37 + 5),
-    (torch.bfloat16, 128, 4, 4, 16, (4,), (125_000, 500_000), 1024),
-    (torch.bfloat16, 128, 32, 8, 16, (8, 8), (50_000, 250_000, 500_000), 8192 + 7),
-    (torch.bfloat16, 128, 8, 2, 16, (8,), (100_000, 500_000), 2048 + 15),
-    (torch.bfloat16, 64, 2, 1, 1, (), (30_000,), 3000),       # token-wise (s = 1)
-    (torch.float32, 128, 2, 1, 4, (3, 2), (200_000, 400_000, 600_000), 997),
-    (torch.bfloat16, 128, 4, 1, 16, (4,), (1_000_000, 1_000_000), 320),  # keep all
+    # dtype, d, Hq, Hkv, s, fanouts, keep ppm (finest first), n_tok, batch
+    (torch.float32, 64, 3, 3, 16, (), (250_000,), 16 * 37 + 5, 2),
+    (torch.bfloat16, 128, 4, 4, 16, (4,), (125_000, 500_000), 1024, 2),
+    (torch.bfloat16, 128, 32, 8, 16, (8, 8), (50_000, 250_000, 500_000), 8192 + 7, 2),
+    (torch.bfloat16, 128, 8, 2, 16, (8,), (100_000, 500_000), 2048 + 15, 2),
+    (torch.bfloat16, 64, 2, 1, 1, (), (30_000,), 3000, 2),       # token-wise (s = 1): sort path
+    (torch.float32, 128, 2, 1, 4, (3, 2), (200_000, 400_000, 600_000), 997, 2),
+    (torch.bfloat16, 128, 4, 1, 16, (4,), (1_000_000, 1_000_000), 320, 2),  # keep all
+    (torch.bfloat16, 128, 2, 1, 4, (), (150_000,), 2003, 2),     # 500 candidates: counting-rank path
+    (torch.bfloat16, 128, 40, 20, 16, (4,), (125_000, 500_000), 700, 8),  # 160 units: 8-warp CTAs
+    (torch.bfloat16, 64, 40, 40, 16, (4,), (125_000, 500_000), 600, 8),   # 320 units: 4-warp CTAs
 ]
 
 
-@pytest.mark.parametrize("dtype,d,Hq,Hkv,s,fan,keep,N", SELECT_CASES)
-def test_selection(dtype, d, Hq, Hkv, s, fan, keep, N):
+@pytest.mark.parametrize("dtype,d,Hq,Hkv,s,fan,keep,N,B", SELECT_CASES)
+def test_selection(dtype, d, Hq, Hkv, s, fan, keep, N, B):
     g = torch.Generator().manual_seed(N + d)
-    L, B = 1, 2
+    L = 1
     G = Hq // Hkv
     eng = H.make_engine(synth.Workload("t", L, B, Hq, Hkv, d, "f32" if dtype == torch.float32 else "bf16",
                                        N, N, O.PPM, s, fan, keep, 1, 4, "iid"), 4)
@@ -227,7 +230,7 @@ def test_selection(dtype, d, Hq, Hkv, s, fan, keep, N):
                     ties += 1
                     assert np.all(np.diff(got) > 0) and got.min(initial=0) >= 0
                     assert got.max(initial=-1) < N // s
-    assert ties <= 1
+    assert ties <= max(1, 3 * B * Hkv // 100)
 
 
 # ----------------------------------------------- static eviction alone ----
