@@ -159,11 +159,13 @@ int validate_static(const mpc_static_args* a, StaticParams* p) {
 }
 
 // Row statistics (m, 1/l) of every window row.
-// Row statistics of the window: per (ref, b, query head) one array of
-// -(m + log2 l), padded to a multiple of 128 rows (one bulk copy per row tile).
+// Row statistics of the window, per (ref, b, query head), rows padded to a
+// multiple of 128 (one bulk copy per row tile): -(m + log2 l) as fp32 for
+// the SIMT passes, then the same value over the log2 scale as three bf16
+// parts in a 16-byte row for the tcgen05 passes.
 int stats_ld_of(int win_rows) { return (win_rows + 127) / 128 * 128; }
 size_t static_ws(const StaticParams& p) {
-  return (size_t)p.n_refs * p.B * p.Hq * stats_ld_of(p.win_rows) * sizeof(float);
+  return (size_t)p.n_refs * p.B * p.Hq * stats_ld_of(p.win_rows) * (sizeof(float) + 16);
 }
 
 // ------------------------------------------------------------ clusters ----
@@ -433,6 +435,7 @@ MPC_API int mpc_static_evict(const mpc_static_args* args, void* workspace, size_
   if (!aligned16(workspace)) return fail(MPC_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
   p.stats = static_cast<float*>(workspace);
   p.stats_ld = stats_ld_of(p.win_rows);
+  p.aug = static_cast<uint8_t*>(workspace) + (size_t)p.n_refs * p.B * p.Hq * p.stats_ld * sizeof(float);
   int span = 0;
   for (int i = 0; i < args->n_refs; ++i) span = args->refs[i].layer + 1 > span ? args->refs[i].layer + 1 : span;
   const cudaError_t e = launch_static(p, args->dtype, args->head_dim, span, static_cast<cudaStream_t>(stream));

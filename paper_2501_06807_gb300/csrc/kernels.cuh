@@ -72,8 +72,10 @@ struct StaticParams {
   float* scores;      // [group][b][Hkv][t_max]
   int* kept;          // [group][b][Hkv][keep_cap]
   int* n_keep;        // [b]
-  float* stats;       // [ref][b][Hq][stats_ld]: -(m + log2 l) per window row
+  float* stats;       // [ref][b][Hq][stats_ld]: -(m + log2 l) per window row (SIMT passes)
   int stats_ld;       // win_rows rounded up to 128
+  void* aug;          // [ref][b][Hq][stats_ld][8] bf16: -(m + log2 l) / scale_log2 as the sum of
+                      // three bf16 parts, then five zeros (tcgen05 passes)
 };
 
 // Window scoring on tcgen05 (bf16 queries and dense keys).
@@ -96,6 +98,7 @@ struct ScoreTcParams {
   float* scores;
   float* stats;  // as StaticParams::stats
   int stats_ld;
+  void* aug;     // as StaticParams::aug
 };
 
 struct KvSrc {

@@ -12,11 +12,15 @@
 //     A = the 128 key rows (fixed), B = 128-row tiles of window queries of
 //     every query head of the GQA group.  S^T = A B^T puts one key per TMEM
 //     lane, so each thread sums 2^(s_ij - m_i) / l_i over the rows i in its
-//     own registers, in a fixed order (deterministic scores).  Each row's
-//     statistic arrives as -(m_i + log2 l_i) by bulk copy with its query
-//     tile, so a score costs one FMA, one ex2 and one add; rows past the
-//     window carry -inf, so they add exact zeros.
-//
+//     own registers, in a fixed order (deterministic scores).  The row
+//     statistic -(m_i + log2 l_i) enters through the MMA itself: one extra
+//     K = 16 step multiplies a constant key-side operand (1, 1, 1, 0, ...)
+//     with the row's statistic over the log2 scale, stored by pass 0 as three
+//     bf16 parts, so the accumulator holds s_ij + that value and the
+//     epilogue needs one multiply, one ex2 and one add per score and no
+//     shared-memory loads (every lane would need every row's value, and
+//     broadcast loads were this pass's bound).
+
 // Roles: warp 0 issues TMA tile loads (128B-swizzled, K-major boxes of
 // 128 rows x 64 channels), warp 1 allocates TMEM and issues tcgen05.mma
 // (M = N = 128, K = 16, bf16 in, fp32 accumulate) into one of two 128-column
@@ -52,8 +56,9 @@ struct TcSmem {
   static constexpr int A_OFF = 0;
   static constexpr int B_OFF = TILE;
   static constexpr int STAGE = TILE;                // one streamed B tile
-  static constexpr int STATS_OFF = B_OFF + kStagesTc * STAGE;  // pass 1: kStatSlots x 128 -(m + log2 l)
-  static constexpr int XCH_OFF = STATS_OFF + kStatSlots * 128 * 4;  // halves' partials, 128 x float2
+  static constexpr int AUG_OFF = B_OFF + kStagesTc * STAGE;    // pass 1: kStatSlots x 128 rows x 16 B
+  static constexpr int ONE_OFF = AUG_OFF + kStatSlots * 2048;   // pass 1: constant K-side core matrices
+  static constexpr int XCH_OFF = ONE_OFF + 256;                 // halves' partials, 128 x float2
   static constexpr int BAR_OFF = XCH_OFF + 128 * 8;
   static constexpr int USED = BAR_OFF + 256 + 1024;  // + alignment slack
   // at least 80 KB so that at most two CTAs (2 x 256 TMEM columns) share an SM
@@ -189,6 +194,21 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
   return d;
 }
 
+// Shared-memory matrix descriptor without swizzle (K-major): 8-row x 16-byte
+// core matrices stored as 128 contiguous bytes; `lbo` is the byte step
+// between the two core matrices of a 16-element K step, `sbo` the step
+// between 8-row groups.
+__device__ __forceinline__ uint64_t plain_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+  d |= (uint64_t)1 << 46;  // descriptor version of tcgen05; layout 0 = no swizzle
+  return d;
+}
+__device__ __forceinline__ uint32_t pack_bf16_pair(bf16 lo, bf16 hi) {
+  return (uint32_t)__bfloat16_as_ushort(lo) | ((uint32_t)__bfloat16_as_ushort(hi) << 16);
+}
+
 // Instruction descriptor: bf16 A and B (K-major), fp32 D, M = N = 128.
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
 
@@ -226,7 +246,6 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
   uint64_t* stats_empty = stats_full + kStatSlots;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(stats_empty + kStatSlots);
   volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  float* stats_s = reinterpret_cast<float*>(smem + S::STATS_OFF);  // [slot][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // ---- work unit
@@ -270,7 +289,7 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
     }
     for (int i = 0; i < kStatSlots; ++i) {
       mbar_init(&stats_full[i], 1);
-      mbar_init(&stats_empty[i], kTcEpiWarps);
+      mbar_init(&stats_empty[i], 1);  // released by the MMA that read the slot
     }
     *abort = 0;
     fence_barrier_init();
@@ -278,6 +297,15 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
   if (warp == 1) {
     tmem_alloc(tmem_slot, 256);
     tmem_relinquish();
+  }
+  if (PASS == 1 && threadIdx.x >= 64 && threadIdx.x < 80) {
+    // K-side operand of the statistic step: one 8-row core matrix whose rows
+    // are (1, 1, 1, 0, 0, 0, 0, 0) (every 8-row group reuses it), then a zero
+    // core matrix for channels 8..15
+    const int i = threadIdx.x - 64;
+    reinterpret_cast<uint4*>(smem + S::ONE_OFF)[i] =
+        i < 8 ? make_uint4(0x3F803F80u, 0x00003F80u, 0u, 0u) : make_uint4(0u, 0u, 0u, 0u);
+    fence_proxy_async_smem();
   }
   tc_fence_before();
   __syncthreads();
@@ -343,13 +371,14 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
         for (int kh = 0; kh < KH; ++kh)
           tma_load_3d(st + kh * kBoxBytes, &p.map_q, kh * 64, qrow0 + hq * p.win_rows + it, layer, &full[s]);
         n_issued = t + 1;
-        // the rows' -(m + log2 l) into their ring slot, once the epilogue
-        // has finished the tile that used the slot before
+        // the rows' statistic (16 bytes per row) into their ring slot, once
+        // the MMA that read the slot before has completed
         const int sb = t % kStatSlots;
         if (t >= kStatSlots && !wait_or_abort(&stats_empty[sb], ((t / kStatSlots) - 1) & 1, abort)) break;
-        const float* src = p.stats + (((int64_t)ri * p.B + b) * p.Hq + hq) * p.stats_ld + it;
-        mbar_arrive_expect_tx(&stats_full[sb], 512);
-        bulk_g2s(stats_s + sb * 128, src, 512, &stats_full[sb]);
+        const uint8_t* src =
+            static_cast<const uint8_t*>(p.aug) + ((((int64_t)ri * p.B + b) * p.Hq + hq) * p.stats_ld + it) * 16;
+        mbar_arrive_expect_tx(&stats_full[sb], 2048);
+        bulk_g2s(smem + S::AUG_OFF + sb * 2048, src, 2048, &stats_full[sb]);
         n_stats = t + 1;
       }
       n_issued = t + 1;
@@ -372,12 +401,20 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
         const int s = t % kStagesTc, buf = t & 1;
         if (!wait_or_abort(&full[s], (t / kStagesTc) & 1, abort)) break;
         if (t >= 2 && !wait_or_abort(&acc_empty[buf], ((t >> 1) - 1) & 1, abort)) break;
+        if (PASS == 1 && !wait_or_abort(&stats_full[t % kStatSlots], (t / kStatSlots) & 1, abort)) break;
         tc_fence_after();
         const uint32_t b_base = smem_u32(smem + S::B_OFF + s * S::STAGE);
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t off = (kk >> 2) * kBoxBytes + (kk & 3) * 32;
           umma_bf16(tmem + buf * 128, sw128_desc(a_base + off), sw128_desc(b_base + off), kIdesc, kk > 0);
+        }
+        if (PASS == 1) {
+          // one more K step adds the rows' statistic: S^T + (x1 + x2 + x3)
+          const int sb = t % kStatSlots;
+          umma_bf16(tmem + buf * 128, plain_desc(smem_u32(smem + S::ONE_OFF), 128, 0),
+                    plain_desc(smem_u32(smem + S::AUG_OFF + sb * 2048), 0, 128), kIdesc, 1);
+          umma_commit(&stats_empty[sb]);
         }
         umma_commit(&empty[s]);
         umma_commit(&acc_full[buf]);
@@ -404,8 +441,7 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
     int t = 0;
     for (; t < n_tiles; ++t) {
       const int buf = t & 1;
-      bool ok = wait_or_abort(&acc_full[buf], (t >> 1) & 1, abort);
-      if (PASS == 1 && ok) ok = wait_or_abort(&stats_full[t % kStatSlots], (t / kStatSlots) & 1, abort);
+      const bool ok = wait_or_abort(&acc_full[buf], (t >> 1) & 1, abort);
       if (!epilogue_all(ok)) break;
       tc_fence_after();
       if (PASS == 0) {
@@ -438,9 +474,10 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
         }
       } else {
         const int it = i_start + (t % tiles_per_g) * 128 + col0;  // first row of this thread's columns
-        const float* nm_s = stats_s + (t % kStatSlots) * 128 + col0;
-        // row i sees key j when j <= base + i; rows past the window have -m = -inf
+        // the accumulator already holds s + statistic / scale_log2 (about
+        // -3e38 past the window); row i sees key j when j <= base + i
         const bool need_mask = j0 + 127 > base + it;
+        const uint64_t zero2 = pk2(0.f, 0.f);
         uint64_t s2 = pk2(0.f, 0.f);
 #pragma unroll 1
         for (int c = 0; c < 2; ++c) {
@@ -452,11 +489,7 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
               if (j_key > base + it + c * 32 + k) v[k] = kNegInf;
           }
 #pragma unroll
-          for (int k = 0; k < 32; k += 4) {
-            const float4 nm4 = *reinterpret_cast<const float4*>(nm_s + c * 32 + k);
-            s2 = fadd2(s2, exp2_mufu2(ffma2(pk2(v[k], v[k + 1]), sc2, pk2(nm4.x, nm4.y))));
-            s2 = fadd2(s2, exp2_mufu2(ffma2(pk2(v[k + 2], v[k + 3]), sc2, pk2(nm4.z, nm4.w))));
-          }
+          for (int k = 0; k < 32; k += 2) s2 = fadd2(s2, exp2_mufu2(ffma2(pk2(v[k], v[k + 1]), sc2, zero2)));
         }
         float s0, s1;
         upk2(s2, s0, s1);
@@ -464,10 +497,7 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&acc_empty[buf]);
-        if (PASS == 1) mbar_arrive(&stats_empty[t % kStatSlots]);
-      }
+      if (lane == 0) mbar_arrive(&acc_empty[buf]);
     }
     // combine the two column halves of every lane (fixed order: half 0 + half 1)
     float2* xch = reinterpret_cast<float2*>(smem + S::XCH_OFF);
@@ -478,11 +508,22 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
       if (PASS == 0) {
         const float M = fmaxf(m, o.x);
         const float L = (m == kNegInf ? 0.f : l * fast_exp2(m - M)) + (o.x == kNegInf ? 0.f : o.y * fast_exp2(o.x - M));
-        float* st = p.stats + (((int64_t)ri * p.B + b) * p.Hq + head) * p.stats_ld;
-        if (i_row < w)
-          st[i_row] = -(M + log2f(L));
-        else if (i_row < (w + 127) / 128 * 128)
-          st[i_row] = kNegInf;  // past the window: contributes nothing in pass 1
+        // the statistic over the log2 scale, split into three bf16 parts
+        // (x1 + x2 + x3 = x to fp32 precision), so pass 1's extra MMA step
+        // adds it to every score of the row.  Rows past the window get a
+        // large finite negative value (ex2 of it is 0): -inf would meet the
+        // zero channels of the step's other operand and give 0 x inf = NaN
+        uint4* ar = reinterpret_cast<uint4*>(p.aug) + (((int64_t)ri * p.B + b) * p.Hq + head) * p.stats_ld + i_row;
+        if (i_row < w) {
+          const float x = -(M + log2f(L)) / p.scale_log2;
+          const bf16 x1 = __float2bfloat16_rn(x);
+          const float r1 = x - __bfloat162float(x1);
+          const bf16 x2 = __float2bfloat16_rn(r1);
+          const bf16 x3 = __float2bfloat16_rn(r1 - __bfloat162float(x2));
+          *ar = make_uint4(pack_bf16_pair(x1, x2), pack_bf16_pair(x3, __float2bfloat16_rn(0.f)), 0u, 0u);
+        } else if (i_row < (w + 127) / 128 * 128) {
+          *ar = make_uint4(pack_bf16_pair(__float2bfloat16_rn(-3.0e38f), __float2bfloat16_rn(0.f)), 0u, 0u, 0u);
+        }
       } else if (j_key < T_b) {
         p.scores[((int64_t)(group * p.B + b) * p.Hkv + head) * p.t_max + j_key] = acc + o.x;
       }

@@ -333,6 +333,7 @@ cudaError_t launch_static(const StaticParams& p, int dtype, int D, int n_layer_s
     t.scores = p.scores;
     t.stats = p.stats;
     t.stats_ld = p.stats_ld;
+    t.aug = p.aug;
     t.page_table = p.page_table;
     t.page_size = p.page_size;
     t.max_pages = p.max_pages;

@@ -141,9 +141,9 @@ def test_select_and_static_validation(lib):
     a.t_max, a.win_rows, a.keep_cap = 32768, 4916, 8192
     a.window_ppm, a.long_window_ppm, a.long_prompt_threshold, a.keep_ppm = 200_000, 100_000, 24576, 250_000
     rc, n = _ws(lib, "mpc_static_evict_workspace_size", a)
-    # row statistics: one fp32 array -(m + log2 l) per (ref, b, query head),
-    # rows padded to a multiple of 128 (4916 -> 4992)
-    assert rc == 0 and n == 1 * 2 * 8 * 4992 * 4
+    # row statistics per (ref, b, query head), rows padded to a multiple of
+    # 128 (4916 -> 4992): fp32 -(m + log2 l), plus a 16-byte bf16 row
+    assert rc == 0 and n == 1 * 2 * 8 * 4992 * (4 + 16)
     a.win_rows = 4915      # the longest window (T = 24576) needs 4916 rows
     assert _ws(lib, "mpc_static_evict_workspace_size", a)[0] == mpcache.MPC_ERR_BAD_SHAPE
     a.win_rows, a.keep_cap = 4916, 8191
