@@ -72,6 +72,31 @@ def rules(w):
     return R, leaders
 
 
+# ---------------------------------------------------------- replicas ----
+#
+# The path has no exchange step: --gpus N runs N independent replicas (one
+# process per GPU, each with its own seeded workload) and reports the units
+# all ranks processed over the slowest rank's time.
+
+def replica_workload(w, rank):
+    """The workload of one replica: rank r draws its inputs from seed + 7919 r."""
+    return w.replace(seed=w.seed + 7919 * rank) if rank else w
+
+
+def max_over_ranks(x, dist, device=None):
+    """max over the ranks of a float (a time), through one all-reduce."""
+    if dist is None:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(units_per_rank, world, ms):
+    """Whole-job throughput: the units every rank processed over the slowest time."""
+    return units_per_rank * world / (ms / 1e3)
+
+
 def select_rows(w, n_tok):
     """Representative rows the hierarchical selection of one (leader, b, kv
     head) scores for a cache of n_tok rows: every cluster of the coarsest
@@ -153,9 +178,7 @@ def run_ours(args, rank, world, dist):
     mpcache.load()
     dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
     torch.cuda.set_device(dev)
-    w = synth.WORKLOADS[args.workload]
-    if world > 1:
-        w = w.replace(seed=w.seed + 7919 * rank)  # independent replica per rank
+    w = replica_workload(synth.WORKLOADS[args.workload], rank)
     E = args.decode_steps or w.decode_steps
     R, leaders = rules(w)
     x = synth.generate(w, R, device="cuda", decode_steps=E)
@@ -229,16 +252,12 @@ def run_ours(args, rank, world, dist):
     clk = clocks.stop()
     if dist is not None:
         dist.barrier()
-    total_ms = t_start.elapsed_time(t_end)
+    total_ms = max_over_ranks(t_start.elapsed_time(t_end), dist, dev)
     static_ms = sum(m[0].elapsed_time(m[1]) for m in marks) / args.steps
     build_ms = sum(m[1].elapsed_time(m[2]) for m in marks) / args.steps
     decode_ms = sum(m[2].elapsed_time(m[3]) for m in marks) / args.steps
-    if dist is not None:
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
     ms_per_step = total_ms / args.steps
-    value = attended * world / (ms_per_step / 1e3)
+    value = job_value(attended, world, ms_per_step)
 
     # e2e through the public API with host buffers
     e2e = None
@@ -267,12 +286,8 @@ def run_ours(args, rank, world, dist):
             e2e_step()
         b.record(stream)
         torch.cuda.synchronize()
-        e2e_ms = a.elapsed_time(b) / args.steps
-        if dist is not None:
-            t = torch.tensor([e2e_ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_ms = float(t.item())
-        e2e = {"value": attended * world / (e2e_ms / 1e3), "unit": UNIT, "ms_per_step": e2e_ms,
+        e2e_ms = max_over_ranks(a.elapsed_time(b) / args.steps, dist, dev)
+        e2e = {"value": job_value(attended, world, e2e_ms), "unit": UNIT, "ms_per_step": e2e_ms,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
 
     pk, pk_kind = peaks()
