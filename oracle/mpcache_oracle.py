@@ -186,24 +186,33 @@ def cluster_pyramid(keys: np.ndarray, s: int, fanouts: Sequence[int],
 
 def hierarchical_select(q_group: np.ndarray, levels: List[Level],
                         fanouts: Sequence[int], level_keep_ppm: Sequence[int],
-                        trace: Optional[list] = None) -> np.ndarray:
+                        trace: Optional[list] = None, metric: str = "eq3") -> np.ndarray:
     """Coarse-to-fine cluster selection (Sec. 3.3; Alg. 2 Sim + topk).
 
-    q_group: [G][d] decode queries of one kv group; the similarity of cluster c
-    is (sum_g q_g) . rep_c (Eq. 3 summed over the group).  At the coarsest
-    level every cluster is a candidate; at each finer level the candidates are
-    the children of the kept parents.  Returns the kept finest-level ids in
-    ascending order.  ``trace``, if given, receives per level (coarsest
-    first) the candidate ids, their similarities and k, for tests that need
-    the margin at each cut.
+    q_group: [G][d] decode queries of one kv group, scored through their sum
+    q = sum_g q_g.  The similarity of cluster c is q . rep_c (Eq. 3, the
+    default) or, with metric="bound", the upper bound of Eq. 2,
+    sum_i max(q_i r_max_ci, q_i r_min_ci), evaluated on the same summed query.
+    At the coarsest level every cluster is a candidate; at each finer level
+    the candidates are the children of the kept parents.  Returns the kept
+    finest-level ids in ascending order.  ``trace``, if given, receives per
+    level (coarsest first) the candidate ids, their similarities and k, for
+    tests that need the margin at each cut.
     """
+    if metric not in ("eq3", "bound"):
+        raise ValueError(metric)
     qsum = np.asarray(q_group, dtype=np.float64).sum(axis=0)
     n = len(levels)
     cand = np.arange(levels[-1].rep.shape[0])
     kept = cand
     for lvl in range(n - 1, -1, -1):
         lev = levels[lvl]
-        sim = lev.rep[cand] @ qsum if len(cand) else np.zeros(0)
+        if not len(cand):
+            sim = np.zeros(0)
+        elif metric == "eq3":
+            sim = lev.rep[cand] @ qsum
+        else:
+            sim = np.maximum(lev.r_max[cand] * qsum, lev.r_min[cand] * qsum).sum(axis=1)
         k = selected_count(lev.rep.shape[0], level_keep_ppm[lvl], len(cand))
         if trace is not None:
             trace.append((np.asarray(cand), np.asarray(sim), k))

@@ -285,11 +285,12 @@ def test_p6_bound_and_linearisation():
 
 # ---------------------------------------------------------------- P7 -------
 
-def _brute_select(qsum, keys, s, fanouts, level_keep):
+def _brute_select(qsum, keys, s, fanouts, level_keep, metric="eq3"):
     """Coarse-to-fine selection by exhaustive search: at every level, try every
     subset of the candidates of the required size and keep the one with the
     largest total similarity (ties: the lexicographically smallest id list).
-    Summaries are recomputed from the member tokens with explicit loops."""
+    Summaries are recomputed from the member tokens with explicit loops; the
+    similarity is Eq. 3 (alpha 0.6) or the Eq. 2 bound, channel by channel."""
     N, d = keys.shape
     n_full = N // s
     sizes = [s]
@@ -306,7 +307,10 @@ def _brute_select(qsum, keys, s, fanouts, level_keep):
         for i in range(d):
             mx = max(keys[t][i] for t in toks)
             mn = min(keys[t][i] for t in toks)
-            total += qsum[i] * (0.6 * mx + 0.4 * mn)
+            if metric == "eq3":
+                total += qsum[i] * (0.6 * mx + 0.4 * mn)
+            else:
+                total += max(qsum[i] * mx, qsum[i] * mn)
         return total
 
     n_level = [n_full]
@@ -328,8 +332,9 @@ def _brute_select(qsum, keys, s, fanouts, level_keep):
     return chosen
 
 
+@pytest.mark.parametrize("metric", ["eq3", "bound"])
 @pytest.mark.parametrize("seed", range(6))
-def test_p7_brute_force_tiny(seed):
+def test_p7_brute_force_tiny(seed, metric):
     rng = np.random.default_rng(100 + seed)
     s = int(rng.choice([2, 4]))
     fan = [(), (2,), (3,), (2, 2)][seed % 4]
@@ -339,9 +344,30 @@ def test_p7_brute_force_tiny(seed):
     qg = rng.standard_normal((G, d))
     keep = O.level_keep_fractions(int(rng.choice([250_000, 400_000])), 1 + len(fan))
     levels = O.cluster_pyramid(keys, s, fan, 0.6)
-    got = O.hierarchical_select(qg, levels, fan, keep)
-    want = _brute_select(qg.sum(0), keys, s, fan, keep)
+    got = O.hierarchical_select(qg, levels, fan, keep, metric=metric)
+    want = _brute_select(qg.sum(0), keys, s, fan, keep, metric)
     assert list(got) == sorted(want)
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_bound_equals_eq3_at_alpha_one_for_nonnegative_queries(seed):
+    # Eq. 2's max(q r_max, q r_min) is q r_max when q >= 0, which is Eq. 3 at
+    # alpha = 1: the two metrics must select the same clusters
+    rng = np.random.default_rng(300 + seed)
+    keys = rng.standard_normal((400, 16))
+    qg = np.abs(rng.standard_normal((2, 16)))
+    fan = (4, 2)
+    keep = O.level_keep_fractions(150_000, 3)
+    levels = O.cluster_pyramid(keys, 4, fan, 1.0)
+    a = O.hierarchical_select(qg, levels, fan, keep, metric="bound")
+    b = O.hierarchical_select(qg, levels, fan, keep, metric="eq3")
+    assert np.array_equal(a, b)
+    # and with mixed-sign queries the two generally differ (the test is live)
+    qm = rng.standard_normal((2, 16))
+    diff = sum(not np.array_equal(O.hierarchical_select(qm * (j + 1) + j, levels, fan, keep, metric="bound"),
+                                  O.hierarchical_select(qm * (j + 1) + j, levels, fan, keep, metric="eq3"))
+               for j in range(4))
+    assert diff >= 1
 
 
 # ---------------------------------------------------------------- P8 -------
