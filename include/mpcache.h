@@ -70,7 +70,7 @@ extern "C" {
 
 #define MPC_API __attribute__((visibility("default")))
 
-#define MPC_ABI_VERSION 1
+#define MPC_ABI_VERSION 2
 #define MPC_MAX_LEVELS 4
 #define MPC_MAX_REFS 128
 
@@ -83,6 +83,9 @@ enum mpc_status {
 };
 
 enum mpc_dtype { MPC_F32 = 0, MPC_BF16 = 1 };
+
+/* Cluster similarity of mpc_select. */
+enum mpc_sim_metric { MPC_SIM_EQ3 = 0, MPC_SIM_BOUND = 1 };
 
 typedef struct {
   int32_t layer;   /* index along per-layer tensors */
@@ -177,8 +180,10 @@ typedef struct {
 /* ---- mpc_select ----------------------------------------------------------
  * Dynamic selection of one decode step for leader layers (Sec. 3.3-3.4; Alg.
  * 2 Step 2, Sim + topk).  With C_1 = floor(n_tok_b / s) sealed clusters and
- * C_{l+1} = ceil(C_l / fanout[l]), for every ref, sequence b and kv head h:
- *   sim(c) = (sum over the group's query heads of q) . rep_c      (Eq. 3)
+ * C_{l+1} = ceil(C_l / fanout[l]), for every ref, sequence b and kv head h,
+ * with q = the sum of the group's query heads:
+ *   metric MPC_SIM_EQ3:   sim(c) = q . rep_c                          (Eq. 3)
+ *   metric MPC_SIM_BOUND: sim(c) = sum_i max(q_i r_max_ci, q_i r_min_ci) (Eq. 2)
  *   the coarsest level ranks all of its clusters; every finer level ranks
  *   the children of the clusters its parent level kept; level l keeps
  *   k_l = count(C_l, level_keep_ppm[l]) (at most its candidates); equal
@@ -202,6 +207,9 @@ typedef struct {
   int32_t sel_cap;             /* >= every k_1 */
   int32_t* out_sel;            /* device */
   int32_t* out_n_sel;          /* device [batch] */
+  int32_t metric;              /* MPC_SIM_EQ3 (0) or MPC_SIM_BOUND (1) */
+  const float* r_max;          /* device, laid out like rep; read for MPC_SIM_BOUND only */
+  const float* r_min;          /* device, laid out like rep; read for MPC_SIM_BOUND only */
 } mpc_select_args;
 
 /* ---- mpc_sparse_decode_attn ----------------------------------------------

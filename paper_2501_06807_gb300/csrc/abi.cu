@@ -223,6 +223,10 @@ int validate_select(const mpc_select_args* a, SelectParams* p) {
   MPC_TRY(make_pyramid(a->cap_tokens, a->cluster_size, a->n_levels, a->fanout, a->summary_rows, &p->pyr, true));
   for (int l = 0; l < a->n_levels; ++l) MPC_TRY(check_ppm(a->level_keep_ppm[l], "level_keep_ppm"));
   if (!aligned16(a->rep)) return fail(MPC_ERR_INVALID_ARG, "rep must be 16-byte aligned");
+  if (a->metric != MPC_SIM_EQ3 && a->metric != MPC_SIM_BOUND)
+    return fail(MPC_ERR_INVALID_ARG, "metric %d is not MPC_SIM_EQ3 or MPC_SIM_BOUND", a->metric);
+  if (a->metric == MPC_SIM_BOUND && (!aligned16(a->r_max) || !aligned16(a->r_min)))
+    return fail(MPC_ERR_INVALID_ARG, "r_max / r_min must be 16-byte aligned");
   // bound on the candidates of any level
   int kmax[kMaxLevels] = {0};
   long long mc = 0;
@@ -267,8 +271,12 @@ int validate_select(const mpc_select_args* a, SelectParams* p) {
     if (r > p->pyr.cap[l]) r = p->pyr.cap[l];
     if (r > need) need = r;
   }
-  const long long budget =
-      (kSmemOptin - 256 - (long long)select_smem_bytes(a->head_dim, P, 0)) / ((long long)a->head_dim * 4 + 4);
+  const int n_src = a->metric == MPC_SIM_BOUND ? 2 : 1;  // summary rows per candidate
+  p->metric = a->metric;
+  p->rmax = a->r_max;
+  p->rmin = a->r_min;
+  const long long budget = (kSmemOptin - 256 - (long long)select_smem_bytes(a->head_dim, P, 0, n_src)) /
+                           ((long long)a->head_dim * 4 * n_src + 4);
   if (budget < 1) return fail(MPC_ERR_BAD_SHAPE, "%d candidates leave no shared memory to stage representatives", P);
   p->row_buf = (int)(need < budget ? need : budget);
   return MPC_OK;
@@ -484,6 +492,8 @@ MPC_API int mpc_select(const mpc_select_args* args, void* workspace, size_t work
   MPC_TRY(validate_select(args, &p));
   if (!args->q || !args->rep || !args->n_tok || !args->out_sel || !args->out_n_sel)
     return fail(MPC_ERR_INVALID_ARG, "a required pointer is NULL");
+  if (args->metric == MPC_SIM_BOUND && (!args->r_max || !args->r_min))
+    return fail(MPC_ERR_INVALID_ARG, "MPC_SIM_BOUND needs r_max and r_min");
   const int units = args->n_refs * args->batch * args->n_kv_heads;
   const cudaError_t e = launch_select(p, args->dtype, args->head_dim, units, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "mpc_select launch");

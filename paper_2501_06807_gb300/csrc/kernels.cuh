@@ -51,8 +51,11 @@ struct SelectParams {
   int* out_sel;
   int* out_n_sel;
   int max_cand;  // power of two, capacity of the shared candidate arrays
-  int row_buf;   // representative rows staged in shared memory at once
+  int row_buf;   // candidates whose summary rows are staged in shared memory at once
   int spec_first;  // the first round also scores the whole level below the coarsest
+  int metric;      // MPC_SIM_EQ3: rep; MPC_SIM_BOUND: r_max and r_min
+  const float* rmax;
+  const float* rmin;
 };
 
 struct StaticParams {
@@ -132,7 +135,7 @@ int attn_smem_bytes(int dtype, int D, int G, int B);
 int attn_persist_ctas_max();
 int attn_persist_batch_max();
 cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cudaStream_t st);
-int select_smem_bytes(int D, int max_cand, int row_buf);
+int select_smem_bytes(int D, int max_cand, int row_buf, int n_src);
 int select_spec_first(int units);
 cudaError_t launch_clusters(const ClusterParams& p, int dtype, int D, int n_units, int groups_x,
                             bool any_leader, cudaStream_t st);

@@ -39,11 +39,12 @@ __device__ __forceinline__ int key_id(unsigned long long key) {
   return (int)(0xffffffffu - (uint32_t)(key & 0xffffffffull));
 }
 
-// Shared-memory layout of one select CTA (host and device).
+// Shared-memory layout of one select CTA (host and device): n_src staged
+// row arrays (rep, or r_max and r_min), then the scalars.
 struct SelLayout {
   size_t qsum, cs, keys, mark, kept, total;
-  __host__ __device__ SelLayout(int D, int MC, int RB) {
-    qsum = (size_t)RB * D * 4;             // staged rows first (16-byte aligned)
+  __host__ __device__ SelLayout(int D, int MC, int RB, int n_src) {
+    qsum = (size_t)n_src * RB * D * 4;     // staged rows first (16-byte aligned)
     cs = qsum + (size_t)D * 4;              // scores of the first round's children
     keys = (cs + (size_t)RB * 4 + 15) & ~(size_t)15;
     mark = keys + (size_t)MC * 16;          // two key arrays
@@ -71,7 +72,8 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   constexpr int kFastMax = 16 * NW;  // candidates ranked from registers (NW / 2 keys per lane)
   extern __shared__ __align__(128) uint8_t smem[];
   const int MC = p.max_cand, RB = p.row_buf;
-  const SelLayout L(D, MC, RB);
+  const int NSRC = p.metric == MPC_SIM_BOUND ? 2 : 1;  // summary rows per candidate
+  const SelLayout L(D, MC, RB, NSRC);
   float* rows = reinterpret_cast<float*>(smem);
   float* qsum = reinterpret_cast<float*>(smem + L.qsum);
   float* cs = reinterpret_cast<float*>(smem + L.cs);
@@ -91,16 +93,21 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   const int layer = p.refs.layer[ri], group = p.refs.group[ri];
   const int G = p.G;
   const int top = p.pyr.n_levels - 1;
-  const float* rep0 = p.rep + ((int64_t)(group * p.B + b) * p.Hkv + h) * p.pyr.rows * D;
+  const int64_t unit_off = ((int64_t)(group * p.B + b) * p.Hkv + h) * p.pyr.rows * D;
+  // staged source w of a candidate: rep (Eq. 3), or r_max then r_min (Eq. 2),
+  // each into its own RB-row array of the buffer
+  const float* src0[2] = {(NSRC == 2 ? p.rmax : p.rep) + unit_off, (NSRC == 2 ? p.rmin : p.rep) + unit_off};
   int* out = p.out_sel + ((int64_t)(group * p.B + b) * p.Hkv + h) * p.sel_cap;
   uint32_t phase = 0;
   bool timed_out = false;
 
-  // q_sum . (staged row r) for rows [0, nrows) of the buffer; put(r, score)
-  // runs on the first lane of each row.  Channel order is fixed: x, y, z, w
-  // per lane, then a butterfly over the row's lanes.
+  // similarity of staged row r for rows [0, nrows) of the buffer;
+  // put(r, score) runs on the first lane of each row.  Channel order is
+  // fixed: x, y, z, w per lane, then a butterfly over the row's lanes.
+  //   Eq. 3: q_sum . rep;  Eq. 2: sum_i max(q_i r_max_i, q_i r_min_i)
   auto score_rows = [&](int nrows, auto&& put) {
     const float4 qv = reinterpret_cast<const float4*>(qsum)[c4];
+    const float* rows2 = rows + (size_t)RB * D;
     for (int r0 = warp * U * RPW; r0 < nrows; r0 += NW * U * RPW) {
       float acc[U];
 #pragma unroll
@@ -109,10 +116,19 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
         const float4 v = r < nrows ? reinterpret_cast<const float4*>(rows + (size_t)r * D)[c4]
                                    : make_float4(0.f, 0.f, 0.f, 0.f);
         float a = 0.f;
-        a = fmaf(v.x, qv.x, a);
-        a = fmaf(v.y, qv.y, a);
-        a = fmaf(v.z, qv.z, a);
-        a = fmaf(v.w, qv.w, a);
+        if (NSRC == 1) {
+          a = fmaf(v.x, qv.x, a);
+          a = fmaf(v.y, qv.y, a);
+          a = fmaf(v.z, qv.z, a);
+          a = fmaf(v.w, qv.w, a);
+        } else {
+          const float4 m = r < nrows ? reinterpret_cast<const float4*>(rows2 + (size_t)r * D)[c4]
+                                     : make_float4(0.f, 0.f, 0.f, 0.f);
+          a += fmaxf(qv.x * v.x, qv.x * m.x);
+          a += fmaxf(qv.y * v.y, qv.y * m.y);
+          a += fmaxf(qv.z * v.z, qv.z * m.z);
+          a += fmaxf(qv.w * v.w, qv.w * m.w);
+        }
         acc[u] = a;
       }
 #pragma unroll
@@ -148,18 +164,20 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   const int capC = top > 0 ? p.pyr.cap[top - 1] : 0;
   const bool spec0 = p.spec_first && top > 0 && capT + capC <= RB;
   const int nT0 = capT < RB ? capT : RB;
-  const float* repT = rep0 + (int64_t)p.pyr.off[top] * D;
-  const float* repC = rep0 + (int64_t)(top > 0 ? p.pyr.off[top - 1] : 0) * D;
+  const int64_t offT = (int64_t)p.pyr.off[top] * D;
+  const int64_t offC = (int64_t)(top > 0 ? p.pyr.off[top - 1] : 0) * D;
   const int ntok = p.n_tok[b];
   int C[kMaxLevels];
   level_counts(p.pyr, ntok, C);
   if (warp == 0) {
     const int nT = max(0, min(C[top], nT0));
     const int nCc = spec0 ? max(0, min(C[top - 1], capC)) : 0;
-    if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)(nT + nCc) * ROWB);
+    if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)(nT + nCc) * ROWB * NSRC);
     __syncwarp();
-    warp_copy(rows, repT, (uint32_t)nT * ROWB, &s_bar, lane);
-    if (nCc > 0) warp_copy(rows + (size_t)capT * D, repC, (uint32_t)nCc * ROWB, &s_bar, lane);
+    for (int w = 0; w < NSRC; ++w) {
+      warp_copy(rows + (size_t)w * RB * D, src0[w] + offT, (uint32_t)nT * ROWB, &s_bar, lane);
+      if (nCc > 0) warp_copy(rows + ((size_t)w * RB + capT) * D, src0[w] + offC, (uint32_t)nCc * ROWB, &s_bar, lane);
+    }
   }
 
   // q_sum = sum over the group's query heads (fixed order)
@@ -190,9 +208,10 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
     for (int x0 = nT0; x0 < n; x0 += RB) {
       const int nb = min(RB, n - x0);
       if (warp == 0) {
-        if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)nb * ROWB);
+        if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)nb * ROWB * NSRC);
         __syncwarp();
-        warp_copy(rows, repT + (int64_t)x0 * D, (uint32_t)nb * ROWB, &s_bar, lane);
+        for (int w = 0; w < NSRC; ++w)
+          warp_copy(rows + (size_t)w * RB * D, src0[w] + offT + (int64_t)x0 * D, (uint32_t)nb * ROWB, &s_bar, lane);
       }
       wait_rows();
       score_rows(nb, [&](int r, float sc) { keysA[x0 + r] = sel_key(sc, x0 + r); });
@@ -211,16 +230,17 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
       // candidates are the children of the kept clusters of level l + 1, so
       // every run of fl consecutive candidates is one run of rows
       const int fl = p.pyr.fanout[l];
-      const float* repL = rep0 + (int64_t)p.pyr.off[l] * D;
+      const int64_t offL = (int64_t)p.pyr.off[l] * D;
       for (int x0 = 0; x0 < n; x0 += RB) {
         const int x1 = min(n, x0 + RB);
         if (warp == 0) {
-          if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)(x1 - x0) * ROWB);
+          if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)(x1 - x0) * ROWB * NSRC);
           __syncwarp();
           for (int kk = x0 / fl + lane; kk * fl < x1; kk += 32) {
             const int s0 = max(x0, kk * fl), s1 = min(x1, kk * fl + fl);
-            bulk_g2s(rows + (size_t)(s0 - x0) * D, repL + (int64_t)key_id(keysA[s0]) * D, (uint32_t)(s1 - s0) * ROWB,
-                     &s_bar);
+            for (int w = 0; w < NSRC; ++w)
+              bulk_g2s(rows + ((size_t)w * RB + (s0 - x0)) * D, src0[w] + offL + (int64_t)key_id(keysA[s0]) * D,
+                       (uint32_t)(s1 - s0) * ROWB, &s_bar);
           }
         }
         wait_rows();
@@ -424,7 +444,9 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
 // they fit two CTAs per SM, else 4 (up to five CTAs per SM).
 static int select_threads(int units) { return units <= 152 ? 512 : (units <= 304 ? 256 : 128); }
 
-int select_smem_bytes(int D, int max_cand, int row_buf) { return (int)SelLayout(D, max_cand, row_buf).total; }
+int select_smem_bytes(int D, int max_cand, int row_buf, int n_src) {
+  return (int)SelLayout(D, max_cand, row_buf, n_src).total;
+}
 
 // Scoring the whole level below the coarsest in the first round saves a
 // dependent round but reads the children of unkept clusters too: worth it
@@ -439,7 +461,7 @@ static cudaError_t launch_sel(K kernel, int units, int nt, int smem, cudaStream_
 }
 
 cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cudaStream_t st) {
-  const int smem = select_smem_bytes(D, p.max_cand, p.row_buf);
+  const int smem = select_smem_bytes(D, p.max_cand, p.row_buf, p.metric == MPC_SIM_BOUND ? 2 : 1);
   const int nt = select_threads(units);
 #define MPC_SEL(TT, DD)                                                                     \
   if (D == DD) {                                                                            \

@@ -25,7 +25,9 @@ from . import build as _build
 
 MPC_OK, MPC_ERR_INVALID_ARG, MPC_ERR_BAD_SHAPE, MPC_ERR_WORKSPACE, MPC_ERR_CUDA = 0, -1, -2, -3, -4
 MPC_F32, MPC_BF16 = 0, 1
+MPC_SIM_EQ3, MPC_SIM_BOUND = 0, 1
 MAX_LEVELS = 4
+ABI_VERSION = 2
 MAX_REFS = 128
 PPM = 1_000_000
 
@@ -70,7 +72,8 @@ class SelectArgs(C.Structure):
                 ("cap_tokens", C.c_int32), ("n_tok", C.c_void_p), ("cluster_size", C.c_int32),
                 ("n_levels", C.c_int32), ("fanout", C.c_int32 * MAX_LEVELS),
                 ("level_keep_ppm", C.c_int32 * MAX_LEVELS), ("sel_cap", C.c_int32),
-                ("out_sel", C.c_void_p), ("out_n_sel", C.c_void_p)]
+                ("out_sel", C.c_void_p), ("out_n_sel", C.c_void_p), ("metric", C.c_int32),
+                ("r_max", C.c_void_p), ("r_min", C.c_void_p)]
 
 
 class AttnArgs(C.Structure):
@@ -124,6 +127,8 @@ def load(path: Optional[str] = None) -> C.CDLL:
     lib.mpc_abi_version.restype = C.c_int
     lib.mpc_sparse_decode_attn_static_scratch.restype = C.c_int
     lib.mpc_sparse_decode_attn_static_scratch.argtypes = [C.c_void_p, C.c_void_p]
+    if lib.mpc_abi_version() != ABI_VERSION:
+        raise MPCError(f"libmpcache ABI {lib.mpc_abi_version()} does not match the binding's {ABI_VERSION}")
     if path is None:
         _LIB = lib
     return lib
@@ -336,8 +341,9 @@ class Engine:
         self.build_clusters(k, v, page_table, page_size)
 
     # ---------------------------------------------------------- decode ----
-    def select(self, q: torch.Tensor):
-        """q: [L][B][Hq][d] queries of this step (only the leaders' are read)."""
+    def select(self, q: torch.Tensor, metric: int = MPC_SIM_EQ3):
+        """q: [L][B][Hq][d] queries of this step (only the leaders' are read);
+        metric MPC_SIM_EQ3 (Eq. 3 with rep) or MPC_SIM_BOUND (Eq. 2 bound)."""
         lib = load()
         refs = _refs(self.refs_lead)
         a = SelectArgs()
@@ -350,6 +356,7 @@ class Engine:
         a.cluster_size, a.n_levels, a.fanout = self.s, self.n_levels, _fan(self.fanouts)
         a.level_keep_ppm = _fan(self.level_keep_ppm)
         a.sel_cap, a.out_sel, a.out_n_sel = self.sel_cap, _ptr(self.sel), _ptr(self.n_sel)
+        a.metric, a.r_max, a.r_min = metric, _ptr(self.rmax), _ptr(self.rmin)
         _check(lib.mpc_select(C.byref(a), None, 0, C.c_void_p(_stream())))
 
     def attn_args(self, q, k_new, v_new, advance=True, refs_list=None, out=None) -> AttnArgs:

@@ -33,7 +33,7 @@ def test_exports_every_declared_symbol(lib):
                          capture_output=True, text=True).stdout
     exported = set(re.findall(r"\b(mpc_\w+)\b", out))
     assert set(names) <= exported
-    assert lib.mpc_abi_version() == 1
+    assert lib.mpc_abi_version() == mpcache.ABI_VERSION == 2
 
 
 def test_struct_layout_matches_c(tmp_path):
@@ -125,6 +125,15 @@ def test_select_and_static_validation(lib):
     assert _ws(lib, "mpc_select_workspace_size", s)[0] == mpcache.MPC_ERR_INVALID_ARG  # not a leader
     refs[0].leader = 1
     assert _ws(lib, "mpc_select_workspace_size", s) == (0, 0)
+    s.metric = 7                       # not a metric
+    assert _ws(lib, "mpc_select_workspace_size", s)[0] == mpcache.MPC_ERR_INVALID_ARG
+    s.metric, s.r_max, s.r_min = mpcache.MPC_SIM_BOUND, 4100, 8192  # r_max misaligned
+    assert _ws(lib, "mpc_select_workspace_size", s)[0] == mpcache.MPC_ERR_INVALID_ARG
+    s.r_max = 4096
+    assert _ws(lib, "mpc_select_workspace_size", s) == (0, 0)
+    s.q, s.n_tok, s.out_sel, s.out_n_sel, s.r_min = 8192, 8192, 8192, 8192, None
+    assert lib.mpc_select(C.byref(s), None, 0, None) == mpcache.MPC_ERR_INVALID_ARG  # bound needs r_min
+    s.metric, s.r_max, s.r_min, s.q, s.n_tok, s.out_sel, s.out_n_sel = mpcache.MPC_SIM_EQ3, None, None, None, None, None, None
     s.sel_cap = 3
     assert _ws(lib, "mpc_select_workspace_size", s)[0] == mpcache.MPC_ERR_BAD_SHAPE
     s.sel_cap = 4

@@ -17,7 +17,7 @@ import pytest
 import torch
 
 from oracle import mpcache_oracle as O
-from paper_2501_06807_gb300 import synth
+from paper_2501_06807_gb300 import mpcache, synth
 from tests import helpers as H
 
 pytestmark = pytest.mark.gpu
@@ -194,8 +194,9 @@ SELECT_CASES = [
 ]
 
 
+@pytest.mark.parametrize("metric", ["eq3", "bound"])
 @pytest.mark.parametrize("dtype,d,Hq,Hkv,s,fan,keep,N,B", SELECT_CASES)
-def test_selection(dtype, d, Hq, Hkv, s, fan, keep, N, B):
+def test_selection(dtype, d, Hq, Hkv, s, fan, keep, N, B, metric):
     g = torch.Generator().manual_seed(N + d)
     L = 1
     G = Hq // Hkv
@@ -212,7 +213,7 @@ def test_selection(dtype, d, Hq, Hkv, s, fan, keep, N, B):
     ties = 0
     for rep_i in range(3):
         q = (torch.randn((L, B, Hq, d), generator=g) * 2).to(dtype)
-        eng.select(q.cuda())
+        eng.select(q.cuda(), mpcache.MPC_SIM_BOUND if metric == "bound" else mpcache.MPC_SIM_EQ3)
         sel = eng.sel.cpu().numpy()
         n_sel = eng.n_sel.cpu().numpy()
         for b in range(B):
@@ -220,7 +221,7 @@ def test_selection(dtype, d, Hq, Hkv, s, fan, keep, N, B):
                 levels = O.cluster_pyramid(K[0, b, h].double().numpy(), s, fan, 0.6)
                 qg = q[0, b, h * G:(h + 1) * G].double().numpy()
                 tr = []
-                ref = O.hierarchical_select(qg, levels, fan, keep, trace=tr)
+                ref = O.hierarchical_select(qg, levels, fan, keep, trace=tr, metric=metric)
                 got = sel[0, b, h, :n_sel[b]]
                 assert n_sel[b] == len(ref)
                 assert (sel[0, b, h, n_sel[b]:] == -1).all()
