@@ -283,7 +283,7 @@ __device__ __forceinline__ void finish_grid(const AttnParams& p) {
 
 // ------------------------------------------------ bf16 path (persistent) ----
 //
-// One CTA per SM, four warps.  The tiles of all units (every selected
+// One CTA per SM, four to eight warps.  The tiles of all units (every selected
 // cluster row tile, tail and appended row of every (layer, sequence, kv
 // head)) form one list, cut into contiguous, equal ranges, one per warp slot
 // (slots interleaved over the CTAs, at most one slot per tile).  Every warp
@@ -328,19 +328,28 @@ struct PSmem {
   static constexpr int TILEB = 16 * ROWB;
   static __host__ __device__ constexpr int qbytes(int G) { return ((G * D * 2 + 127) / 128) * 128; }
   static __host__ __device__ constexpr int stage(int G) { return 2 * TILEB + qbytes(G); }
-  static __host__ __device__ constexpr int key_off(int G, int nst) { return kWarps * nst * stage(G); }
-  static __host__ __device__ constexpr int sel_off(int G, int nst) { return key_off(G, nst) + kWarps * nst * 16; }
-  static __host__ __device__ constexpr int tab_off(int G, int nst) { return sel_off(G, nst) + kWarps * kSelSmem * 4; }
-  static __host__ __device__ constexpr int total(int G, int nst, int B) { return tab_off(G, nst) + (4 * B + 2) * 4; }
+  // wpc warps per CTA, each with an nst-stage ring
+  static __host__ __device__ constexpr int key_off(int G, int nst, int wpc) { return wpc * nst * stage(G); }
+  static __host__ __device__ constexpr int sel_off(int G, int nst, int wpc) { return key_off(G, nst, wpc) + wpc * nst * 16; }
+  static __host__ __device__ constexpr int tab_off(int G, int nst, int wpc) { return sel_off(G, nst, wpc) + wpc * kSelSmem * 4; }
+  static __host__ __device__ constexpr int total(int G, int nst, int wpc, int B) { return tab_off(G, nst, wpc) + (4 * B + 2) * 4; }
 };
 
-// Ring depth per warp (compile-time for cp.async.wait_group): d 64 takes 8
-// stages; d 128 takes 6 when they fit shared memory with the batch's tables
-// (up to 8 heads per group), else 5 (up to 8 heads) or 4 (up to 16).
-inline int persist_stages(int D, int G, int B) {
-  if (D == 64) return 8;
-  if (G <= 8 && PSmem<128>::total(G, 6, B) <= kSmemOptin) return 6;
-  return G <= 8 ? 5 : 4;
+// Warps per CTA and ring depth per warp (compile-time for
+// cp.async.wait_group).  More warps hide the per-tile compute better than
+// deeper rings at the same bytes in flight (measured: 2 x 12 and 4 x 6 are
+// slower than 6 x 4; 8 x 3 is best with one query head per group, whose
+// tiles carry the same mma work for a quarter of the heads).  d 64: 4 x 8.
+// d 128, up to 8 heads per group: 8 x 3 (one head) or 6 x 4 when that fits
+// shared memory with the batch's tables, else 4 x 5; up to 16 heads: 4 x 4.
+struct PersistCfg {
+  int wpc, nst;
+};
+inline PersistCfg persist_cfg(int D, int G, int B) {
+  if (D == 64) return {4, 8};
+  if (G == 1 && PSmem<128>::total(G, 3, 8, B) <= kSmemOptin) return {8, 3};
+  if (G <= 8 && PSmem<128>::total(G, 4, 6, B) <= kSmemOptin) return {6, 4};
+  return {4, G <= 8 ? 5 : 4};
 }
 
 struct Cursor {
@@ -354,8 +363,8 @@ __device__ __forceinline__ uint32_t movmatrix_t(uint32_t a) {
   return d;
 }
 
-template <int D, int HN, int NST>
-__global__ void __launch_bounds__(128, 1) attn_bf16_persist_kernel(const __grid_constant__ AttnParams p) {
+template <int D, int HN, int NST, int WPC>
+__global__ void __launch_bounds__(WPC * 32, 1) attn_bf16_persist_kernel(const __grid_constant__ AttnParams p) {
   using S = PSmem<D>;
   constexpr int ROWB = S::ROWB;
   constexpr int TILEB = S::TILEB;
@@ -366,9 +375,9 @@ __global__ void __launch_bounds__(128, 1) attn_bf16_persist_kernel(const __grid_
   const int STAGE = S::stage(G);
   constexpr int CH = ROWB / 16;  // 16-byte chunks per row
   uint8_t* ring = smem + warp * NST * STAGE;
-  int8_t* keys = reinterpret_cast<int8_t*>(smem + S::key_off(G, NST)) + warp * NST * 16;
-  int* sel_s = reinterpret_cast<int*>(smem + S::sel_off(G, NST)) + warp * kSelSmem;
-  int* s_nt = reinterpret_cast<int*>(smem + S::tab_off(G, NST));  // tiles per unit of sequence b
+  int8_t* keys = reinterpret_cast<int8_t*>(smem + S::key_off(G, NST, WPC)) + warp * NST * 16;
+  int* sel_s = reinterpret_cast<int*>(smem + S::sel_off(G, NST, WPC)) + warp * kSelSmem;
+  int* s_nt = reinterpret_cast<int*>(smem + S::tab_off(G, NST, WPC));  // tiles per unit of sequence b
   int* s_pre = s_nt + B;                                           // exclusive prefix of s_nt (B + 1)
   int* s_n = s_pre + B + 1;                                        // cache rows before the append
   int* s_k1 = s_n + B;                                             // selected clusters
@@ -413,7 +422,7 @@ __global__ void __launch_bounds__(128, 1) attn_bf16_persist_kernel(const __grid_
 
   const int64_t TPR = (int64_t)Hkv * s_pre[B];
   const int64_t NT = TPR * p.n_refs;
-  const int64_t NW_all = (int64_t)gridDim.x * kWarps;
+  const int64_t NW_all = (int64_t)gridDim.x * WPC;
   const int NW = (int)(NW_all < NT ? NW_all : NT);
   const int gw = warp * gridDim.x + blockIdx.x;
   const int64_t x0 = gw < NW ? NT * gw / NW : 0, x1 = gw < NW ? NT * (gw + 1) / NW : 0;
@@ -1001,8 +1010,8 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const __grid_constant__ A
 
 int attn_smem_bytes(int dtype, int D, int G, int B) {
   if (dtype == MPC_BF16) {
-    const int nst = persist_stages(D, G, B);
-    return D == 64 ? PSmem<64>::total(G, nst, B) : PSmem<128>::total(G, nst, B);
+    const PersistCfg c = persist_cfg(D, G, B);
+    return D == 64 ? PSmem<64>::total(G, c.nst, c.wpc, B) : PSmem<128>::total(G, c.nst, c.wpc, B);
   }
   return D == 64 ? Smem<64, 4>::total(G) : Smem<128, 4>::total(G);
 }
@@ -1011,10 +1020,10 @@ int attn_persist_ctas_max() { return kMaxPersistCtas; }
 int attn_persist_batch_max() { return kMaxBatchPersist; }
 
 template <typename K>
-static cudaError_t launch_k(K kernel, dim3 grid, int smem, cudaStream_t st, const AttnParams& p) {
+static cudaError_t launch_k(K kernel, dim3 grid, int smem, cudaStream_t st, const AttnParams& p, int threads = 128) {
   cudaError_t e = ensure_dyn_smem((const void*)kernel, smem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(kernel, grid, dim3(128), smem, st, p);
+  return launch_pdl(kernel, grid, dim3(threads), smem, st, p);
 }
 
 // CTAs of the persistent grid: one per SM, at most kMaxPersistCtas.
@@ -1036,16 +1045,22 @@ static int persist_ctas() {
 cudaError_t launch_attn(const AttnParams& p0, int dtype, int D, int n_units, cudaStream_t st) {
   AttnParams p = p0;
   if (dtype == MPC_BF16) {
-    p.n_stages = persist_stages(D, p.G, p.B);
+    const PersistCfg c = persist_cfg(D, p.G, p.B);
+    p.n_stages = c.nst;
     const int smem = attn_smem_bytes(dtype, D, p.G, p.B);
     const dim3 grid(persist_ctas());
-    if (p.G <= 8) {
-      if (D == 64) return launch_k(attn_bf16_persist_kernel<64, 1, 8>, grid, smem, st, p);
-      if (p.n_stages == 6) return launch_k(attn_bf16_persist_kernel<128, 1, 6>, grid, smem, st, p);
-      return launch_k(attn_bf16_persist_kernel<128, 1, 5>, grid, smem, st, p);
-    }
-    if (D == 64) return launch_k(attn_bf16_persist_kernel<64, 2, 8>, grid, smem, st, p);
-    return launch_k(attn_bf16_persist_kernel<128, 2, 4>, grid, smem, st, p);
+    const int th = 32 * c.wpc;
+#define MPC_PERSIST(DD, HH, NN, WW)                                                                 \
+  if (D == DD && (p.G <= 8 ? 1 : 2) == HH && c.nst == NN && c.wpc == WW)                           \
+    return launch_k(attn_bf16_persist_kernel<DD, HH, NN, WW>, grid, smem, st, p, th);
+    MPC_PERSIST(64, 1, 8, 4)
+    MPC_PERSIST(128, 1, 3, 8)
+    MPC_PERSIST(128, 1, 4, 6)
+    MPC_PERSIST(128, 1, 5, 4)
+    MPC_PERSIST(64, 2, 8, 4)
+    MPC_PERSIST(128, 2, 4, 4)
+#undef MPC_PERSIST
+    return cudaErrorInvalidValue;
   }
   const dim3 grid(p.n_split, n_units);
   const int smem = attn_smem_bytes(dtype, D, p.G, p.B);
