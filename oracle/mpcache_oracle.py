@@ -151,6 +151,7 @@ class Level:
     r_max: np.ndarray           # [C][d]
     r_min: np.ndarray           # [C][d]
     rep: np.ndarray             # [C][d] alpha r_max + (1 - alpha) r_min
+    mean: np.ndarray = None     # [C][d] mean of the member keys (average baseline)
 
 
 def cluster_pyramid(keys: np.ndarray, s: int, fanouts: Sequence[int],
@@ -161,7 +162,8 @@ def cluster_pyramid(keys: np.ndarray, s: int, fanouts: Sequence[int],
     tokens [c s, (c+1) s) for c < floor(N / s) (adjacent tokens, Sec. 3.3; the
     partial remainder is the tail).  Level l+1 groups f_l consecutive level-l
     clusters.  r_max / r_min are the channel-wise max / min over all member
-    tokens (Sec. 3.3, Eq. 2) and rep the reordered representative of Eq. 3.
+    tokens (Sec. 3.3, Eq. 2), rep the reordered representative of Eq. 3 and
+    mean the average member key (the average baseline of App. G).
     """
     keys = np.asarray(keys, dtype=np.float64)
     n_full = keys.shape[0] // s
@@ -172,11 +174,13 @@ def cluster_pyramid(keys: np.ndarray, s: int, fanouts: Sequence[int],
         if members:
             r_max = np.stack([keys[m].max(axis=0) for m in members])
             r_min = np.stack([keys[m].min(axis=0) for m in members])
+            mean = np.stack([keys[m].mean(axis=0) for m in members])
         else:
             r_max = np.zeros((0, d))
             r_min = np.zeros((0, d))
+            mean = np.zeros((0, d))
         rep = alpha * r_max + (1.0 - alpha) * r_min
-        levels.append(Level(members, r_max, r_min, rep))
+        levels.append(Level(members, r_max, r_min, rep, mean))
         if lvl < len(fanouts):
             f = fanouts[lvl]
             n_up = -(-len(members) // f)
@@ -191,15 +195,16 @@ def hierarchical_select(q_group: np.ndarray, levels: List[Level],
 
     q_group: [G][d] decode queries of one kv group, scored through their sum
     q = sum_g q_g.  The similarity of cluster c is q . rep_c (Eq. 3, the
-    default) or, with metric="bound", the upper bound of Eq. 2,
-    sum_i max(q_i r_max_ci, q_i r_min_ci), evaluated on the same summed query.
+    default); with metric="bound", the upper bound of Eq. 2,
+    sum_i max(q_i r_max_ci, q_i r_min_ci), evaluated on the same summed query;
+    with metric="mean", q . mean_c (the average-key baseline of App. G).
     At the coarsest level every cluster is a candidate; at each finer level
     the candidates are the children of the kept parents.  Returns the kept
     finest-level ids in ascending order.  ``trace``, if given, receives per
     level (coarsest first) the candidate ids, their similarities and k, for
     tests that need the margin at each cut.
     """
-    if metric not in ("eq3", "bound"):
+    if metric not in ("eq3", "bound", "mean"):
         raise ValueError(metric)
     qsum = np.asarray(q_group, dtype=np.float64).sum(axis=0)
     n = len(levels)
@@ -211,6 +216,8 @@ def hierarchical_select(q_group: np.ndarray, levels: List[Level],
             sim = np.zeros(0)
         elif metric == "eq3":
             sim = lev.rep[cand] @ qsum
+        elif metric == "mean":
+            sim = lev.mean[cand] @ qsum
         else:
             sim = np.maximum(lev.r_max[cand] * qsum, lev.r_min[cand] * qsum).sum(axis=1)
         k = selected_count(lev.rep.shape[0], level_keep_ppm[lvl], len(cand))

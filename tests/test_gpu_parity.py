@@ -197,11 +197,22 @@ SELECT_CASES = [
 @pytest.mark.parametrize("metric", ["eq3", "bound"])
 @pytest.mark.parametrize("dtype,d,Hq,Hkv,s,fan,keep,N,B", SELECT_CASES)
 def test_selection(dtype, d, Hq, Hkv, s, fan, keep, N, B, metric):
+    _check_selection(dtype, d, Hq, Hkv, s, fan, keep, N, B, metric, 0.6)
+
+
+@pytest.mark.parametrize("alpha", [0.0, 0.25, 1.0])
+def test_selection_alpha_sweep(alpha):
+    # Eq. 3's weight between r_max and r_min (the paper's alpha ablation):
+    # the summaries and the selection follow it
+    _check_selection(torch.bfloat16, 128, 8, 2, 16, (8,), (100_000, 500_000), 2048 + 15, 2, "eq3", alpha)
+
+
+def _check_selection(dtype, d, Hq, Hkv, s, fan, keep, N, B, metric, alpha):
     g = torch.Generator().manual_seed(N + d)
     L = 1
     G = Hq // Hkv
     eng = H.make_engine(synth.Workload("t", L, B, Hq, Hkv, d, "f32" if dtype == torch.float32 else "bf16",
-                                       N, N, O.PPM, s, fan, keep, 1, 4, "iid"), 4)
+                                       N, N, O.PPM, s, fan, keep, 1, 4, "iid", alpha=alpha), 4)
     # keys with token-wise locality (a slow drift per channel), the structure
     # clustering relies on; iid keys make coarse summaries indistinguishable
     drift = torch.cumsum(torch.randn((L, B, Hkv, N, d), generator=g) * 0.15, dim=3)
@@ -218,7 +229,7 @@ def test_selection(dtype, d, Hq, Hkv, s, fan, keep, N, B, metric):
         n_sel = eng.n_sel.cpu().numpy()
         for b in range(B):
             for h in range(Hkv):
-                levels = O.cluster_pyramid(K[0, b, h].double().numpy(), s, fan, 0.6)
+                levels = O.cluster_pyramid(K[0, b, h].double().numpy(), s, fan, alpha)
                 qg = q[0, b, h * G:(h + 1) * G].double().numpy()
                 tr = []
                 ref = O.hierarchical_select(qg, levels, fan, keep, trace=tr, metric=metric)

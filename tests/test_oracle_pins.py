@@ -247,6 +247,9 @@ def test_p4_token_wise_equals_topk(G, k_ppm):
     scores = torch.from_numpy(keys) @ torch.from_numpy(qg).sum(0)
     want = np.sort(torch.topk(scores, k).indices.numpy())
     assert np.array_equal(sel, want)
+    # a one-token cluster's mean is its key: the average baseline agrees
+    assert np.array_equal(levels[0].mean, keys)
+    assert np.array_equal(O.hierarchical_select(qg, levels, (), (k_ppm,), metric="mean"), want)
 
 
 # ---------------------------------------------------------------- P5 / P6 --
@@ -290,7 +293,8 @@ def _brute_select(qsum, keys, s, fanouts, level_keep, metric="eq3"):
     subset of the candidates of the required size and keep the one with the
     largest total similarity (ties: the lexicographically smallest id list).
     Summaries are recomputed from the member tokens with explicit loops; the
-    similarity is Eq. 3 (alpha 0.6) or the Eq. 2 bound, channel by channel."""
+    similarity is Eq. 3 (alpha 0.6), the Eq. 2 bound or the mean key, channel by
+    channel."""
     N, d = keys.shape
     n_full = N // s
     sizes = [s]
@@ -309,8 +313,13 @@ def _brute_select(qsum, keys, s, fanouts, level_keep, metric="eq3"):
             mn = min(keys[t][i] for t in toks)
             if metric == "eq3":
                 total += qsum[i] * (0.6 * mx + 0.4 * mn)
-            else:
+            elif metric == "bound":
                 total += max(qsum[i] * mx, qsum[i] * mn)
+            else:
+                acc = 0.0
+                for t in toks:
+                    acc += keys[t][i]
+                total += qsum[i] * acc / len(toks)
         return total
 
     n_level = [n_full]
@@ -332,7 +341,7 @@ def _brute_select(qsum, keys, s, fanouts, level_keep, metric="eq3"):
     return chosen
 
 
-@pytest.mark.parametrize("metric", ["eq3", "bound"])
+@pytest.mark.parametrize("metric", ["eq3", "bound", "mean"])
 @pytest.mark.parametrize("seed", range(6))
 def test_p7_brute_force_tiny(seed, metric):
     rng = np.random.default_rng(100 + seed)
@@ -467,3 +476,21 @@ def test_p11_commonality():
     sel = [list(run.selected[(0, l, 0, 0)]) for l in range(2, 6)]
     k = len(sel[0])
     assert O.commonality([sel[0], sel[1]], k, 1) == 1.0      # layers 2, 3 share
+
+
+def test_mean_summary_composes_by_member_counts():
+    """A coarse cluster's mean key is its children's means weighted by their
+    token counts (the last cluster of a level may hold fewer children)."""
+    rng = np.random.default_rng(77)
+    keys = rng.standard_normal((16 * 23 + 5, 8))
+    fan = (3, 2)
+    levels = O.cluster_pyramid(keys, 16, fan, 0.6)
+    for l in (1, 2):
+        f = fan[l - 1]
+        child = levels[l - 1]
+        for c, m in enumerate(levels[l].members):
+            kids = range(c * f, min((c + 1) * f, len(child.members)))
+            w = np.array([len(child.members[q]) for q in kids], dtype=np.float64)
+            want = (w[:, None] * child.mean[list(kids)]).sum(0) / w.sum()
+            assert np.allclose(levels[l].mean[c], want, rtol=1e-13, atol=1e-15)
+            assert len(m) == w.sum()
