@@ -70,7 +70,7 @@ extern "C" {
 
 #define MPC_API __attribute__((visibility("default")))
 
-#define MPC_ABI_VERSION 2
+#define MPC_ABI_VERSION 3
 #define MPC_MAX_LEVELS 4
 #define MPC_MAX_REFS 128
 
@@ -85,7 +85,7 @@ enum mpc_status {
 enum mpc_dtype { MPC_F32 = 0, MPC_BF16 = 1 };
 
 /* Cluster similarity of mpc_select. */
-enum mpc_sim_metric { MPC_SIM_EQ3 = 0, MPC_SIM_BOUND = 1 };
+enum mpc_sim_metric { MPC_SIM_EQ3 = 0, MPC_SIM_BOUND = 1, MPC_SIM_MEAN = 2 };
 
 typedef struct {
   int32_t layer;   /* index along per-layer tensors */
@@ -175,6 +175,8 @@ typedef struct {
   int32_t fanout[MPC_MAX_LEVELS]; /* fanout[l] >= 2 for l < n_levels - 1 */
   float alpha;                 /* Eq. 3 weight, default 0.6 */
   int32_t* out_n_tok;          /* device [batch] */
+  float* mean;                 /* optional device pyramid like rep: the mean member key of
+                                  every cluster (the average-key baseline); NULL skips it */
 } mpc_cluster_args;
 
 /* ---- mpc_select ----------------------------------------------------------
@@ -184,6 +186,7 @@ typedef struct {
  * with q = the sum of the group's query heads:
  *   metric MPC_SIM_EQ3:   sim(c) = q . rep_c                          (Eq. 3)
  *   metric MPC_SIM_BOUND: sim(c) = sum_i max(q_i r_max_ci, q_i r_min_ci) (Eq. 2)
+ *   metric MPC_SIM_MEAN:  sim(c) = q . mean_c, the mean member key (App. G baseline)
  *   the coarsest level ranks all of its clusters; every finer level ranks
  *   the children of the clusters its parent level kept; level l keeps
  *   k_l = count(C_l, level_keep_ppm[l]) (at most its candidates); equal
@@ -207,9 +210,10 @@ typedef struct {
   int32_t sel_cap;             /* >= every k_1 */
   int32_t* out_sel;            /* device */
   int32_t* out_n_sel;          /* device [batch] */
-  int32_t metric;              /* MPC_SIM_EQ3 (0) or MPC_SIM_BOUND (1) */
+  int32_t metric;              /* MPC_SIM_EQ3 (0), MPC_SIM_BOUND (1) or MPC_SIM_MEAN (2) */
   const float* r_max;          /* device, laid out like rep; read for MPC_SIM_BOUND only */
   const float* r_min;          /* device, laid out like rep; read for MPC_SIM_BOUND only */
+  const float* mean;           /* device, laid out like rep; read for MPC_SIM_MEAN only */
 } mpc_select_args;
 
 /* ---- mpc_sparse_decode_attn ----------------------------------------------
@@ -252,6 +256,8 @@ typedef struct {
   float scale;                 /* 0 selects 1/sqrt(d) */
   float* out;                  /* device [layer][batch][n_q_heads][d] */
   int64_t out_layer_stride;    /* elements */
+  float* mean;                 /* optional mean pyramid (in/out) kept current when a tail is
+                                  sealed; NULL skips it */
 } mpc_attn_args;
 
 /* Workspace byte counts (0 is a valid answer).  Same validation as the

@@ -207,6 +207,7 @@ int validate_clusters(const mpc_cluster_args* a, ClusterParams* p) {
   p->rmax = a->r_max;
   p->rmin = a->r_min;
   p->rep = a->rep;
+  p->mean = a->mean;
   p->alpha = a->alpha;
   p->out_n_tok = a->out_n_tok;
   return MPC_OK;
@@ -223,10 +224,11 @@ int validate_select(const mpc_select_args* a, SelectParams* p) {
   MPC_TRY(make_pyramid(a->cap_tokens, a->cluster_size, a->n_levels, a->fanout, a->summary_rows, &p->pyr, true));
   for (int l = 0; l < a->n_levels; ++l) MPC_TRY(check_ppm(a->level_keep_ppm[l], "level_keep_ppm"));
   if (!aligned16(a->rep)) return fail(MPC_ERR_INVALID_ARG, "rep must be 16-byte aligned");
-  if (a->metric != MPC_SIM_EQ3 && a->metric != MPC_SIM_BOUND)
-    return fail(MPC_ERR_INVALID_ARG, "metric %d is not MPC_SIM_EQ3 or MPC_SIM_BOUND", a->metric);
+  if (a->metric != MPC_SIM_EQ3 && a->metric != MPC_SIM_BOUND && a->metric != MPC_SIM_MEAN)
+    return fail(MPC_ERR_INVALID_ARG, "metric %d is not MPC_SIM_EQ3, MPC_SIM_BOUND or MPC_SIM_MEAN", a->metric);
   if (a->metric == MPC_SIM_BOUND && (!aligned16(a->r_max) || !aligned16(a->r_min)))
     return fail(MPC_ERR_INVALID_ARG, "r_max / r_min must be 16-byte aligned");
+  if (a->metric == MPC_SIM_MEAN && !aligned16(a->mean)) return fail(MPC_ERR_INVALID_ARG, "mean must be 16-byte aligned");
   // bound on the candidates of any level
   int kmax[kMaxLevels] = {0};
   long long mc = 0;
@@ -252,6 +254,7 @@ int validate_select(const mpc_select_args* a, SelectParams* p) {
   p->q = a->q;
   p->q_ls = a->q_layer_stride;
   p->rep = a->rep;
+  p->mean = a->mean;
   p->n_tok = a->n_tok;
   for (int l = 0; l < a->n_levels; ++l) p->keep_ppm[l] = a->level_keep_ppm[l];
   p->sel_cap = a->sel_cap;
@@ -370,6 +373,7 @@ int validate_attn(const mpc_attn_args* a, AttnParams* p, AttnPlan* plan) {
     p->rmax = a->r_max;
     p->rmin = a->r_min;
     p->rep = a->rep;
+    p->mean = a->mean;
   }
   p->alpha = a->alpha;
   p->n_tok = a->n_tok;
@@ -494,6 +498,7 @@ MPC_API int mpc_select(const mpc_select_args* args, void* workspace, size_t work
     return fail(MPC_ERR_INVALID_ARG, "a required pointer is NULL");
   if (args->metric == MPC_SIM_BOUND && (!args->r_max || !args->r_min))
     return fail(MPC_ERR_INVALID_ARG, "MPC_SIM_BOUND needs r_max and r_min");
+  if (args->metric == MPC_SIM_MEAN && !args->mean) return fail(MPC_ERR_INVALID_ARG, "MPC_SIM_MEAN needs mean");
   const int units = args->n_refs * args->batch * args->n_kv_heads;
   const cudaError_t e = launch_select(p, args->dtype, args->head_dim, units, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "mpc_select launch");

@@ -6,8 +6,10 @@
 // last, partial one is the tail).  Lanes own 16-byte chunks of a row, so a
 // warp moves whole rows with coalesced 16-byte loads and stores, writing each
 // chunk to its swizzled slot, and leaders fold the chunk into a running
-// channel max / min.  coarse_kernel: one CTA per (ref, b, h) builds the
-// coarser levels from the level below (element-wise max / min of children).
+// channel max / min (and sum, for the optional mean key).  coarse_kernel: one
+// CTA per (ref, b, h) builds the coarser levels from the level below
+// (element-wise max / min of children; means weighted by their finest
+// clusters).
 #include "kernels.cuh"
 
 namespace mpc {
@@ -49,11 +51,12 @@ __global__ void __launch_bounds__(128) gather_kernel(const __grid_constant__ Clu
   T* kc = (T*)p.kc + layer * p.cache_ls + (int64_t)(b * p.Hkv + h) * p.cap_tokens * D;
   T* vc = (T*)p.vc + layer * p.cache_ls + (int64_t)(b * p.Hkv + h) * p.cap_tokens * D;
   const int ch = lane % CH, ro = lane / CH;
-  float mx[E], mn[E];
+  float mx[E], mn[E], sm[E];
 #pragma unroll
   for (int e = 0; e < E; ++e) {
     mx[e] = kNegInf;
     mn[e] = kPosInf;
+    sm[e] = 0.f;
   }
   for (int r = r0 + ro; r < r1; r += RPW) {
     const int t = kept[r];
@@ -73,6 +76,7 @@ __global__ void __launch_bounds__(128) gather_kernel(const __grid_constant__ Clu
         const float x = to_float<T>(el[e]);
         mx[e] = fmaxf(mx[e], x);
         mn[e] = fminf(mn[e], x);
+        sm[e] += x;
       }
     }
   }
@@ -83,6 +87,7 @@ __global__ void __launch_bounds__(128) gather_kernel(const __grid_constant__ Clu
     for (int e = 0; e < E; ++e) {
       mx[e] = fmaxf(mx[e], __shfl_xor_sync(0xffffffffu, mx[e], o));
       mn[e] = fminf(mn[e], __shfl_xor_sync(0xffffffffu, mn[e], o));
+      sm[e] += __shfl_xor_sync(0xffffffffu, sm[e], o);
     }
   if (ro != 0) return;
   if (c >= p.pyr.cap[0]) {
@@ -97,6 +102,7 @@ __global__ void __launch_bounds__(128) gather_kernel(const __grid_constant__ Clu
     p.rmax[row + cc] = mx[e];
     p.rmin[row + cc] = mn[e];
     p.rep[row + cc] = fmaf(a, mx[e], am * mn[e]);
+    if (p.mean != nullptr) p.mean[row + cc] = sm[e] / (float)s;
   }
 }
 
@@ -111,9 +117,12 @@ __global__ void __launch_bounds__(256) coarse_kernel(const __grid_constant__ Clu
   if (C[0] > p.pyr.cap[0]) return;  // reported by gather_kernel
   const int64_t ubase = ((int64_t)(group * p.B + b) * p.Hkv + h) * p.pyr.rows;
   const float a = p.alpha, am = 1.f - p.alpha;
+  int P = 1;  // finest clusters under one level l-1 cluster
   for (int l = 1; l < p.pyr.n_levels; ++l) {
     const int f = p.pyr.fanout[l - 1];
     const int nc = min(C[l], p.pyr.cap[l]);
+    const float* cm = p.mean ? p.mean + (ubase + p.pyr.off[l - 1]) * D : nullptr;
+    float* Rm = p.mean ? p.mean + (ubase + p.pyr.off[l]) * D : nullptr;
     const float* cx = p.rmax + (ubase + p.pyr.off[l - 1]) * D;
     const float* cn = p.rmin + (ubase + p.pyr.off[l - 1]) * D;
     float* Rx = p.rmax + (ubase + p.pyr.off[l]) * D;
@@ -122,15 +131,23 @@ __global__ void __launch_bounds__(256) coarse_kernel(const __grid_constant__ Clu
     for (int i = threadIdx.x; i < nc * D; i += blockDim.x) {
       const int node = i / D, cc = i % D;
       const int q0 = node * f, q1 = min(q0 + f, C[l - 1]);
-      float x = kNegInf, n = kPosInf;
+      float x = kNegInf, n = kPosInf, wsum = 0.f;
+      int cnt = 0;
       for (int q = q0; q < q1; ++q) {
         x = fmaxf(x, cx[(int64_t)q * D + cc]);
         n = fminf(n, cn[(int64_t)q * D + cc]);
+        if (Rm) {  // children weighted by their finest clusters (the last may hold fewer)
+          const int w = min((q + 1) * P, C[0]) - q * P;
+          wsum = fmaf((float)w, cm[(int64_t)q * D + cc], wsum);
+          cnt += w;
+        }
       }
       Rx[i] = x;
       Rn[i] = n;
       Rp[i] = fmaf(a, x, am * n);
+      if (Rm) Rm[i] = wsum / (float)cnt;
     }
+    P *= f;
     __syncthreads();
   }
 }

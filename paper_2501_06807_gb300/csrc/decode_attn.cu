@@ -220,11 +220,12 @@ __device__ void seal_tail(const AttnParams& p, const Unit& u, const T* kcache) {
     return;
   }
   constexpr int PER = D / 32;
-  float mx[PER], mn[PER];
+  float mx[PER], mn[PER], sm[PER];
 #pragma unroll
   for (int i = 0; i < PER; ++i) {
     mx[i] = kNegInf;
     mn[i] = -kNegInf;
+    sm[i] = 0.f;
   }
 #pragma unroll 8
   for (int r = c_new * s; r < c_new * s + s; ++r) {
@@ -235,6 +236,7 @@ __device__ void seal_tail(const AttnParams& p, const Unit& u, const T* kcache) {
       const float v = to_float<T>(row[swz<T>(r, c)]);
       mx[i] = fmaxf(mx[i], v);
       mn[i] = fminf(mn[i], v);
+      sm[i] += v;
     }
   }
   const int64_t ubase = ((int64_t)(u.group * p.B + u.b) * p.Hkv + u.h) * p.pyr.rows;
@@ -251,6 +253,8 @@ __device__ void seal_tail(const AttnParams& p, const Unit& u, const T* kcache) {
     float* Rx = p.rmax + (ubase + p.pyr.off[l] + node) * D;
     float* Rn = p.rmin + (ubase + p.pyr.off[l] + node) * D;
     float* Rp = p.rep + (ubase + p.pyr.off[l] + node) * D;
+    float* Rm = p.mean ? p.mean + (ubase + p.pyr.off[l] + node) * D : nullptr;
+    const int n_old = c_new - node * prod;  // finest clusters the node held before
 #pragma unroll
     for (int i = 0; i < PER; ++i) {
       const int c = lane * PER + i;
@@ -262,6 +266,10 @@ __device__ void seal_tail(const AttnParams& p, const Unit& u, const T* kcache) {
       Rx[c] = x;
       Rn[c] = n;
       Rp[c] = fmaf(a, x, am * n);
+      if (Rm) {  // running mean over the node's finest clusters
+        const float m_new = sm[i] / (float)s;
+        Rm[c] = fresh ? m_new : fmaf((float)n_old, Rm[c], m_new) / (float)(n_old + 1);
+      }
     }
   }
 }

@@ -24,6 +24,7 @@ struct AttnParams {
   float* rmax;
   float* rmin;
   float* rep;
+  float* mean;  // optional, kept current by the seal
   Pyramid pyr;
   float alpha;
   int* n_tok;
@@ -53,9 +54,10 @@ struct SelectParams {
   int max_cand;  // power of two, capacity of the shared candidate arrays
   int row_buf;   // candidates whose summary rows are staged in shared memory at once
   int spec_first;  // the first round also scores the whole level below the coarsest
-  int metric;      // MPC_SIM_EQ3: rep; MPC_SIM_BOUND: r_max and r_min
+  int metric;      // MPC_SIM_EQ3: rep; MPC_SIM_BOUND: r_max and r_min; MPC_SIM_MEAN: mean
   const float* rmax;
   const float* rmin;
+  const float* mean;
 };
 
 struct StaticParams {
@@ -125,6 +127,7 @@ struct ClusterParams {
   float* rmax;
   float* rmin;
   float* rep;
+  float* mean;  // optional mean member key per cluster
   Pyramid pyr;
   float alpha;
   int* out_n_tok;

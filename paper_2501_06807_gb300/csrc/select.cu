@@ -94,9 +94,10 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   const int G = p.G;
   const int top = p.pyr.n_levels - 1;
   const int64_t unit_off = ((int64_t)(group * p.B + b) * p.Hkv + h) * p.pyr.rows * D;
-  // staged source w of a candidate: rep (Eq. 3), or r_max then r_min (Eq. 2),
-  // each into its own RB-row array of the buffer
-  const float* src0[2] = {(NSRC == 2 ? p.rmax : p.rep) + unit_off, (NSRC == 2 ? p.rmin : p.rep) + unit_off};
+  // staged source w of a candidate: rep (Eq. 3) or mean (average key), or
+  // r_max then r_min (Eq. 2), each into its own RB-row array of the buffer
+  const float* one = p.metric == MPC_SIM_MEAN ? p.mean : p.rep;
+  const float* src0[2] = {(NSRC == 2 ? p.rmax : one) + unit_off, (NSRC == 2 ? p.rmin : one) + unit_off};
   int* out = p.out_sel + ((int64_t)(group * p.B + b) * p.Hkv + h) * p.sel_cap;
   uint32_t phase = 0;
   bool timed_out = false;
@@ -104,7 +105,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   // similarity of staged row r for rows [0, nrows) of the buffer;
   // put(r, score) runs on the first lane of each row.  Channel order is
   // fixed: x, y, z, w per lane, then a butterfly over the row's lanes.
-  //   Eq. 3: q_sum . rep;  Eq. 2: sum_i max(q_i r_max_i, q_i r_min_i)
+  //   Eq. 3: q_sum . rep;  mean: q_sum . mean;  Eq. 2: sum_i max(q_i r_max_i, q_i r_min_i)
   auto score_rows = [&](int nrows, auto&& put) {
     const float4 qv = reinterpret_cast<const float4*>(qsum)[c4];
     const float* rows2 = rows + (size_t)RB * D;

@@ -25,9 +25,9 @@ from . import build as _build
 
 MPC_OK, MPC_ERR_INVALID_ARG, MPC_ERR_BAD_SHAPE, MPC_ERR_WORKSPACE, MPC_ERR_CUDA = 0, -1, -2, -3, -4
 MPC_F32, MPC_BF16 = 0, 1
-MPC_SIM_EQ3, MPC_SIM_BOUND = 0, 1
+MPC_SIM_EQ3, MPC_SIM_BOUND, MPC_SIM_MEAN = 0, 1, 2
 MAX_LEVELS = 4
-ABI_VERSION = 2
+ABI_VERSION = 3
 MAX_REFS = 128
 PPM = 1_000_000
 
@@ -61,7 +61,7 @@ class ClusterArgs(C.Structure):
                 ("cap_tokens", C.c_int32), ("r_max", C.c_void_p), ("r_min", C.c_void_p),
                 ("rep", C.c_void_p), ("summary_rows", C.c_int32), ("cluster_size", C.c_int32),
                 ("n_levels", C.c_int32), ("fanout", C.c_int32 * MAX_LEVELS), ("alpha", C.c_float),
-                ("out_n_tok", C.c_void_p)]
+                ("out_n_tok", C.c_void_p), ("mean", C.c_void_p)]
 
 
 class SelectArgs(C.Structure):
@@ -73,7 +73,7 @@ class SelectArgs(C.Structure):
                 ("n_levels", C.c_int32), ("fanout", C.c_int32 * MAX_LEVELS),
                 ("level_keep_ppm", C.c_int32 * MAX_LEVELS), ("sel_cap", C.c_int32),
                 ("out_sel", C.c_void_p), ("out_n_sel", C.c_void_p), ("metric", C.c_int32),
-                ("r_max", C.c_void_p), ("r_min", C.c_void_p)]
+                ("r_max", C.c_void_p), ("r_min", C.c_void_p), ("mean", C.c_void_p)]
 
 
 class AttnArgs(C.Structure):
@@ -87,7 +87,8 @@ class AttnArgs(C.Structure):
                 ("r_min", C.c_void_p), ("rep", C.c_void_p), ("summary_rows", C.c_int32),
                 ("cluster_size", C.c_int32), ("n_levels", C.c_int32), ("fanout", C.c_int32 * MAX_LEVELS),
                 ("alpha", C.c_float), ("n_tok", C.c_void_p), ("advance", C.c_int32),
-                ("scale", C.c_float), ("out", C.c_void_p), ("out_layer_stride", C.c_int64)]
+                ("scale", C.c_float), ("out", C.c_void_p), ("out_layer_stride", C.c_int64),
+                ("mean", C.c_void_p)]
 
 
 ENTRY_POINTS = ("mpc_static_evict_workspace_size", "mpc_build_clusters_workspace_size",
@@ -267,6 +268,7 @@ class Engine:
         self.kc = torch.zeros((n_layers, B, Hkv, self.cap_tokens, d), dtype=dtype, device=dev)
         self.vc = torch.zeros_like(self.kc)
         self.rmax = torch.zeros((G, B, Hkv, self.rows, d), **f32)
+        self.mean = torch.zeros((G, B, Hkv, self.rows, d), **f32)  # mean member key per cluster
         self.rmin = torch.zeros_like(self.rmax)
         self.rep = torch.zeros_like(self.rmax)
         self.n_tok = torch.zeros((B,), **i32)
@@ -331,6 +333,7 @@ class Engine:
         a.kept, a.keep_cap, a.n_keep = _ptr(self.kept), self.keep_cap, _ptr(self.n_keep)
         a.kc, a.vc, a.cache_layer_stride, a.cap_tokens = _ptr(self.kc), _ptr(self.vc), self.kc.stride(0), self.cap_tokens
         a.r_max, a.r_min, a.rep, a.summary_rows = _ptr(self.rmax), _ptr(self.rmin), _ptr(self.rep), self.rows
+        a.mean = _ptr(self.mean)
         a.cluster_size, a.n_levels, a.fanout, a.alpha = self.s, self.n_levels, _fan(self.fanouts), self.alpha
         a.out_n_tok = _ptr(self.n_tok)
         _check(lib.mpc_build_clusters(C.byref(a), None, 0, C.c_void_p(_stream())))
@@ -343,7 +346,8 @@ class Engine:
     # ---------------------------------------------------------- decode ----
     def select(self, q: torch.Tensor, metric: int = MPC_SIM_EQ3):
         """q: [L][B][Hq][d] queries of this step (only the leaders' are read);
-        metric MPC_SIM_EQ3 (Eq. 3 with rep) or MPC_SIM_BOUND (Eq. 2 bound)."""
+        metric MPC_SIM_EQ3 (Eq. 3 with rep), MPC_SIM_BOUND (Eq. 2 bound) or
+        MPC_SIM_MEAN (mean member key)."""
         lib = load()
         refs = _refs(self.refs_lead)
         a = SelectArgs()
@@ -356,7 +360,7 @@ class Engine:
         a.cluster_size, a.n_levels, a.fanout = self.s, self.n_levels, _fan(self.fanouts)
         a.level_keep_ppm = _fan(self.level_keep_ppm)
         a.sel_cap, a.out_sel, a.out_n_sel = self.sel_cap, _ptr(self.sel), _ptr(self.n_sel)
-        a.metric, a.r_max, a.r_min = metric, _ptr(self.rmax), _ptr(self.rmin)
+        a.metric, a.r_max, a.r_min, a.mean = metric, _ptr(self.rmax), _ptr(self.rmin), _ptr(self.mean)
         _check(lib.mpc_select(C.byref(a), None, 0, C.c_void_p(_stream())))
 
     def attn_args(self, q, k_new, v_new, advance=True, refs_list=None, out=None) -> AttnArgs:
@@ -372,6 +376,7 @@ class Engine:
         a.kc, a.vc, a.cache_layer_stride, a.cap_tokens = _ptr(self.kc), _ptr(self.vc), self.kc.stride(0), self.cap_tokens
         a.sel, a.n_sel, a.sel_cap = _ptr(self.sel), _ptr(self.n_sel), self.sel_cap
         a.r_max, a.r_min, a.rep, a.summary_rows = _ptr(self.rmax), _ptr(self.rmin), _ptr(self.rep), self.rows
+        a.mean = _ptr(self.mean)
         a.cluster_size, a.n_levels, a.fanout, a.alpha = self.s, self.n_levels, _fan(self.fanouts), self.alpha
         a.n_tok, a.advance, a.scale = _ptr(self.n_tok), int(bool(advance)), self.scale
         out = self.out if out is None else out

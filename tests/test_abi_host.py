@@ -33,7 +33,7 @@ def test_exports_every_declared_symbol(lib):
                          capture_output=True, text=True).stdout
     exported = set(re.findall(r"\b(mpc_\w+)\b", out))
     assert set(names) <= exported
-    assert lib.mpc_abi_version() == mpcache.ABI_VERSION == 2
+    assert lib.mpc_abi_version() == mpcache.ABI_VERSION == 3
 
 
 def test_struct_layout_matches_c(tmp_path):

@@ -3,7 +3,8 @@
 Tolerances:
 * attention outputs: max |o - o_ref| / max |o_ref| per output vector
   <= 1e-5 (fp32 KV) and <= 2e-3 (bf16 KV);
-* summaries: r_max / r_min bit-exact, rep within fp32 rounding;
+* summaries: r_max / r_min bit-exact, rep within fp32 rounding, the mean key
+  within 64 u of the largest member key;
 * cache contents: bit-exact;
 * scores and index sets: within bands derived from the kernels' fp32
   arithmetic (``static_band`` / ``select_band``); an index set must equal
@@ -127,6 +128,11 @@ def test_attention_cache_and_seal(dtype, d, Hq, Hkv, s, fan, N, E):
                         assert np.array_equal(eng.rmin[grp, b, h, rows].cpu().double().numpy(), lv.r_min)
                         rep = eng.rep[grp, b, h, rows].cpu().double().numpy()
                         assert np.allclose(rep, lv.rep, rtol=4e-7, atol=4e-7 * np.abs(lv.rep).max(initial=0))
+                        # mean key: fp32 sums of s rows, weighted child means and
+                        # running means at seals; bounded by 64 u of the largest key
+                        mean = eng.mean[grp, b, h, rows].cpu().double().numpy()
+                        kmax = np.abs(caches[(l, b, h)][0][:n_tok]).max(initial=0)
+                        assert np.allclose(mean, lv.mean, rtol=0, atol=64 * 2.0 ** -24 * kmax)
 
     check_pyramid(N)
     scale = 1 / math.sqrt(d)
@@ -194,7 +200,7 @@ SELECT_CASES = [
 ]
 
 
-@pytest.mark.parametrize("metric", ["eq3", "bound"])
+@pytest.mark.parametrize("metric", ["eq3", "bound", "mean"])
 @pytest.mark.parametrize("dtype,d,Hq,Hkv,s,fan,keep,N,B", SELECT_CASES)
 def test_selection(dtype, d, Hq, Hkv, s, fan, keep, N, B, metric):
     _check_selection(dtype, d, Hq, Hkv, s, fan, keep, N, B, metric, 0.6)
@@ -224,7 +230,8 @@ def _check_selection(dtype, d, Hq, Hkv, s, fan, keep, N, B, metric, alpha):
     ties = 0
     for rep_i in range(3):
         q = (torch.randn((L, B, Hq, d), generator=g) * 2).to(dtype)
-        eng.select(q.cuda(), mpcache.MPC_SIM_BOUND if metric == "bound" else mpcache.MPC_SIM_EQ3)
+        eng.select(q.cuda(), {"eq3": mpcache.MPC_SIM_EQ3, "bound": mpcache.MPC_SIM_BOUND,
+                              "mean": mpcache.MPC_SIM_MEAN}[metric])
         sel = eng.sel.cpu().numpy()
         n_sel = eng.n_sel.cpu().numpy()
         for b in range(B):
