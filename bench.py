@@ -259,35 +259,57 @@ def run_ours(args, rank, world, dist):
     ms_per_step = total_ms / args.steps
     value = job_value(attended, world, ms_per_step)
 
-    # e2e through the public API with host buffers
+    # e2e through the public API with host buffers.  The step copies what the
+    # path reads: the leader layers' keys and window queries first (static
+    # eviction reads only those), then, on a side stream while static
+    # eviction runs, the other layers' keys, all values and the decode
+    # inputs; gathering waits for the side stream.  Non-leader window
+    # queries are never read, so they are not copied.
     e2e = None
     if not args.no_e2e:
         host = {n: getattr(x, n).cpu().pin_memory() for n in ("k", "v", "q_win", "q", "k_new", "v_new")}
         host_lens = x.prompt_lens.pin_memory()
         out_host = torch.empty(out_all.shape, dtype=out_all.dtype).pin_memory()
-        h2d = sum(t.numel() * t.element_size() for t in host.values()) + host_lens.numel() * 4
+        others = [l for l in range(w.n_layers) if l not in leaders]
+        first = [(x.k[l], host["k"][l]) for l in leaders] + [(x.q_win[l], host["q_win"][l]) for l in leaders]
+        second = ([(x.k[l], host["k"][l]) for l in others] +
+                  [(getattr(x, n), host[n]) for n in ("v", "q", "k_new", "v_new")])
+        h2d = sum(src.numel() * src.element_size() for _, src in first + second) + host_lens.numel() * 4
         d2h = out_host.numel() * out_host.element_size()
+        side = torch.cuda.Stream(device=dev)
 
         def e2e_step():
-            for n, t in host.items():
-                getattr(x, n).copy_(t, non_blocking=True)
+            for dst, src in first:
+                dst.copy_(src, non_blocking=True)
             lens.copy_(host_lens, non_blocking=True)
-            prefill()
+            side.wait_stream(stream)  # the previous step is done with the inputs
+            with torch.cuda.stream(side):
+                for dst, src in second:
+                    dst.copy_(src, non_blocking=True)
+            eng.static_evict(x.k, x.q_win, lens, pt, w.page_size)
+            stream.wait_stream(side)
+            eng.build_clusters(x.k, x.v, pt, w.page_size)
             graph.replay()
             out_host.copy_(out_all, non_blocking=True)
 
-        e2e_step()
+        for _ in range(max(3, args.warmup)):  # first passes over new pinned pages run slow
+            e2e_step()
         torch.cuda.synchronize()
-        a, b = ev(), ev()
         if dist is not None:
             dist.barrier()
-        a.record(stream)
-        for _ in range(args.steps):
+        # per-step events: the host link is shared with other tenants of the
+        # machine and some passes copy several times slower, so the median step
+        # is the figure and the mean is reported beside it
+        em = [(ev(), ev()) for _ in range(args.steps)]
+        for m in em:
+            m[0].record(stream)
             e2e_step()
-        b.record(stream)
+            m[1].record(stream)
         torch.cuda.synchronize()
-        e2e_ms = max_over_ranks(a.elapsed_time(b) / args.steps, dist, dev)
+        per = [m[0].elapsed_time(m[1]) for m in em]
+        e2e_ms = max_over_ranks(statistics.median(per), dist, dev)
         e2e = {"value": job_value(attended, world, e2e_ms), "unit": UNIT, "ms_per_step": e2e_ms,
+               "ms_per_step_mean": max_over_ranks(sum(per) / len(per), dist, dev),
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
 
     pk, pk_kind = peaks()
