@@ -70,7 +70,7 @@ extern "C" {
 
 #define MPC_API __attribute__((visibility("default")))
 
-#define MPC_ABI_VERSION 3
+#define MPC_ABI_VERSION 4
 #define MPC_MAX_LEVELS 4
 #define MPC_MAX_REFS 128
 
@@ -294,6 +294,32 @@ MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace,
  *   ordering between them) race and corrupt each other's results.
  * - Allocates nothing (no cudaMalloc / cudaFree). */
 MPC_API int mpc_sparse_decode_attn_static_scratch(const mpc_attn_args* args, void* stream);
+
+/* ---- mpc_commonality --------------------------------------------------------
+ * Commonality of the selected clusters across adjacent layers (Sec. 2,
+ * Observation 3), the statistic that motivates cross-layer index sharing: for
+ * the first k entries S_l of the selection lists of n_layers consecutive
+ * layers (each its own leader), per (sequence b, kv head h)
+ *   out_total[b][h] = sum over l < n_layers - m of |S_l n ... n S_{l+m}|
+ *   out_score[b][h] = out_total[b][h] / (k (n_layers - m))
+ * 1 means the layers selected the same clusters.  sel entries are cluster ids
+ * < n_clusters or -1 (padding, ignored); an id >= n_clusters sets status bit 4.
+ * Read-only on sel; asynchronous on stream. */
+typedef struct {
+  uint32_t struct_size;        /* sizeof(mpc_commonality_args) */
+  int32_t n_layers;            /* >= 2 */
+  int32_t batch, n_kv_heads;
+  const int32_t* sel;          /* device [n_layers][batch][n_kv_heads][sel_cap] */
+  int64_t sel_layer_stride;    /* elements between layers */
+  int32_t sel_cap;
+  int32_t n_clusters;          /* every id < n_clusters (bitmap size) */
+  int32_t k;                   /* entries compared per list, 1 .. sel_cap */
+  int32_t m;                   /* windows of m + 1 layers, 1 .. n_layers - 1 */
+  int32_t* out_total;          /* device [batch][n_kv_heads] */
+  float* out_score;            /* device [batch][n_kv_heads] */
+} mpc_commonality_args;
+
+MPC_API int mpc_commonality(const mpc_commonality_args* args, void* stream);
 
 /* Rows of the summary pyramid for a cache of cap_tokens rows (the sum of the
  * level capacities above), or a negative MPC_ERR_* code. */

@@ -417,8 +417,8 @@ MPC_API int mpc_device_status(int* flags) {
   if (flags == nullptr) return fail(MPC_ERR_INVALID_ARG, "flags is NULL");
   const cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
-  const int parts[5] = {take_status_attn(), take_status_select(), take_status_clusters(), take_status_static(),
-                        take_status_score_tc()};
+  const int parts[6] = {take_status_attn(),   take_status_select(),   take_status_clusters(),
+                        take_status_static(), take_status_score_tc(), take_status_commonality()};
   int v = 0;
   for (int x : parts) {
     if (x < 0) return fail(MPC_ERR_CUDA, "reading the device status word failed");

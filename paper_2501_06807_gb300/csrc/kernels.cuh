@@ -148,6 +148,7 @@ int static_tile_smem(int D);
 
 // Records `msg` as this thread's last error (mpc_last_error) and returns code.
 int set_error(int code, const char* msg);
+int take_status_commonality();
 
 // Device status word of each translation unit: read it and clear it.
 int take_status_attn();

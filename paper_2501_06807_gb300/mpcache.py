@@ -27,7 +27,7 @@ MPC_OK, MPC_ERR_INVALID_ARG, MPC_ERR_BAD_SHAPE, MPC_ERR_WORKSPACE, MPC_ERR_CUDA 
 MPC_F32, MPC_BF16 = 0, 1
 MPC_SIM_EQ3, MPC_SIM_BOUND, MPC_SIM_MEAN = 0, 1, 2
 MAX_LEVELS = 4
-ABI_VERSION = 3
+ABI_VERSION = 4
 MAX_REFS = 128
 PPM = 1_000_000
 
@@ -76,6 +76,13 @@ class SelectArgs(C.Structure):
                 ("r_max", C.c_void_p), ("r_min", C.c_void_p), ("mean", C.c_void_p)]
 
 
+class CommonalityArgs(C.Structure):
+    _fields_ = [("struct_size", C.c_uint32), ("n_layers", C.c_int32), ("batch", C.c_int32),
+                ("n_kv_heads", C.c_int32), ("sel", C.c_void_p), ("sel_layer_stride", C.c_int64),
+                ("sel_cap", C.c_int32), ("n_clusters", C.c_int32), ("k", C.c_int32), ("m", C.c_int32),
+                ("out_total", C.c_void_p), ("out_score", C.c_void_p)]
+
+
 class AttnArgs(C.Structure):
     _fields_ = [("struct_size", C.c_uint32), ("n_refs", C.c_int32), ("refs", C.POINTER(LayerRef)),
                 ("batch", C.c_int32), ("n_q_heads", C.c_int32), ("n_kv_heads", C.c_int32),
@@ -95,7 +102,7 @@ ENTRY_POINTS = ("mpc_static_evict_workspace_size", "mpc_build_clusters_workspace
                 "mpc_select_workspace_size", "mpc_sparse_decode_attn_workspace_size",
                 "mpc_static_evict", "mpc_build_clusters", "mpc_select", "mpc_sparse_decode_attn",
                 "mpc_summary_rows", "mpc_last_error", "mpc_device_status", "mpc_abi_version",
-                "mpc_sparse_decode_attn_static_scratch")
+                "mpc_sparse_decode_attn_static_scratch", "mpc_commonality")
 
 _LIB = None
 
@@ -128,8 +135,11 @@ def load(path: Optional[str] = None) -> C.CDLL:
     lib.mpc_abi_version.restype = C.c_int
     lib.mpc_sparse_decode_attn_static_scratch.restype = C.c_int
     lib.mpc_sparse_decode_attn_static_scratch.argtypes = [C.c_void_p, C.c_void_p]
+    lib.mpc_commonality.restype = C.c_int
+    lib.mpc_commonality.argtypes = [C.c_void_p, C.c_void_p]
     if lib.mpc_abi_version() != ABI_VERSION:
-        raise MPCError(f"libmpcache ABI {lib.mpc_abi_version()} does not match the binding's {ABI_VERSION}")
+        raise MPCError(MPC_ERR_INVALID_ARG,
+                       f"libmpcache ABI {lib.mpc_abi_version()} does not match the binding's {ABI_VERSION}")
     if path is None:
         _LIB = lib
     return lib
@@ -204,6 +214,39 @@ def sharing_leader(layer: int, share_every: int) -> int:
     if share_every <= 1 or layer < 2:
         return layer
     return 2 + share_every * ((layer - 2) // share_every)
+
+
+def commonality(sel: torch.Tensor, k: int, m: int, n_clusters: int):
+    """Commonality of per-layer selections (Sec. 2, Observation 3; mpc_commonality).
+
+    sel: int32 [L][B][Hkv][sel_cap] selections of consecutive layers, each its
+    own leader (ids ascending, -1 padded).  Returns (total, score), each
+    [B][Hkv]: total = sum over l < L - m of |S_l n ... n S_{l+m}| over the
+    first k ids of each list, score = total / (k (L - m)).
+    """
+    L, B, Hkv, cap = sel.shape
+    total = torch.zeros((B, Hkv), dtype=torch.int32, device=sel.device)
+    score = torch.zeros((B, Hkv), dtype=torch.float32, device=sel.device)
+    a = CommonalityArgs()
+    a.struct_size = C.sizeof(CommonalityArgs)
+    a.n_layers, a.batch, a.n_kv_heads = L, B, Hkv
+    a.sel, a.sel_layer_stride, a.sel_cap = _ptr(sel), sel.stride(0), cap
+    a.n_clusters, a.k, a.m = n_clusters, k, m
+    a.out_total, a.out_score = _ptr(total), _ptr(score)
+    _check(load().mpc_commonality(C.byref(a), C.c_void_p(_stream())))
+    return total, score
+
+
+def choose_share_every(scores: dict, threshold: float) -> int:
+    """Adaptive sharing-group size: the largest m whose commonality score of
+    m + 1 adjacent layers (``scores[m]``, e.g. the mean over sequences and kv
+    heads) reaches ``threshold`` -- groups of m + 1 layers then select nearly
+    the same clusters, so one leader can serve them -- else 1 (no sharing)."""
+    best = 1
+    for m in sorted(scores):
+        if scores[m] >= threshold:
+            best = max(best, m + 1)
+    return best
 
 
 def summary_rows(cap_tokens: int, s: int, fanouts: Sequence[int]) -> int:

@@ -33,13 +33,14 @@ def test_exports_every_declared_symbol(lib):
                          capture_output=True, text=True).stdout
     exported = set(re.findall(r"\b(mpc_\w+)\b", out))
     assert set(names) <= exported
-    assert lib.mpc_abi_version() == mpcache.ABI_VERSION == 3
+    assert lib.mpc_abi_version() == mpcache.ABI_VERSION == 4
 
 
 def test_struct_layout_matches_c(tmp_path):
     structs = {"mpc_layer_ref": mpcache.LayerRef, "mpc_kv_tensor": mpcache.KvTensor,
                "mpc_static_args": mpcache.StaticArgs, "mpc_cluster_args": mpcache.ClusterArgs,
-               "mpc_select_args": mpcache.SelectArgs, "mpc_attn_args": mpcache.AttnArgs}
+               "mpc_select_args": mpcache.SelectArgs, "mpc_attn_args": mpcache.AttnArgs,
+               "mpc_commonality_args": mpcache.CommonalityArgs}
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "mpcache.h"', 'int main(void){']
     for cname, py in structs.items():
         lines.append(f'printf("{cname} size %zu\\n", sizeof({cname}));')
@@ -179,3 +180,23 @@ def test_host_rules_match_oracle():
 def test_missing_library_fails_loudly(tmp_path):
     with pytest.raises(OSError):
         mpcache.load(str(tmp_path / "nope.so"))
+
+
+def test_commonality_validation(lib):
+    a = mpcache.CommonalityArgs()
+    a.struct_size = C.sizeof(mpcache.CommonalityArgs)
+    a.n_layers, a.batch, a.n_kv_heads, a.sel_cap, a.n_clusters, a.k, a.m = 4, 2, 3, 8, 100, 8, 1
+    a.sel_layer_stride = 2 * 3 * 8
+    a.sel = a.out_total = a.out_score = None
+    assert lib.mpc_commonality(C.byref(a), None) == mpcache.MPC_ERR_INVALID_ARG  # NULL pointers
+    for field, bad in (("m", 0), ("m", 4), ("k", 9), ("n_layers", 1), ("sel_layer_stride", 47)):
+        b = mpcache.CommonalityArgs.from_buffer_copy(a)
+        setattr(b, field, bad)
+        assert lib.mpc_commonality(C.byref(b), None) == mpcache.MPC_ERR_BAD_SHAPE, field
+    a.struct_size = 3
+    assert lib.mpc_commonality(C.byref(a), None) == mpcache.MPC_ERR_INVALID_ARG
+
+
+def test_choose_share_every():
+    assert mpcache.choose_share_every({1: 0.95, 2: 0.9, 3: 0.6}, 0.85) == 3   # groups of 3 layers
+    assert mpcache.choose_share_every({1: 0.5}, 0.85) == 1                     # no sharing

@@ -411,3 +411,57 @@ def test_pipeline_gqa_three_levels_needles():
 def test_pipeline_paged_ragged_batch():
     w = synth.C4.replace(n_layers=3, batch=3, prompt_len=700, prompt_len_min=300, n_q_heads=4, n_kv_heads=4)
     _pipeline(w, 10, [0, 1, 2])
+
+
+# ------------------------------------------------- commonality score ----
+
+@pytest.mark.parametrize("L,m,k,n_clusters,overlap", [(6, 1, 12, 200, 0.8), (10, 3, 26, 512, 0.6),
+                                                      (4, 3, 5, 33, 1.0), (32, 2, 64, 4000, 0.3)])
+def test_commonality_synthetic(L, m, k, n_clusters, overlap):
+    """mpc_commonality against the oracle's commonality (Sec. 2, Obs. 3) on
+    index sets with a controlled share of common ids; totals are exact."""
+    from paper_2501_06807_gb300 import mpcache
+    rng = np.random.default_rng(L * 100 + k)
+    B, Hkv, cap = 2, 3, k + 4
+    sel = np.full((L, B, Hkv, cap), -1, dtype=np.int32)
+    sets = {}
+    for b in range(B):
+        for h in range(Hkv):
+            base = rng.choice(n_clusters, k, replace=False)
+            for l in range(L):
+                keep = base[rng.random(k) < overlap]
+                fresh = rng.choice(np.setdiff1d(np.arange(n_clusters), keep), k - len(keep), replace=False)
+                ids = np.sort(np.concatenate([keep, fresh]))
+                sel[l, b, h, :k] = ids
+                sets[(b, h, l)] = list(ids)
+    total, score = mpcache.commonality(torch.from_numpy(sel).cuda(), k, m, n_clusters)
+    total, score = total.cpu().numpy(), score.cpu().numpy()
+    for b in range(B):
+        for h in range(Hkv):
+            ref = O.commonality([sets[(b, h, l)] for l in range(L)], k, m)
+            assert total[b, h] == round(ref * k * (L - m))
+            assert abs(score[b, h] - ref) <= 1e-6 * max(ref, 1e-6)
+
+
+def test_commonality_of_unshared_selections():
+    """Every layer its own leader (m = 1 sharing): the commonality of the
+    engine's per-layer selections equals the oracle's on the same sets."""
+    from paper_2501_06807_gb300 import mpcache
+    w = synth.C3.replace(n_layers=6, prompt_len=2048, prompt_len_min=2048, share_every=1, decode_steps=2)
+    R = mpcache.window_rows_bound(w.prompt_len, w.window_ppm, w.long_window_ppm, w.long_prompt_threshold)
+    x = synth.generate(w, R, device="cuda", decode_steps=2)
+    eng = H.make_engine(w, 2)
+    eng.prefill(x.k, x.v, x.q_win, x.prompt_lens.cuda())
+    eng.select(x.q[0])
+    torch.cuda.synchronize()
+    n_sel = int(eng.n_sel[0])
+    sel = eng.sel[:, :, :, :]                    # [L (each its own group)][B][Hkv][sel_cap]
+    assert sel.shape[0] == w.n_layers
+    n_clusters = int(eng.n_tok[0]) // w.cluster_size
+    for m in (1, 2):
+        total, score = mpcache.commonality(sel.contiguous(), n_sel, m, n_clusters)
+        s_cpu = sel.cpu().numpy()
+        for b in range(w.batch):
+            for h in range(w.n_kv_heads):
+                ref = O.commonality([list(s_cpu[l, b, h, :n_sel]) for l in range(w.n_layers)], n_sel, m)
+                assert int(total[b, h]) == round(ref * n_sel * (w.n_layers - m))
