@@ -413,6 +413,16 @@ def test_pipeline_paged_ragged_batch():
     _pipeline(w, 10, [0, 1, 2])
 
 
+def test_pipeline_token_wise_without_static_eviction():
+    """The LongCache-style comparator (next-rows item 3): no static eviction
+    (keep every prompt token) and one token per finest cluster, so selection
+    ranks single tokens through a two-level pyramid of token groups."""
+    w = synth.C3.replace(n_layers=2, prompt_len=1024, prompt_len_min=1024, n_q_heads=8, n_kv_heads=2,
+                         keep_ppm=1_000_000, cluster_size=1, fanouts=(16,), level_keep_ppm=(50_000, 250_000),
+                         share_every=1)
+    _pipeline(w, 6, [0, 1])
+
+
 # ------------------------------------------------- commonality score ----
 
 @pytest.mark.parametrize("L,m,k,n_clusters,overlap", [(6, 1, 12, 200, 0.8), (10, 3, 26, 512, 0.6),
