@@ -37,7 +37,12 @@ the design notes):
     may be partial; a coarse summary is the max / min over all member tokens;
   * GQA selection scores (sum_g q_g) . rep once per kv head;
   * sharing: layers 0 and 1 lead themselves; for l >= 2 the leader is
-    2 + m * floor((l - 2) / m).
+    2 + m * floor((l - 2) / m);
+  * fixed-point Eq. 3 (the ring arithmetic of App. B emulated on plaintext
+    values): f = 18 fractional bits unless given, enc(x) = rint(x 2^f) with
+    ties to even, truncation by floor after each product and once per dot
+    product, alpha and 1 - alpha encoded as public constants, scores
+    saturated to int32 for ranking.
 """
 from __future__ import annotations
 
@@ -188,23 +193,75 @@ def cluster_pyramid(keys: np.ndarray, s: int, fanouts: Sequence[int],
     return levels
 
 
+# ------------------------------------------- fixed-point emulation ----
+# The MPC runtime evaluates Eq. 3 on secret shares of fixed-point values in
+# the ring Z_{2^64} (App. B: arithmetic sharing with l = 64).  In plaintext
+# the shares add up to the value itself, so the arithmetic is emulated here
+# on the values: x is encoded as rint(x 2^f) (f fractional bits, the ring's
+# two's-complement representative), sums are ring sums, and a product of two
+# encodings carries 2f fractional bits until one truncation (an arithmetic
+# shift right by f, i.e. floor) brings it back to f.  A dot product is one
+# ring sum of products truncated once.
+
+FXP_FRAC_BITS = 18  # default fractional bits of the encoding
+
+
+def fxp_encode(x, frac_bits: int = FXP_FRAC_BITS) -> np.ndarray:
+    """rint(x 2^f) (round half to even) as int64; |x| must stay below 2^(62-f)."""
+    v = np.rint(np.asarray(x, dtype=np.float64) * float(1 << frac_bits))
+    if np.any(np.abs(v) >= 2.0 ** 62):
+        raise ValueError("value out of the fixed-point range")
+    return v.astype(np.int64)
+
+
+def fxp_dot(a: np.ndarray, b: np.ndarray, frac_bits: int = FXP_FRAC_BITS) -> np.ndarray:
+    """Truncated ring dot product over the last axis: floor((sum_i a_i b_i
+    mod 2^64) / 2^f).  numpy int64 products and sums wrap modulo 2^64, and
+    >> on int64 is the arithmetic (floor) shift."""
+    with np.errstate(over="ignore"):
+        return (np.asarray(a, dtype=np.int64) * np.asarray(b, dtype=np.int64)).sum(axis=-1) >> frac_bits
+
+
+def sim_fxp(q_group: np.ndarray, r_max: np.ndarray, r_min: np.ndarray, alpha: float,
+            frac_bits: int = FXP_FRAC_BITS) -> np.ndarray:
+    """Eq. 3 in the ring, per cluster c (rows of r_max / r_min, [C][d]):
+      q_i     = sum_g enc(q_gi)                         (ring sum)
+      rep_ci  = dot(enc(alpha), enc(r_max_ci)) + dot(enc(1 - alpha), enc(r_min_ci))
+      sim_c   = dot(q, rep_c)
+    with alpha and 1 - alpha public constants encoded like any value (each
+    product of rep is a one-term dot, truncated on its own).  Returns the
+    int64 scores (units of 2^-f) saturated to the int32 range."""
+    d = np.shape(q_group)[-1]
+    q = fxp_encode(q_group, frac_bits).reshape(-1, d).sum(axis=0)
+    ea = fxp_encode([alpha], frac_bits)
+    eb = fxp_encode([1.0 - alpha], frac_bits)
+    emax = fxp_encode(r_max, frac_bits).reshape(-1, d)
+    emin = fxp_encode(r_min, frac_bits).reshape(-1, d)
+    rep = fxp_dot(emax[..., None], ea[None], frac_bits) + fxp_dot(emin[..., None], eb[None], frac_bits)
+    sc = fxp_dot(q[None, :], rep, frac_bits)
+    return np.clip(sc, -(1 << 31), (1 << 31) - 1)
+
+
 def hierarchical_select(q_group: np.ndarray, levels: List[Level],
                         fanouts: Sequence[int], level_keep_ppm: Sequence[int],
-                        trace: Optional[list] = None, metric: str = "eq3") -> np.ndarray:
+                        trace: Optional[list] = None, metric: str = "eq3",
+                        alpha: float = 0.6, frac_bits: int = FXP_FRAC_BITS) -> np.ndarray:
     """Coarse-to-fine cluster selection (Sec. 3.3; Alg. 2 Sim + topk).
 
     q_group: [G][d] decode queries of one kv group, scored through their sum
     q = sum_g q_g.  The similarity of cluster c is q . rep_c (Eq. 3, the
     default); with metric="bound", the upper bound of Eq. 2,
     sum_i max(q_i r_max_ci, q_i r_min_ci), evaluated on the same summed query;
-    with metric="mean", q . mean_c (the average-key baseline of App. G).
+    with metric="mean", q . mean_c (the average-key baseline of App. G);
+    with metric="fxp", Eq. 3 in the fixed-point ring (sim_fxp, weight
+    ``alpha``, ``frac_bits`` fractional bits), ranked as integers.
     At the coarsest level every cluster is a candidate; at each finer level
     the candidates are the children of the kept parents.  Returns the kept
     finest-level ids in ascending order.  ``trace``, if given, receives per
     level (coarsest first) the candidate ids, their similarities and k, for
     tests that need the margin at each cut.
     """
-    if metric not in ("eq3", "bound", "mean"):
+    if metric not in ("eq3", "bound", "mean", "fxp"):
         raise ValueError(metric)
     qsum = np.asarray(q_group, dtype=np.float64).sum(axis=0)
     n = len(levels)
@@ -218,6 +275,8 @@ def hierarchical_select(q_group: np.ndarray, levels: List[Level],
             sim = lev.rep[cand] @ qsum
         elif metric == "mean":
             sim = lev.mean[cand] @ qsum
+        elif metric == "fxp":
+            sim = sim_fxp(q_group, lev.r_max[cand], lev.r_min[cand], alpha, frac_bits).astype(np.float64)
         else:
             sim = np.maximum(lev.r_max[cand] * qsum, lev.r_min[cand] * qsum).sum(axis=1)
         k = selected_count(lev.rep.shape[0], level_keep_ppm[lvl], len(cand))

@@ -288,14 +288,16 @@ def test_p6_bound_and_linearisation():
 
 # ---------------------------------------------------------------- P7 -------
 
-def _brute_select(qsum, keys, s, fanouts, level_keep, metric="eq3"):
+def _brute_select(qsum, keys, s, fanouts, level_keep, metric="eq3", qg=None, frac_bits=18):
     """Coarse-to-fine selection by exhaustive search: at every level, try every
     subset of the candidates of the required size and keep the one with the
     largest total similarity (ties: the lexicographically smallest id list).
     Summaries are recomputed from the member tokens with explicit loops; the
-    similarity is Eq. 3 (alpha 0.6), the Eq. 2 bound or the mean key, channel by
-    channel."""
+    similarity is Eq. 3 (alpha 0.6), the Eq. 2 bound, the mean key, or Eq. 3
+    in fixed point with Python integers (round() is half to even, // floors),
+    channel by channel."""
     N, d = keys.shape
+    one = 1 << frac_bits
     n_full = N // s
     sizes = [s]
     for f in fanouts:
@@ -315,11 +317,18 @@ def _brute_select(qsum, keys, s, fanouts, level_keep, metric="eq3"):
                 total += qsum[i] * (0.6 * mx + 0.4 * mn)
             elif metric == "bound":
                 total += max(qsum[i] * mx, qsum[i] * mn)
+            elif metric == "fxp":
+                qi = sum(round(float(qg[g][i]) * one) for g in range(len(qg)))
+                rep = round(0.6 * one) * round(float(mx) * one) // one + \
+                    round(0.4 * one) * round(float(mn) * one) // one
+                total += qi * rep
             else:
                 acc = 0.0
                 for t in toks:
                     acc += keys[t][i]
                 total += qsum[i] * acc / len(toks)
+        if metric == "fxp":
+            return float(min(max(total // one, -(1 << 31)), (1 << 31) - 1))
         return total
 
     n_level = [n_full]
@@ -341,7 +350,7 @@ def _brute_select(qsum, keys, s, fanouts, level_keep, metric="eq3"):
     return chosen
 
 
-@pytest.mark.parametrize("metric", ["eq3", "bound", "mean"])
+@pytest.mark.parametrize("metric", ["eq3", "bound", "mean", "fxp"])
 @pytest.mark.parametrize("seed", range(6))
 def test_p7_brute_force_tiny(seed, metric):
     rng = np.random.default_rng(100 + seed)
@@ -353,9 +362,109 @@ def test_p7_brute_force_tiny(seed, metric):
     qg = rng.standard_normal((G, d))
     keep = O.level_keep_fractions(int(rng.choice([250_000, 400_000])), 1 + len(fan))
     levels = O.cluster_pyramid(keys, s, fan, 0.6)
-    got = O.hierarchical_select(qg, levels, fan, keep, metric=metric)
-    want = _brute_select(qg.sum(0), keys, s, fan, keep, metric)
+    # few fractional bits make equal fixed-point scores (the tie rule) likely
+    fb = (3, 6, 18)[seed % 3]
+    got = O.hierarchical_select(qg, levels, fan, keep, metric=metric, frac_bits=fb)
+    want = _brute_select(qg.sum(0), keys, s, fan, keep, metric, qg=qg, frac_bits=fb)
     assert list(got) == sorted(want)
+
+
+# ------------------------------------------------ fixed-point emulation ----
+
+def test_fxp_worked_example():
+    g = _golden("fxp_eq3_ring_worked_example.txt")
+    got = O.sim_fxp(np.array(g["a_q"]), np.array(g["a_r_max"]), np.array(g["a_r_min"]),
+                    g["a_alpha"][0][0], int(g["a_f"][0][0]))
+    assert got.tolist() == [int(g["a_sim"][0][0])]
+    got = O.sim_fxp(np.array(g["b_q"]), np.array(g["b_r_max"]), np.array(g["b_r_min"]),
+                    g["b_alpha"][0][0], int(g["b_f"][0][0]))
+    assert got.tolist() == [int(g["b_sim"][0][0])]
+    assert O.fxp_encode(g["enc_f3_in"][0], 3).tolist() == [int(v) for v in g["enc_f3_out"][0]]
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_fxp_exact_on_dyadic_inputs(seed):
+    # values on a 2^-4 grid, alpha = 3/4: every encoding and every truncation
+    # is exact at f = 16, so the ring result is Eq. 3 itself, computed here
+    # with exact rationals from the definition
+    from fractions import Fraction as F
+    rng = np.random.default_rng(700 + seed)
+    G, d, C = 3, 8, 5
+    qg = rng.integers(-40, 41, (G, d)) / 16.0
+    rmin = rng.integers(-60, 20, (C, d)) / 16.0
+    rmax = rmin + rng.integers(0, 50, (C, d)) / 16.0
+    got = O.sim_fxp(qg, rmax, rmin, 0.75, 16)
+    for c in range(C):
+        exact = sum(F(float(qg[gg, i])) * (F(3, 4) * F(float(rmax[c, i])) + F(1, 4) * F(float(rmin[c, i])))
+                    for gg in range(G) for i in range(d))
+        assert F(int(got[c]), 1 << 16) == exact
+
+
+def _fxp_bound(qg, r_max, r_min, fb):
+    """Rounding bound of the fixed-point Eq. 3 per cluster (derivation below)."""
+    G = len(qg)
+    q = np.asarray(qg).sum(0)
+    u = 2.0 ** -fb
+    e = G * u / 2
+    E = u / 2 * (np.abs(r_max) + np.abs(r_min)) + u / 2 * (1 + u) + 2 * u
+    rep_abs = np.maximum(np.abs(r_max), np.abs(r_min))
+    return (e * rep_abs + np.abs(q) * E + e * E).sum(axis=1) + u
+
+
+@pytest.mark.parametrize("fb", [6, 10, 18])
+def test_fxp_error_within_rounding_bound(fb):
+    # Encodings are off by at most u/2 (u = 2^-f), each truncation by less
+    # than u.  With q' = q + e (|e_i| <= G u/2) and rep' = rep + E
+    # (|E_i| <= u/2 (|r_max_i| + |r_min_i|) + u/2 (1 + u) + 2u):
+    #   |sim' - sim| <= sum_i (|e_i||rep_i| + |q_i||E_i| + |e_i||E_i|) + u
+    rng = np.random.default_rng(800 + fb)
+    G, d, C, a = 4, 128, 64, 0.6
+    qg = rng.standard_normal((G, d))
+    keys = rng.standard_normal((C * 16, d)) * np.where(np.arange(d) < 4, 8.0, 1.0)
+    lev = O.cluster_pyramid(keys, 16, (), a)[0]
+    got = O.sim_fxp(qg, lev.r_max, lev.r_min, a, fb) * 2.0 ** -fb
+    exact = lev.rep @ qg.sum(0)
+    bound = _fxp_bound(qg, lev.r_max, lev.r_min, fb)  # |rep_i| <= max(|r_max_i|, |r_min_i|)
+    err = np.abs(got - exact)
+    assert np.all(err <= bound * (1 + 1e-9))
+    assert err.max() > 0  # the rounding is live
+    assert err.max() > bound.max() / 200  # and the bound not vacuous
+
+
+def test_fxp_saturates_to_int32():
+    # scores beyond the int32 range of the ranking key saturate (equal keys
+    # then rank the lower id first)
+    q = np.full((1, 4), 100.0)
+    r = np.full((3, 4), 100.0)
+    got = O.sim_fxp(q, r, -r, 1.0, 18)
+    assert got.tolist() == [(1 << 31) - 1] * 3
+    assert O.sim_fxp(q, -r, -r, 1.0, 18).tolist() == [-(1 << 31)] * 3
+
+
+def test_fxp_ranking_matches_float_away_from_ties():
+    # where every cut of the float selection has a margin above twice the
+    # rounding bound, the fixed-point selection keeps the same clusters
+    n_clear = 0
+    for seed in range(8):
+        rng = np.random.default_rng(900 + seed)
+        G, d = 4, 32
+        keys = rng.standard_normal((2048, d))
+        qg = rng.standard_normal((G, d))
+        fan = (4, 4)
+        keep = O.level_keep_fractions(100_000, 3)
+        levels = O.cluster_pyramid(keys, 8, fan, 0.6)
+        trace = []
+        want = O.hierarchical_select(qg, levels, fan, keep, trace=trace)
+        got = O.hierarchical_select(qg, levels, fan, keep, metric="fxp", frac_bits=18)
+        clear = True
+        for lvl, (cand, sim, k) in zip(range(len(levels) - 1, -1, -1), trace):
+            srt = np.sort(sim)[::-1]
+            band = _fxp_bound(qg, levels[lvl].r_max[cand], levels[lvl].r_min[cand], 18).max()
+            clear &= bool(k >= len(srt) or srt[k - 1] - srt[k] > 2 * band)
+        if clear:
+            n_clear += 1
+            assert np.array_equal(got, want), seed
+    assert n_clear >= 6  # the comparison is live
 
 
 @pytest.mark.parametrize("seed", range(4))
