@@ -70,7 +70,7 @@ extern "C" {
 
 #define MPC_API __attribute__((visibility("default")))
 
-#define MPC_ABI_VERSION 4
+#define MPC_ABI_VERSION 5
 #define MPC_MAX_LEVELS 4
 #define MPC_MAX_REFS 128
 
@@ -85,7 +85,7 @@ enum mpc_status {
 enum mpc_dtype { MPC_F32 = 0, MPC_BF16 = 1 };
 
 /* Cluster similarity of mpc_select. */
-enum mpc_sim_metric { MPC_SIM_EQ3 = 0, MPC_SIM_BOUND = 1, MPC_SIM_MEAN = 2 };
+enum mpc_sim_metric { MPC_SIM_EQ3 = 0, MPC_SIM_BOUND = 1, MPC_SIM_MEAN = 2, MPC_SIM_FXP = 3 };
 
 typedef struct {
   int32_t layer;   /* index along per-layer tensors */
@@ -187,6 +187,16 @@ typedef struct {
  *   metric MPC_SIM_EQ3:   sim(c) = q . rep_c                          (Eq. 3)
  *   metric MPC_SIM_BOUND: sim(c) = sum_i max(q_i r_max_ci, q_i r_min_ci) (Eq. 2)
  *   metric MPC_SIM_MEAN:  sim(c) = q . mean_c, the mean member key (App. G baseline)
+ *   metric MPC_SIM_FXP:   Eq. 3 evaluated in the fixed-point ring Z_{2^64} of
+ *     the MPC runtime (App. B), emulated on plaintext values: with f =
+ *     frac_bits, enc(x) = rint(x 2^f) (ties to even) as a two's-complement
+ *     int64, tr(y) = floor(y / 2^f) (arithmetic shift), sums and products
+ *     modulo 2^64:
+ *       q_i   = sum_g enc(q_gi)
+ *       rep_i = tr(enc(alpha) enc(r_max_ci)) + tr(enc(1 - alpha) enc(r_min_ci))
+ *       sim   = tr(sum_i q_i rep_i), saturated to int32 and ranked as an integer
+ *     (1 - alpha taken in double precision from the float alpha; every
+ *     |value| must stay below 2^(62 - f), as an encoding needs)
  *   the coarsest level ranks all of its clusters; every finer level ranks
  *   the children of the clusters its parent level kept; level l keeps
  *   k_l = count(C_l, level_keep_ppm[l]) (at most its candidates); equal
@@ -210,10 +220,12 @@ typedef struct {
   int32_t sel_cap;             /* >= every k_1 */
   int32_t* out_sel;            /* device */
   int32_t* out_n_sel;          /* device [batch] */
-  int32_t metric;              /* MPC_SIM_EQ3 (0), MPC_SIM_BOUND (1) or MPC_SIM_MEAN (2) */
-  const float* r_max;          /* device, laid out like rep; read for MPC_SIM_BOUND only */
-  const float* r_min;          /* device, laid out like rep; read for MPC_SIM_BOUND only */
+  int32_t metric;              /* MPC_SIM_EQ3 (0), _BOUND (1), _MEAN (2) or _FXP (3) */
+  const float* r_max;          /* device, laid out like rep; read for MPC_SIM_BOUND / _FXP */
+  const float* r_min;          /* device, laid out like rep; read for MPC_SIM_BOUND / _FXP */
   const float* mean;           /* device, laid out like rep; read for MPC_SIM_MEAN only */
+  float alpha;                 /* MPC_SIM_FXP: Eq. 3 weight in [0, 1] */
+  int32_t frac_bits;           /* MPC_SIM_FXP: fractional bits f in [1, 24] */
 } mpc_select_args;
 
 /* ---- mpc_sparse_decode_attn ----------------------------------------------

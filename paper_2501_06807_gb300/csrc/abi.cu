@@ -224,9 +224,15 @@ int validate_select(const mpc_select_args* a, SelectParams* p) {
   MPC_TRY(make_pyramid(a->cap_tokens, a->cluster_size, a->n_levels, a->fanout, a->summary_rows, &p->pyr, true));
   for (int l = 0; l < a->n_levels; ++l) MPC_TRY(check_ppm(a->level_keep_ppm[l], "level_keep_ppm"));
   if (!aligned16(a->rep)) return fail(MPC_ERR_INVALID_ARG, "rep must be 16-byte aligned");
-  if (a->metric != MPC_SIM_EQ3 && a->metric != MPC_SIM_BOUND && a->metric != MPC_SIM_MEAN)
-    return fail(MPC_ERR_INVALID_ARG, "metric %d is not MPC_SIM_EQ3, MPC_SIM_BOUND or MPC_SIM_MEAN", a->metric);
-  if (a->metric == MPC_SIM_BOUND && (!aligned16(a->r_max) || !aligned16(a->r_min)))
+  if (a->metric != MPC_SIM_EQ3 && a->metric != MPC_SIM_BOUND && a->metric != MPC_SIM_MEAN &&
+      a->metric != MPC_SIM_FXP)
+    return fail(MPC_ERR_INVALID_ARG, "metric %d is not MPC_SIM_EQ3, _BOUND, _MEAN or _FXP", a->metric);
+  if (a->metric == MPC_SIM_FXP) {
+    if (!(a->alpha >= 0.f && a->alpha <= 1.f)) return fail(MPC_ERR_BAD_SHAPE, "alpha %g not in [0, 1]", a->alpha);
+    if (a->frac_bits < 1 || a->frac_bits > 24)
+      return fail(MPC_ERR_BAD_SHAPE, "frac_bits %d not in [1, 24]", a->frac_bits);
+  }
+  if (select_n_src(a->metric) == 2 && (!aligned16(a->r_max) || !aligned16(a->r_min)))
     return fail(MPC_ERR_INVALID_ARG, "r_max / r_min must be 16-byte aligned");
   if (a->metric == MPC_SIM_MEAN && !aligned16(a->mean)) return fail(MPC_ERR_INVALID_ARG, "mean must be 16-byte aligned");
   // bound on the candidates of any level
@@ -274,10 +280,17 @@ int validate_select(const mpc_select_args* a, SelectParams* p) {
     if (r > p->pyr.cap[l]) r = p->pyr.cap[l];
     if (r > need) need = r;
   }
-  const int n_src = a->metric == MPC_SIM_BOUND ? 2 : 1;  // summary rows per candidate
+  const int n_src = select_n_src(a->metric);  // summary rows per candidate
   p->metric = a->metric;
   p->rmax = a->r_max;
   p->rmin = a->r_min;
+  if (a->metric == MPC_SIM_FXP) {
+    // public constants enc(alpha), enc(1 - alpha): x 2^f is exact in double,
+    // nearbyint rounds ties to even
+    p->frac_bits = a->frac_bits;
+    p->fxp_a = (long long)std::nearbyint(std::ldexp((double)a->alpha, a->frac_bits));
+    p->fxp_b = (long long)std::nearbyint(std::ldexp(1.0 - (double)a->alpha, a->frac_bits));
+  }
   const long long budget = (kSmemOptin - 256 - (long long)select_smem_bytes(a->head_dim, P, 0, n_src)) /
                            ((long long)a->head_dim * 4 * n_src + 4);
   if (budget < 1) return fail(MPC_ERR_BAD_SHAPE, "%d candidates leave no shared memory to stage representatives", P);
@@ -496,8 +509,8 @@ MPC_API int mpc_select(const mpc_select_args* args, void* workspace, size_t work
   MPC_TRY(validate_select(args, &p));
   if (!args->q || !args->rep || !args->n_tok || !args->out_sel || !args->out_n_sel)
     return fail(MPC_ERR_INVALID_ARG, "a required pointer is NULL");
-  if (args->metric == MPC_SIM_BOUND && (!args->r_max || !args->r_min))
-    return fail(MPC_ERR_INVALID_ARG, "MPC_SIM_BOUND needs r_max and r_min");
+  if (select_n_src(args->metric) == 2 && (!args->r_max || !args->r_min))
+    return fail(MPC_ERR_INVALID_ARG, "MPC_SIM_BOUND and MPC_SIM_FXP need r_max and r_min");
   if (args->metric == MPC_SIM_MEAN && !args->mean) return fail(MPC_ERR_INVALID_ARG, "MPC_SIM_MEAN needs mean");
   const int units = args->n_refs * args->batch * args->n_kv_heads;
   const cudaError_t e = launch_select(p, args->dtype, args->head_dim, units, static_cast<cudaStream_t>(stream));

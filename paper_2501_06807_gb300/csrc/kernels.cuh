@@ -54,10 +54,12 @@ struct SelectParams {
   int max_cand;  // power of two, capacity of the shared candidate arrays
   int row_buf;   // candidates whose summary rows are staged in shared memory at once
   int spec_first;  // the first round also scores the whole level below the coarsest
-  int metric;      // MPC_SIM_EQ3: rep; MPC_SIM_BOUND: r_max and r_min; MPC_SIM_MEAN: mean
+  int metric;      // MPC_SIM_EQ3: rep; MPC_SIM_BOUND / _FXP: r_max and r_min; MPC_SIM_MEAN: mean
   const float* rmax;
   const float* rmin;
   const float* mean;
+  int frac_bits;           // MPC_SIM_FXP: fractional bits f
+  long long fxp_a, fxp_b;  // MPC_SIM_FXP: enc(alpha), enc(1 - alpha)
 };
 
 struct StaticParams {
@@ -132,6 +134,12 @@ struct ClusterParams {
   float alpha;
   int* out_n_tok;
 };
+
+// Summary rows staged per candidate by the select kernel: r_max and r_min for
+// the metrics that read both, else one (rep or mean).
+__host__ __device__ inline int select_n_src(int metric) {
+  return metric == MPC_SIM_BOUND || metric == MPC_SIM_FXP ? 2 : 1;
+}
 
 cudaError_t launch_attn(const AttnParams& p, int dtype, int D, int n_units, cudaStream_t st);
 int attn_smem_bytes(int dtype, int D, int G, int B);

@@ -6,6 +6,8 @@
 // levels are walked from the coarsest down.  Each candidate is held as one
 // 64-bit key (orderable score, inverted id: all keys distinct, larger score
 // first, then smaller id), so the key alone carries the id and the score.
+// The orderable score is the fp32 similarity's order-preserving bit pattern,
+// or, for the fixed-point metric, the int32 score with its sign bit flipped.
 //
 // The walk is bounded by global-load latency, so the fp32 representatives
 // a level needs are staged in shared memory by 1-D bulk copies (contiguous
@@ -32,20 +34,47 @@ constexpr int kRankMax = 1024;  // candidates ranked by counting
 
 constexpr int kSelChunk = 8192; // bytes per bulk copy
 
-__device__ __forceinline__ unsigned long long sel_key(float score, int id) {
-  return ((unsigned long long)orderable(score) << 32) | (unsigned long long)(0xffffffffu - (uint32_t)id);
+__device__ __forceinline__ unsigned long long sel_key(uint32_t oscore, int id) {
+  return ((unsigned long long)oscore << 32) | (unsigned long long)(0xffffffffu - (uint32_t)id);
+}
+
+// Fixed-point Eq. 3 (ring Z_{2^64}, f fractional bits) of four channels:
+// sum_j q_j rep_j with rep_j = tr(a enc(r_max_j)) + tr(b enc(r_min_j)), the
+// products and sums wrapping modulo 2^64; tr is the arithmetic shift by f.
+// x 2^f is exact in fp32, and the conversion rounds ties to even.
+__device__ __forceinline__ unsigned long long fxp_dot4(const long long (&q)[4], float4 mx, float4 mn, float sc,
+                                                       long long a, long long b, int f) {
+  const float x[4] = {mx.x, mx.y, mx.z, mx.w}, y[4] = {mn.x, mn.y, mn.z, mn.w};
+  unsigned long long acc = 0ull;
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const long long ex = __float2ll_rn(x[j] * sc), ey = __float2ll_rn(y[j] * sc);
+    const long long pa = (long long)((unsigned long long)a * (unsigned long long)ex) >> f;
+    const long long pb = (long long)((unsigned long long)b * (unsigned long long)ey) >> f;
+    const unsigned long long r = (unsigned long long)pa + (unsigned long long)pb;
+    acc += (unsigned long long)q[j] * r;
+  }
+  return acc;
+}
+
+// Orderable key of a truncated ring dot product: tr(acc) saturated to int32.
+__device__ __forceinline__ uint32_t fxp_oscore(unsigned long long acc, int f) {
+  long long v = (long long)acc >> f;
+  v = v > 2147483647ll ? 2147483647ll : (v < -2147483648ll ? -2147483648ll : v);
+  return (uint32_t)(int32_t)v ^ 0x80000000u;
 }
 __device__ __forceinline__ int key_id(unsigned long long key) {
   return (int)(0xffffffffu - (uint32_t)(key & 0xffffffffull));
 }
 
 // Shared-memory layout of one select CTA (host and device): n_src staged
-// row arrays (rep, or r_max and r_min), then the scalars.
+// row arrays (rep or mean, or r_max and r_min), then the summed query (fp32,
+// or int64 encodings for the fixed-point metric), then the scalars.
 struct SelLayout {
   size_t qsum, cs, keys, mark, kept, total;
   __host__ __device__ SelLayout(int D, int MC, int RB, int n_src) {
     qsum = (size_t)n_src * RB * D * 4;     // staged rows first (16-byte aligned)
-    cs = qsum + (size_t)D * 4;              // scores of the first round's children
+    cs = qsum + (size_t)D * 8;              // orderable scores of the first round's children
     keys = (cs + (size_t)RB * 4 + 15) & ~(size_t)15;
     mark = keys + (size_t)MC * 16;          // two key arrays
     kept = mark + (size_t)MC * 4;
@@ -62,7 +91,9 @@ __device__ __forceinline__ void warp_copy(void* dst, const void* src, uint32_t n
   }
 }
 
-template <typename T, int D, int NT>
+// FXP: the fixed-point metric (its own instantiation, so the fp32 metrics
+// keep their register budget).
+template <typename T, int D, int NT, bool FXP>
 __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ SelectParams p) {
   constexpr int NW = NT / 32;
   constexpr int LPR = D / 4;     // lanes per representative row (one float4 each)
@@ -72,11 +103,11 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   constexpr int kFastMax = 16 * NW;  // candidates ranked from registers (NW / 2 keys per lane)
   extern __shared__ __align__(128) uint8_t smem[];
   const int MC = p.max_cand, RB = p.row_buf;
-  const int NSRC = p.metric == MPC_SIM_BOUND ? 2 : 1;  // summary rows per candidate
+  const int NSRC = FXP ? 2 : select_n_src(p.metric);  // summary rows per candidate
   const SelLayout L(D, MC, RB, NSRC);
   float* rows = reinterpret_cast<float*>(smem);
   float* qsum = reinterpret_cast<float*>(smem + L.qsum);
-  float* cs = reinterpret_cast<float*>(smem + L.cs);
+  uint32_t* cs = reinterpret_cast<uint32_t*>(smem + L.cs);
   unsigned long long* keysA = reinterpret_cast<unsigned long long*>(smem + L.keys);
   unsigned long long* keysB = keysA + MC;
   int* mark = reinterpret_cast<int*>(smem + L.mark);
@@ -95,7 +126,8 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   const int top = p.pyr.n_levels - 1;
   const int64_t unit_off = ((int64_t)(group * p.B + b) * p.Hkv + h) * p.pyr.rows * D;
   // staged source w of a candidate: rep (Eq. 3) or mean (average key), or
-  // r_max then r_min (Eq. 2), each into its own RB-row array of the buffer
+  // r_max then r_min (Eq. 2, fixed-point Eq. 3), each into its own RB-row
+  // array of the buffer
   const float* one = p.metric == MPC_SIM_MEAN ? p.mean : p.rep;
   const float* src0[2] = {(NSRC == 2 ? p.rmax : one) + unit_off, (NSRC == 2 ? p.rmin : one) + unit_off};
   int* out = p.out_sel + ((int64_t)(group * p.B + b) * p.Hkv + h) * p.sel_cap;
@@ -103,45 +135,76 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   bool timed_out = false;
 
   // similarity of staged row r for rows [0, nrows) of the buffer;
-  // put(r, score) runs on the first lane of each row.  Channel order is
-  // fixed: x, y, z, w per lane, then a butterfly over the row's lanes.
-  //   Eq. 3: q_sum . rep;  mean: q_sum . mean;  Eq. 2: sum_i max(q_i r_max_i, q_i r_min_i)
+  // put(r, orderable score) runs on the first lane of each row.  Channel
+  // order is fixed: x, y, z, w per lane, then a butterfly over the row's lanes.
+  //   Eq. 3: q_sum . rep;  mean: q_sum . mean;  Eq. 2: sum_i max(q_i r_max_i, q_i r_min_i);
+  //   fixed point: integer, so the order of the ring sums does not matter
   auto score_rows = [&](int nrows, auto&& put) {
-    const float4 qv = reinterpret_cast<const float4*>(qsum)[c4];
     const float* rows2 = rows + (size_t)RB * D;
-    for (int r0 = warp * U * RPW; r0 < nrows; r0 += NW * U * RPW) {
-      float acc[U];
-#pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int r = r0 + u * RPW + sub;
-        const float4 v = r < nrows ? reinterpret_cast<const float4*>(rows + (size_t)r * D)[c4]
-                                   : make_float4(0.f, 0.f, 0.f, 0.f);
-        float a = 0.f;
-        if (NSRC == 1) {
-          a = fmaf(v.x, qv.x, a);
-          a = fmaf(v.y, qv.y, a);
-          a = fmaf(v.z, qv.z, a);
-          a = fmaf(v.w, qv.w, a);
-        } else {
-          const float4 m = r < nrows ? reinterpret_cast<const float4*>(rows2 + (size_t)r * D)[c4]
-                                     : make_float4(0.f, 0.f, 0.f, 0.f);
-          a += fmaxf(qv.x * v.x, qv.x * m.x);
-          a += fmaxf(qv.y * v.y, qv.y * m.y);
-          a += fmaxf(qv.z * v.z, qv.z * m.z);
-          a += fmaxf(qv.w * v.w, qv.w * m.w);
-        }
-        acc[u] = a;
-      }
-#pragma unroll
-      for (int o = LPR / 2; o > 0; o >>= 1) {
-#pragma unroll
-        for (int u = 0; u < U; ++u) acc[u] += __shfl_xor_sync(0xffffffffu, acc[u], o);
-      }
-      if (c4 == 0) {
+    if constexpr (FXP) {
+      const long long* qf = reinterpret_cast<const long long*>(qsum) + c4 * 4;
+      const long long qx[4] = {qf[0], qf[1], qf[2], qf[3]};
+      const int fb = p.frac_bits;
+      const float sc = (float)(1 << fb);
+      const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int r0 = warp * U * RPW; r0 < nrows; r0 += NW * U * RPW) {
+        unsigned long long acc[U];
 #pragma unroll
         for (int u = 0; u < U; ++u) {
           const int r = r0 + u * RPW + sub;
-          if (r < nrows) put(r, acc[u]);
+          const float4 v = r < nrows ? reinterpret_cast<const float4*>(rows + (size_t)r * D)[c4] : z;
+          const float4 m = r < nrows ? reinterpret_cast<const float4*>(rows2 + (size_t)r * D)[c4] : z;
+          acc[u] = fxp_dot4(qx, v, m, sc, p.fxp_a, p.fxp_b, fb);
+        }
+#pragma unroll
+        for (int o = LPR / 2; o > 0; o >>= 1) {
+#pragma unroll
+          for (int u = 0; u < U; ++u) acc[u] += __shfl_xor_sync(0xffffffffu, acc[u], o);
+        }
+        if (c4 == 0) {
+#pragma unroll
+          for (int u = 0; u < U; ++u) {
+            const int r = r0 + u * RPW + sub;
+            if (r < nrows) put(r, fxp_oscore(acc[u], fb));
+          }
+        }
+      }
+    } else {
+      const float4 qv = reinterpret_cast<const float4*>(qsum)[c4];
+      for (int r0 = warp * U * RPW; r0 < nrows; r0 += NW * U * RPW) {
+        float acc[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          const int r = r0 + u * RPW + sub;
+          const float4 v = r < nrows ? reinterpret_cast<const float4*>(rows + (size_t)r * D)[c4]
+                                     : make_float4(0.f, 0.f, 0.f, 0.f);
+          float a = 0.f;
+          if (NSRC == 1) {
+            a = fmaf(v.x, qv.x, a);
+            a = fmaf(v.y, qv.y, a);
+            a = fmaf(v.z, qv.z, a);
+            a = fmaf(v.w, qv.w, a);
+          } else {
+            const float4 m = r < nrows ? reinterpret_cast<const float4*>(rows2 + (size_t)r * D)[c4]
+                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+            a += fmaxf(qv.x * v.x, qv.x * m.x);
+            a += fmaxf(qv.y * v.y, qv.y * m.y);
+            a += fmaxf(qv.z * v.z, qv.z * m.z);
+            a += fmaxf(qv.w * v.w, qv.w * m.w);
+          }
+          acc[u] = a;
+        }
+#pragma unroll
+        for (int o = LPR / 2; o > 0; o >>= 1) {
+#pragma unroll
+          for (int u = 0; u < U; ++u) acc[u] += __shfl_xor_sync(0xffffffffu, acc[u], o);
+        }
+        if (c4 == 0) {
+#pragma unroll
+          for (int u = 0; u < U; ++u) {
+            const int r = r0 + u * RPW + sub;
+            if (r < nrows) put(r, orderable(acc[u]));
+          }
         }
       }
     }
@@ -181,12 +244,22 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
     }
   }
 
-  // q_sum = sum over the group's query heads (fixed order)
+  // q_sum = sum over the group's query heads (fixed order); fixed point:
+  // the ring sum of the heads' encodings
   const T* qp = (const T*)p.q + layer * p.q_ls + ((int64_t)b * p.Hq + h * G) * D;
-  for (int c = tid; c < D; c += NT) {
-    float acc = 0.f;
-    for (int g = 0; g < G; ++g) acc += to_float<T>(qp[g * D + c]);
-    qsum[c] = acc;
+  if constexpr (FXP) {
+    const float sc = (float)(1 << p.frac_bits);
+    for (int c = tid; c < D; c += NT) {
+      unsigned long long acc = 0ull;
+      for (int g = 0; g < G; ++g) acc += (unsigned long long)__float2ll_rn(to_float<T>(qp[g * D + c]) * sc);
+      reinterpret_cast<long long*>(qsum)[c] = (long long)acc;
+    }
+  } else {
+    for (int c = tid; c < D; c += NT) {
+      float acc = 0.f;
+      for (int g = 0; g < G; ++g) acc += to_float<T>(qp[g * D + c]);
+      qsum[c] = acc;
+    }
   }
   if (tid < kMaxLevels) {
     s_C[tid] = C[tid];
@@ -200,7 +273,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   {
     const int nC = top > 0 ? C[top - 1] : 0;
     const int own = n < nT0 ? n : nT0;
-    score_rows(spec0 ? capT + nC : own, [&](int r, float sc) {
+    score_rows(spec0 ? capT + nC : own, [&](int r, uint32_t sc) {
       if (r < own) keysA[r] = sel_key(sc, r);
       else if (r >= capT) cs[r - capT] = sc;
     });
@@ -215,7 +288,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
           warp_copy(rows + (size_t)w * RB * D, src0[w] + offT + (int64_t)x0 * D, (uint32_t)nb * ROWB, &s_bar, lane);
       }
       wait_rows();
-      score_rows(nb, [&](int r, float sc) { keysA[x0 + r] = sel_key(sc, x0 + r); });
+      score_rows(nb, [&](int r, uint32_t sc) { keysA[x0 + r] = sel_key(sc, x0 + r); });
       __syncthreads();
     }
   }
@@ -245,7 +318,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
           }
         }
         wait_rows();
-        score_rows(x1 - x0, [&](int r, float sc) { keysA[x0 + r] = sel_key(sc, key_id(keysA[x0 + r])); });
+        score_rows(x1 - x0, [&](int r, uint32_t sc) { keysA[x0 + r] = sel_key(sc, key_id(keysA[x0 + r])); });
         __syncthreads();
       }
     }
@@ -301,7 +374,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
         } else {
           for (int j = lane; j < f; j += 32) {
             const int cid = id * f + j;
-            if (cid < nC) keysB[pos * f + j] = have_child ? sel_key(cs[i * f + j], cid) : sel_key(0.f, cid);
+            if (cid < nC) keysB[pos * f + j] = have_child ? sel_key(cs[i * f + j], cid) : sel_key(0u, cid);
           }
         }
       }
@@ -422,7 +495,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
       const int kk = x / f, j = x - kk * f;
       const int i = kept[kk];
       const int id = key_id(keysA[i]) * f + j;
-      keysB[x] = have_child ? sel_key(cs[i * f + j], id) : sel_key(0.f, id);
+      keysB[x] = have_child ? sel_key(cs[i * f + j], id) : sel_key(0u, id);
     }
     need_score = !have_child;
     have_child = false;
@@ -462,13 +535,15 @@ static cudaError_t launch_sel(K kernel, int units, int nt, int smem, cudaStream_
 }
 
 cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cudaStream_t st) {
-  const int smem = select_smem_bytes(D, p.max_cand, p.row_buf, p.metric == MPC_SIM_BOUND ? 2 : 1);
-  const int nt = select_threads(units);
-#define MPC_SEL(TT, DD)                                                                     \
-  if (D == DD) {                                                                            \
-    if (nt == 512) return launch_sel(select_kernel<TT, DD, 512>, units, nt, smem, st, p);  \
-    if (nt == 256) return launch_sel(select_kernel<TT, DD, 256>, units, nt, smem, st, p);  \
-    return launch_sel(select_kernel<TT, DD, 128>, units, nt, smem, st, p);                 \
+  const int smem = select_smem_bytes(D, p.max_cand, p.row_buf, select_n_src(p.metric));
+  // the fixed-point metric is a diagnostic path: one thread count
+  const int nt = p.metric == MPC_SIM_FXP ? 256 : select_threads(units);
+#define MPC_SEL(TT, DD)                                                                            \
+  if (D == DD) {                                                                                   \
+    if (p.metric == MPC_SIM_FXP) return launch_sel(select_kernel<TT, DD, 256, true>, units, nt, smem, st, p); \
+    if (nt == 512) return launch_sel(select_kernel<TT, DD, 512, false>, units, nt, smem, st, p);  \
+    if (nt == 256) return launch_sel(select_kernel<TT, DD, 256, false>, units, nt, smem, st, p);  \
+    return launch_sel(select_kernel<TT, DD, 128, false>, units, nt, smem, st, p);                 \
   }
   if (dtype == MPC_BF16) {
     MPC_SEL(bf16, 64)

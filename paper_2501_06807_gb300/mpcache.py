@@ -25,9 +25,10 @@ from . import build as _build
 
 MPC_OK, MPC_ERR_INVALID_ARG, MPC_ERR_BAD_SHAPE, MPC_ERR_WORKSPACE, MPC_ERR_CUDA = 0, -1, -2, -3, -4
 MPC_F32, MPC_BF16 = 0, 1
-MPC_SIM_EQ3, MPC_SIM_BOUND, MPC_SIM_MEAN = 0, 1, 2
+MPC_SIM_EQ3, MPC_SIM_BOUND, MPC_SIM_MEAN, MPC_SIM_FXP = 0, 1, 2, 3
+FXP_FRAC_BITS = 18
 MAX_LEVELS = 4
-ABI_VERSION = 4
+ABI_VERSION = 5
 MAX_REFS = 128
 PPM = 1_000_000
 
@@ -73,7 +74,8 @@ class SelectArgs(C.Structure):
                 ("n_levels", C.c_int32), ("fanout", C.c_int32 * MAX_LEVELS),
                 ("level_keep_ppm", C.c_int32 * MAX_LEVELS), ("sel_cap", C.c_int32),
                 ("out_sel", C.c_void_p), ("out_n_sel", C.c_void_p), ("metric", C.c_int32),
-                ("r_max", C.c_void_p), ("r_min", C.c_void_p), ("mean", C.c_void_p)]
+                ("r_max", C.c_void_p), ("r_min", C.c_void_p), ("mean", C.c_void_p),
+                ("alpha", C.c_float), ("frac_bits", C.c_int32)]
 
 
 class CommonalityArgs(C.Structure):
@@ -387,10 +389,11 @@ class Engine:
         self.build_clusters(k, v, page_table, page_size)
 
     # ---------------------------------------------------------- decode ----
-    def select(self, q: torch.Tensor, metric: int = MPC_SIM_EQ3):
+    def select(self, q: torch.Tensor, metric: int = MPC_SIM_EQ3, frac_bits: int = FXP_FRAC_BITS):
         """q: [L][B][Hq][d] queries of this step (only the leaders' are read);
-        metric MPC_SIM_EQ3 (Eq. 3 with rep), MPC_SIM_BOUND (Eq. 2 bound) or
-        MPC_SIM_MEAN (mean member key)."""
+        metric MPC_SIM_EQ3 (Eq. 3 with rep), MPC_SIM_BOUND (Eq. 2 bound),
+        MPC_SIM_MEAN (mean member key) or MPC_SIM_FXP (Eq. 3 in the
+        fixed-point ring with ``frac_bits`` fractional bits and the cache's alpha)."""
         lib = load()
         refs = _refs(self.refs_lead)
         a = SelectArgs()
@@ -404,6 +407,7 @@ class Engine:
         a.level_keep_ppm = _fan(self.level_keep_ppm)
         a.sel_cap, a.out_sel, a.out_n_sel = self.sel_cap, _ptr(self.sel), _ptr(self.n_sel)
         a.metric, a.r_max, a.r_min, a.mean = metric, _ptr(self.rmax), _ptr(self.rmin), _ptr(self.mean)
+        a.alpha, a.frac_bits = self.alpha, frac_bits
         _check(lib.mpc_select(C.byref(a), None, 0, C.c_void_p(_stream())))
 
     def attn_args(self, q, k_new, v_new, advance=True, refs_list=None, out=None) -> AttnArgs:

@@ -33,7 +33,7 @@ def test_exports_every_declared_symbol(lib):
                          capture_output=True, text=True).stdout
     exported = set(re.findall(r"\b(mpc_\w+)\b", out))
     assert set(names) <= exported
-    assert lib.mpc_abi_version() == mpcache.ABI_VERSION == 4
+    assert lib.mpc_abi_version() == mpcache.ABI_VERSION == 5
 
 
 def test_struct_layout_matches_c(tmp_path):
@@ -134,6 +134,16 @@ def test_select_and_static_validation(lib):
     assert _ws(lib, "mpc_select_workspace_size", s) == (0, 0)
     s.q, s.n_tok, s.out_sel, s.out_n_sel, s.r_min = 8192, 8192, 8192, 8192, None
     assert lib.mpc_select(C.byref(s), None, 0, None) == mpcache.MPC_ERR_INVALID_ARG  # bound needs r_min
+    # the fixed-point metric reads r_max and r_min and checks alpha and f
+    s.metric, s.r_min, s.alpha, s.frac_bits = mpcache.MPC_SIM_FXP, 8192, 0.6, 18
+    assert _ws(lib, "mpc_select_workspace_size", s) == (0, 0)
+    for alpha, fb in ((1.5, 18), (-0.1, 18), (float("nan"), 18), (0.6, 0), (0.6, 25)):
+        s.alpha, s.frac_bits = alpha, fb
+        assert _ws(lib, "mpc_select_workspace_size", s)[0] == mpcache.MPC_ERR_BAD_SHAPE, (alpha, fb)
+    s.alpha, s.frac_bits, s.r_max = 0.6, 24, 4100
+    assert _ws(lib, "mpc_select_workspace_size", s)[0] == mpcache.MPC_ERR_INVALID_ARG  # misaligned
+    s.r_max, s.r_min = 4096, None
+    assert lib.mpc_select(C.byref(s), None, 0, None) == mpcache.MPC_ERR_INVALID_ARG  # needs r_min
     s.metric, s.r_max, s.r_min, s.q, s.n_tok, s.out_sel, s.out_n_sel = mpcache.MPC_SIM_EQ3, None, None, None, None, None, None
     s.sel_cap = 3
     assert _ws(lib, "mpc_select_workspace_size", s)[0] == mpcache.MPC_ERR_BAD_SHAPE

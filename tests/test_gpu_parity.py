@@ -252,6 +252,98 @@ def _check_selection(dtype, d, Hq, Hkv, s, fan, keep, N, B, metric, alpha):
     assert ties <= max(1, 3 * B * Hkv // 100)
 
 
+@pytest.mark.parametrize("frac_bits", [18, 5])
+@pytest.mark.parametrize("dtype,d,Hq,Hkv,s,fan,keep,N,B", SELECT_CASES)
+def test_selection_fixed_point(dtype, d, Hq, Hkv, s, fan, keep, N, B, frac_bits):
+    _check_selection_fxp(dtype, d, Hq, Hkv, s, fan, keep, N, B, frac_bits, 1.0)
+
+
+def test_selection_fixed_point_ring_wraps():
+    # f = 24 and large values: the ring sums leave the int64 range and wrap
+    # modulo 2^64 on both sides
+    _check_selection_fxp(torch.bfloat16, 128, 4, 1, 16, (4,), (125_000, 500_000), 1024, 2, 24, 60.0, wraps=True)
+
+
+def _check_selection_fxp(dtype, d, Hq, Hkv, s, fan, keep, N, B, frac_bits, scale, wraps=False):
+    """Eq. 3 in the fixed-point ring: integer scores, so the selection is
+    bit-exact (equal scores rank the lower id first on both sides)."""
+    g = torch.Generator().manual_seed(N + d + frac_bits)
+    G = Hq // Hkv
+    alpha = float(np.float32(0.6))
+    eng = H.make_engine(synth.Workload("t", 1, B, Hq, Hkv, d, "f32" if dtype == torch.float32 else "bf16",
+                                       N, N, O.PPM, s, fan, keep, 1, 4, "iid"), 4)
+    drift = torch.cumsum(torch.randn((1, B, Hkv, N, d), generator=g) * 0.15, dim=3)
+    K = ((torch.randn((1, B, Hkv, N, d), generator=g) + drift)
+         * torch.rand((1, 1, Hkv, 1, d), generator=g) * 3 * scale).to(dtype)
+    eng.kept[..., :N] = torch.arange(N, dtype=torch.int32).cuda()
+    eng.n_keep.fill_(N)
+    eng.build_clusters(K.cuda(), K.cuda())
+    wrapped = False
+    for rep_i in range(3):
+        q = (torch.randn((1, B, Hq, d), generator=g) * 2 * scale).to(dtype)
+        eng.select(q.cuda(), mpcache.MPC_SIM_FXP, frac_bits)
+        sel = eng.sel.cpu().numpy()
+        n_sel = eng.n_sel.cpu().numpy()
+        for b in range(B):
+            for h in range(Hkv):
+                levels = O.cluster_pyramid(K[0, b, h].double().numpy(), s, fan, alpha)
+                qg = q[0, b, h * G:(h + 1) * G].double().numpy()
+                ref = O.hierarchical_select(qg, levels, fan, keep, metric="fxp", alpha=alpha, frac_bits=frac_bits)
+                assert n_sel[b] == len(ref)
+                assert np.array_equal(sel[0, b, h, :n_sel[b]], ref), (b, h)
+                assert (sel[0, b, h, n_sel[b]:] == -1).all()
+                if wraps:
+                    qs = O.fxp_encode(qg, frac_bits).sum(0).astype(object)
+                    rep = levels[0].r_max[0] * alpha + levels[0].r_min[0] * (1 - alpha)
+                    wrapped |= abs(int(sum(qs * O.fxp_encode(rep, frac_bits).astype(object)))) >= 2 ** 63
+    assert wrapped or not wraps
+
+
+def test_fixed_point_ranking_survives_on_needle_workload():
+    """Eq. 3 in the fixed-point ring at the default 18 fractional bits, on the
+    needle workload (three-level pyramid, GQA): the selections equal the fp32
+    ones almost everywhere, and every cluster of the needle passage that the
+    fp32 selection keeps is kept.  Coarser encodings are reported alongside."""
+    w = synth.C5.replace(n_layers=3, prompt_len=4096, prompt_len_min=4096, n_q_heads=8, n_kv_heads=2,
+                         level_keep_ppm=(100_000, 250_000, 500_000))
+    E = 12
+    x = synth.generate(w, H.window_rows_for(w), device="cpu", decode_steps=E)
+    xc = H.to_cuda(x)
+    eng = H.make_engine(w, E)
+    eng.prefill(xc.k, xc.v, xc.q_win, x.prompt_lens.cuda(), None, w.page_size)
+    kept = eng.kept.cpu().numpy()
+    same = {18: 0, 8: 0, 5: 0, 3: 0}
+    units = needles = needles_kept = 0
+    for e in range(E):
+        eng.select(xc.q[e])
+        ref = eng.sel.cpu().numpy().copy()
+        for fb in same:
+            eng.select(xc.q[e], mpcache.MPC_SIM_FXP, fb)
+            got = eng.sel.cpu().numpy()
+            same[fb] += int((got == ref).all(axis=-1).sum())
+            if fb != 18:
+                continue
+            for lead in eng.leaders:
+                grp = eng.group_of[lead]
+                for b in range(w.batch):
+                    for h in range(w.n_kv_heads):
+                        p0 = int(x.needle_pos[lead, b, h])
+                        pos = kept[grp, b, h]
+                        hit = np.nonzero((pos >= p0) & (pos < p0 + w.needle_len))[0]
+                        clusters = set((hit // w.cluster_size).tolist())
+                        want = clusters & set(ref[grp, b, h].tolist())
+                        needles += len(want)
+                        needles_kept += len(want & set(got[grp, b, h].tolist()))
+        units += ref.shape[0] * ref.shape[1] * ref.shape[2]
+        eng.decode_step(xc.q[e], xc.k_new[e], xc.v_new[e])
+    frac = {fb: same[fb] / units for fb in same}
+    print("identical selections (fraction of units) by fractional bits:", frac,
+          "needle clusters kept:", needles_kept, "/", needles)
+    assert needles > 0 and needles_kept == needles
+    assert frac[18] >= 0.95
+    assert mpcache.device_status() == 0
+
+
 # ----------------------------------------------- static eviction alone ----
 
 STATIC_CASES = [
