@@ -636,16 +636,32 @@ __global__ void __launch_bounds__(WPC * 32, 1) attn_bf16_persist_kernel(const __
           p.unit_counter[unit_id] = 0;
         }
         __syncwarp();
+        // the records of warps gw + 1 .. gw + nother are contiguous: copy
+        // them into this warp's ring (idle: the owner piece ends the warp's
+        // range, after its last tile) with one batch of copies in flight,
+        // instead of one dependent round trip per record
+        const int rec = G * (D + 4);
+        const float* recs = p.part + (int64_t)(gw + 1) * rec;
+        const bool staged = nother * rec * 4 <= NST * STAGE;
+        auto ld_rec = [&](const float* a) { return staged ? *a : __ldcg(a); };
+        if (staged) {
+          const uint8_t* src = reinterpret_cast<const uint8_t*>(recs);
+          for (int i = lane; i < nother * rec / 4; i += 32) cp_async16(ring + i * 16, src + i * 16);
+          cp_async_commit();
+          cp_async_wait<0>();
+          __syncwarp();
+          recs = reinterpret_cast<const float*>(ring);
+        }
         for (int k = 1; k <= nother; ++k) {
-          const float* rec = p.part + (int64_t)(gw + k) * G * (D + 4);
+          const float* rec_k = recs + (int64_t)(k - 1) * rec;
 #pragma unroll
           for (int hn = 0; hn < HN; ++hn)
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
               const int g = hn * 8 + h_off + e;
               if (g < G) {
-                const float* rg = rec + g * (D + 4);
-                const float mk = __ldcg(rg), lk = __ldcg(rg + 1);
+                const float* rg = rec_k + g * (D + 4);
+                const float mk = ld_rec(rg), lk = ld_rec(rg + 1);
                 const float M = fmaxf(m_run[hn][e], mk);
                 const float wa = (m_run[hn][e] == kNegInf) ? 0.f : fast_exp2(m_run[hn][e] - M);
                 const float wb = (mk == kNegInf) ? 0.f : fast_exp2(mk - M);
@@ -653,8 +669,8 @@ __global__ void __launch_bounds__(WPC * 32, 1) attn_bf16_persist_kernel(const __
                 lq[hn][e] = lq[hn][e] * wa + lk * wb;
 #pragma unroll
                 for (int mt = 0; mt < KS; ++mt) {
-                  o[mt][hn][e] = o[mt][hn][e] * wa + wb * __ldcg(rg + 4 + mt * 16 + r_tok);
-                  o[mt][hn][2 + e] = o[mt][hn][2 + e] * wa + wb * __ldcg(rg + 4 + mt * 16 + r_tok + 8);
+                  o[mt][hn][e] = o[mt][hn][e] * wa + wb * ld_rec(rg + 4 + mt * 16 + r_tok);
+                  o[mt][hn][2 + e] = o[mt][hn][2 + e] * wa + wb * ld_rec(rg + 4 + mt * 16 + r_tok + 8);
                 }
               }
             }

@@ -101,6 +101,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   constexpr int U = 8;           // rows per lane per pass
   constexpr uint32_t ROWB = D * 4;
   constexpr int kFastMax = 16 * NW;  // candidates ranked from registers (NW / 2 keys per lane)
+  constexpr int kWarpMax = 32;       // candidates ranked by warp 0 alone (one per lane)
   extern __shared__ __align__(128) uint8_t smem[];
   const int MC = p.max_cand, RB = p.row_buf;
   const int NSRC = FXP ? 2 : select_n_src(p.metric);  // summary rows per candidate
@@ -115,6 +116,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   __shared__ __align__(8) uint64_t s_bar;
   __shared__ int s_C[kMaxLevels], s_k[kMaxLevels];
   __shared__ int s_nk, s_next;
+  __shared__ int s_walk[4];  // warp walk: level reached, candidates, kept, flags
   __shared__ uint32_t s_wmask[NW];
 
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -135,8 +137,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   bool timed_out = false;
 
   // similarity of staged row r for rows [0, nrows) of the buffer;
-  // put(r, orderable score) runs on the first lane of each row.  Channel
-  // order is fixed: x, y, z, w per lane, then a butterfly over the row's lanes.
+  // put(r, orderable score) runs on one lane of each row.
   //   Eq. 3: q_sum . rep;  mean: q_sum . mean;  Eq. 2: sum_i max(q_i r_max_i, q_i r_min_i);
   //   fixed point: integer, so the order of the ring sums does not matter
   auto score_rows = [&](int nrows, auto&& put) {
@@ -170,42 +171,43 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
         }
       }
     } else {
-      const float4 qv = reinterpret_cast<const float4*>(qsum)[c4];
-      for (int r0 = warp * U * RPW; r0 < nrows; r0 += NW * U * RPW) {
-        float acc[U];
+      // 4 lanes per row, each with a quarter of the channels and that
+      // quarter of q in registers: chunk ql + 4 ((j + rot) % V4) of the row
+      // for j < V4, rotated by the row's parity so that the 32 lanes of a
+      // read hit 8 distinct 16-byte bank groups (4 wavefronts, the minimum)
+      constexpr int V4 = D / 16;  // float4 chunks per lane
+      const int ql = lane & 3, rs = lane >> 2, rot = rs & 1;
+      float4 qv[V4];
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
-          const int r = r0 + u * RPW + sub;
-          const float4 v = r < nrows ? reinterpret_cast<const float4*>(rows + (size_t)r * D)[c4]
-                                     : make_float4(0.f, 0.f, 0.f, 0.f);
-          float a = 0.f;
-          if (NSRC == 1) {
-            a = fmaf(v.x, qv.x, a);
-            a = fmaf(v.y, qv.y, a);
-            a = fmaf(v.z, qv.z, a);
-            a = fmaf(v.w, qv.w, a);
-          } else {
-            const float4 m = r < nrows ? reinterpret_cast<const float4*>(rows2 + (size_t)r * D)[c4]
-                                       : make_float4(0.f, 0.f, 0.f, 0.f);
-            a += fmaxf(qv.x * v.x, qv.x * m.x);
-            a += fmaxf(qv.y * v.y, qv.y * m.y);
-            a += fmaxf(qv.z * v.z, qv.z * m.z);
-            a += fmaxf(qv.w * v.w, qv.w * m.w);
-          }
-          acc[u] = a;
-        }
+      for (int jj = 0; jj < V4; ++jj) qv[jj] = reinterpret_cast<const float4*>(qsum)[ql + 4 * ((jj + rot) % V4)];
+      for (int r0 = warp * 8; r0 < nrows; r0 += NW * 8) {
+        const int r = r0 + rs;
+        float ax = 0.f, ay = 0.f, az = 0.f, aw = 0.f;
+        if (r < nrows) {
+          const float4* rp = reinterpret_cast<const float4*>(rows + (size_t)r * D);
+          const float4* rp2 = reinterpret_cast<const float4*>(rows2 + (size_t)r * D);
 #pragma unroll
-        for (int o = LPR / 2; o > 0; o >>= 1) {
-#pragma unroll
-          for (int u = 0; u < U; ++u) acc[u] += __shfl_xor_sync(0xffffffffu, acc[u], o);
-        }
-        if (c4 == 0) {
-#pragma unroll
-          for (int u = 0; u < U; ++u) {
-            const int r = r0 + u * RPW + sub;
-            if (r < nrows) put(r, orderable(acc[u]));
+          for (int jj = 0; jj < V4; ++jj) {
+            const int c = ql + 4 * ((jj + rot) % V4);
+            const float4 v = rp[c];
+            if (NSRC == 1) {
+              ax = fmaf(v.x, qv[jj].x, ax);
+              ay = fmaf(v.y, qv[jj].y, ay);
+              az = fmaf(v.z, qv[jj].z, az);
+              aw = fmaf(v.w, qv[jj].w, aw);
+            } else {
+              const float4 m = rp2[c];
+              ax += fmaxf(qv[jj].x * v.x, qv[jj].x * m.x);
+              ay += fmaxf(qv[jj].y * v.y, qv[jj].y * m.y);
+              az += fmaxf(qv[jj].z * v.z, qv[jj].z * m.z);
+              aw += fmaxf(qv[jj].w * v.w, qv[jj].w * m.w);
+            }
           }
         }
+        float a = (ax + ay) + (az + aw);
+        a += __shfl_xor_sync(0xffffffffu, a, 1);
+        a += __shfl_xor_sync(0xffffffffu, a, 2);
+        if (ql == 0 && r < nrows) put(r, orderable(a));
       }
     }
   };
@@ -221,28 +223,28 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   grid_dep_launch();
   grid_dep_wait();
 
-  // ---- first round, requested as soon as the token count is known: the
-  // clusters [0, nT) of the coarsest level at buffer row 0 and, when spec0,
-  // all clusters of the level below it at buffer row capT
+  // ---- first round, requested before the token count arrives: the
+  // capacity rows [0, nT0) of the coarsest level at buffer row 0 and, when
+  // spec0, the capacity of the level below it at buffer row capT (rows past
+  // the live clusters are copied and never scored)
   const int capT = p.pyr.cap[top];
   const int capC = top > 0 ? p.pyr.cap[top - 1] : 0;
   const bool spec0 = p.spec_first && top > 0 && capT + capC <= RB;
   const int nT0 = capT < RB ? capT : RB;
   const int64_t offT = (int64_t)p.pyr.off[top] * D;
   const int64_t offC = (int64_t)(top > 0 ? p.pyr.off[top - 1] : 0) * D;
-  const int ntok = p.n_tok[b];
-  int C[kMaxLevels];
-  level_counts(p.pyr, ntok, C);
   if (warp == 0) {
-    const int nT = max(0, min(C[top], nT0));
-    const int nCc = spec0 ? max(0, min(C[top - 1], capC)) : 0;
-    if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)(nT + nCc) * ROWB * NSRC);
+    const int nCc = spec0 ? capC : 0;
+    if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)(nT0 + nCc) * ROWB * NSRC);
     __syncwarp();
     for (int w = 0; w < NSRC; ++w) {
-      warp_copy(rows + (size_t)w * RB * D, src0[w] + offT, (uint32_t)nT * ROWB, &s_bar, lane);
+      warp_copy(rows + (size_t)w * RB * D, src0[w] + offT, (uint32_t)nT0 * ROWB, &s_bar, lane);
       if (nCc > 0) warp_copy(rows + ((size_t)w * RB + capT) * D, src0[w] + offC, (uint32_t)nCc * ROWB, &s_bar, lane);
     }
   }
+  const int ntok = p.n_tok[b];
+  int C[kMaxLevels];
+  level_counts(p.pyr, ntok, C);
 
   // q_sum = sum over the group's query heads (fixed order); fixed point:
   // the ring sum of the heads' encodings
@@ -294,6 +296,23 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   }
   bool have_child = spec0;  // cs holds the scores of all children of keysA[0, n)
   bool need_score = false;  // keysA holds ids only
+  bool issued = false;      // the first batch of the scoring round is already requested
+
+  // Requests the rows of candidates [x0, x1) of level l (keys in kk):
+  // children of kept clusters of level l + 1, so every run of fl
+  // consecutive candidates is one run of rows.  Warp 0 only.
+  auto request_rows = [&](const unsigned long long* kk, int l, int x0, int x1) {
+    const int fl = p.pyr.fanout[l];
+    const int64_t offL = (int64_t)p.pyr.off[l] * D;
+    if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)(x1 - x0) * ROWB * NSRC);
+    __syncwarp();
+    for (int c = x0 / fl + lane; c * fl < x1; c += 32) {
+      const int s0 = max(x0, c * fl), s1 = min(x1, c * fl + fl);
+      for (int w = 0; w < NSRC; ++w)
+        bulk_g2s(rows + ((size_t)w * RB + (s0 - x0)) * D, src0[w] + offL + (int64_t)key_id(kk[s0]) * D,
+                 (uint32_t)(s1 - s0) * ROWB, &s_bar);
+    }
+  };
 
   int nk = 0;
   for (int l = top; l >= 0 && !overflow; --l) {
@@ -303,27 +322,105 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
       // a round over the candidates' own rows, in batches of RB rows; the
       // candidates are the children of the kept clusters of level l + 1, so
       // every run of fl consecutive candidates is one run of rows
-      const int fl = p.pyr.fanout[l];
-      const int64_t offL = (int64_t)p.pyr.off[l] * D;
       for (int x0 = 0; x0 < n; x0 += RB) {
         const int x1 = min(n, x0 + RB);
-        if (warp == 0) {
-          if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)(x1 - x0) * ROWB * NSRC);
-          __syncwarp();
-          for (int kk = x0 / fl + lane; kk * fl < x1; kk += 32) {
-            const int s0 = max(x0, kk * fl), s1 = min(x1, kk * fl + fl);
-            for (int w = 0; w < NSRC; ++w)
-              bulk_g2s(rows + ((size_t)w * RB + (s0 - x0)) * D, src0[w] + offL + (int64_t)key_id(keysA[s0]) * D,
-                       (uint32_t)(s1 - s0) * ROWB, &s_bar);
-          }
-        }
+        if (warp == 0 && !(x0 == 0 && issued)) request_rows(keysA, l, x0, x1);
         wait_rows();
         score_rows(x1 - x0, [&](int r, uint32_t sc) { keysA[x0 + r] = sel_key(sc, key_id(keysA[x0 + r])); });
         __syncthreads();
       }
+      issued = false;
     }
 
     const int k = min(s_k[l], n);
+    if (n <= kWarpMax) {
+      // warp 0 ranks this level, expands the kept clusters, and goes on
+      // down while the next level's scores are known and its candidates
+      // fit, with no block barrier; it stops at level 0, or before a level
+      // whose rows must be scored (it then requests their first batch)
+      if (warp == 0) {
+        const unsigned lt = (1u << lane) - 1u;
+        unsigned long long* ka = keysA;
+        unsigned long long* kb = keysB;
+        int lw = l, nw = n, nkw = 0, flags = 0;  // flags: 1 need_score, 2 overflow, 4 swapped, 8 done
+        bool hc = have_child;
+        while (true) {
+          const int kl = min(s_k[lw], nw);
+          const int fw = lw > 0 ? p.pyr.fanout[lw - 1] : 1;
+          const int nCw = lw > 0 ? s_C[lw - 1] : 0;
+          // rank from registers: lane i holds candidate i; the keys of the
+          // other lanes arrive by shuffle (all 32 independent, no memory)
+          const unsigned long long ki = lane < nw ? ka[lane] : 0ull;
+          int cnt = 0;
+          if (kl < nw) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) cnt += (int)(__shfl_sync(0xffffffffu, ki, j) > ki);
+          }
+          const bool keep = lane < nw && cnt < kl;
+          const unsigned bal = __ballot_sync(0xffffffffu, keep);
+          if (keep) {
+            const int pos = __popc(bal & lt);
+            const int id = key_id(ki);
+            if (lw == 0) {
+              if (pos < p.sel_cap) out[pos] = id;
+            } else {
+              for (int j = 0; j < fw; ++j) {
+                const int cid = id * fw + j;
+                if (cid < nCw) kb[pos * fw + j] = hc ? sel_key(cs[lane * fw + j], cid) : sel_key(0u, cid);
+              }
+            }
+          }
+          const int base = __popc(bal);
+          const int last = bal ? __shfl_sync(0xffffffffu, key_id(ki), 31 - __clz(bal)) : -1;
+          nkw = base;
+          if (lw == 0) {
+            flags |= 8;
+            break;
+          }
+          const int nn = base > 0 ? (base - 1) * fw + min(fw, nCw - last * fw) : 0;
+          if (nn > MC) {
+            flags |= 2;
+            break;
+          }
+          __syncwarp();
+          unsigned long long* t = ka;
+          ka = kb;
+          kb = t;
+          flags ^= 4;
+          nw = nn;
+          --lw;
+          if (!hc) {
+            flags |= 1;
+            break;
+          }
+          hc = false;
+          if (nw > kWarpMax) break;
+        }
+        if ((flags & 3) == 1 && nw > 0) request_rows(ka, lw, 0, min(nw, RB));
+        if (lane == 0) {
+          s_walk[0] = lw;
+          s_walk[1] = nw;
+          s_walk[2] = nkw;
+          s_walk[3] = flags;
+        }
+      }
+      __syncthreads();
+      const int flags = s_walk[3];
+      nk = s_walk[2];
+      if (flags & 4) {
+        unsigned long long* t = keysA;
+        keysA = keysB;
+        keysB = t;
+      }
+      if (flags & 2) overflow = true;
+      if (flags & 10) break;
+      l = s_walk[0] + 1;  // the loop steps down to the level reached
+      n = s_walk[1];
+      need_score = (flags & 1) != 0;
+      issued = need_score && n > 0;
+      have_child = false;
+      continue;
+    }
     if (n <= kFastMax) {
       // rank, compact and expand in two barriers: every lane holds its
       // share of the keys; warp w ranks candidates [w C, w C + C) with one
