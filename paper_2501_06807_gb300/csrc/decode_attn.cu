@@ -319,14 +319,6 @@ __device__ __forceinline__ void finish_grid(const AttnParams& p) {
 
 constexpr int kMaxPersistCtas = 152;
 
-__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
-}
 constexpr int kMaxBatchPersist = 512;
 constexpr int kSelSmem = 256;  // selected ids staged per warp (longer lists are read from global)
 

@@ -296,40 +296,30 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
   }
   bool have_child = spec0;  // cs holds the scores of all children of keysA[0, n)
   bool need_score = false;  // keysA holds ids only
-  bool issued = false;      // the first batch of the scoring round is already requested
-
-  // Requests the rows of candidates [x0, x1) of level l (keys in kk):
-  // children of kept clusters of level l + 1, so every run of fl
-  // consecutive candidates is one run of rows.  Warp 0 only.
-  auto request_rows = [&](const unsigned long long* kk, int l, int x0, int x1) {
-    const int fl = p.pyr.fanout[l];
-    const int64_t offL = (int64_t)p.pyr.off[l] * D;
-    if (lane == 0) mbar_arrive_expect_tx(&s_bar, (uint32_t)(x1 - x0) * ROWB * NSRC);
-    __syncwarp();
-    for (int c = x0 / fl + lane; c * fl < x1; c += 32) {
-      const int s0 = max(x0, c * fl), s1 = min(x1, c * fl + fl);
-      for (int w = 0; w < NSRC; ++w)
-        bulk_g2s(rows + ((size_t)w * RB + (s0 - x0)) * D, src0[w] + offL + (int64_t)key_id(kk[s0]) * D,
-                 (uint32_t)(s1 - s0) * ROWB, &s_bar);
-    }
-  };
 
   int nk = 0;
   for (int l = top; l >= 0 && !overflow; --l) {
     const int f = l > 0 ? p.pyr.fanout[l - 1] : 1;
     const int nC = l > 0 ? s_C[l - 1] : 0;
     if (need_score) {
-      // a round over the candidates' own rows, in batches of RB rows; the
-      // candidates are the children of the kept clusters of level l + 1, so
-      // every run of fl consecutive candidates is one run of rows
+      // a round over the candidates' own rows, in batches of RB rows,
+      // copied by every thread in 16-byte pieces (the rows are scattered
+      // runs of fl; spreading the copies over all warps issues them at once)
+      constexpr int CPR = ROWB / 16;  // pieces per row
+      const int64_t offL = (int64_t)p.pyr.off[l] * D;
       for (int x0 = 0; x0 < n; x0 += RB) {
         const int x1 = min(n, x0 + RB);
-        if (warp == 0 && !(x0 == 0 && issued)) request_rows(keysA, l, x0, x1);
-        wait_rows();
+        for (int c = tid; c < (x1 - x0) * CPR; c += NT) {
+          const int r = c / CPR, part = c - r * CPR;
+          const int64_t srow = offL + (int64_t)key_id(keysA[x0 + r]) * D + part * 4;
+          for (int w = 0; w < NSRC; ++w) cp_async16(rows + ((size_t)w * RB + r) * D + part * 4, src0[w] + srow);
+        }
+        cp_async_commit();
+        cp_async_wait<0>();
+        __syncthreads();
         score_rows(x1 - x0, [&](int r, uint32_t sc) { keysA[x0 + r] = sel_key(sc, key_id(keysA[x0 + r])); });
         __syncthreads();
       }
-      issued = false;
     }
 
     const int k = min(s_k[l], n);
@@ -337,7 +327,7 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
       // warp 0 ranks this level, expands the kept clusters, and goes on
       // down while the next level's scores are known and its candidates
       // fit, with no block barrier; it stops at level 0, or before a level
-      // whose rows must be scored (it then requests their first batch)
+      // whose rows must be scored
       if (warp == 0) {
         const unsigned lt = (1u << lane) - 1u;
         unsigned long long* ka = keysA;
@@ -396,7 +386,6 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
           hc = false;
           if (nw > kWarpMax) break;
         }
-        if ((flags & 3) == 1 && nw > 0) request_rows(ka, lw, 0, min(nw, RB));
         if (lane == 0) {
           s_walk[0] = lw;
           s_walk[1] = nw;
@@ -417,7 +406,6 @@ __global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ S
       l = s_walk[0] + 1;  // the loop steps down to the level reached
       n = s_walk[1];
       need_score = (flags & 1) != 0;
-      issued = need_score && n > 0;
       have_child = false;
       continue;
     }
