@@ -259,36 +259,77 @@ def run_ours(args, rank, world, dist):
     ms_per_step = total_ms / args.steps
     value = job_value(attended, world, ms_per_step)
 
-    # e2e through the public API with host buffers.  The step copies what the
-    # path reads: the leader layers' keys and window queries first (static
-    # eviction reads only those), then, on a side stream while static
-    # eviction runs, the other layers' keys, all values and the decode
-    # inputs; gathering waits for the side stream.  Non-leader window
-    # queries are never read, so they are not copied.
+    # e2e through the public API with host buffers.  A copy stream moves the
+    # leaders' keys and window queries to the device (static eviction reads
+    # only those), leader by leader, then the decode inputs, then the whole
+    # keys and values of the last group; each leader's static eviction starts
+    # once its copies have landed.  A gather stream then builds the group's
+    # caches from its kept rows (the leader's keys from the device, every
+    # other key and value row straight from pinned host memory, so evicted
+    # rows never cross the host link) while the next leaders are scored; the
+    # last group, whose gather would end the prefill, gathers from its device
+    # copy.  Non-leader window queries are never read, so they are not copied.
     e2e = None
     if not args.no_e2e:
         host = {n: getattr(x, n).cpu().pin_memory() for n in ("k", "v", "q_win", "q", "k_new", "v_new")}
         host_lens = x.prompt_lens.pin_memory()
         out_host = torch.empty(out_all.shape, dtype=out_all.dtype).pin_memory()
-        others = [l for l in range(w.n_layers) if l not in leaders]
-        first = [(x.k[l], host["k"][l]) for l in leaders] + [(x.q_win[l], host["q_win"][l]) for l in leaders]
-        second = ([(x.k[l], host["k"][l]) for l in others] +
-                  [(getattr(x, n), host[n]) for n in ("v", "q", "k_new", "v_new")])
-        h2d = sum(src.numel() * src.element_size() for _, src in first + second) + host_lens.numel() * 4
+        members = {lead: [l for l in range(w.n_layers) if eng.group_of[l] == eng.group_of[lead] and l != lead]
+                   for lead in leaders}
+        copies = [(x.k[l], host["k"][l]) for l in leaders] + [(x.q_win[l], host["q_win"][l]) for l in leaders]
+        decode_in = [(getattr(x, n), host[n]) for n in ("q", "k_new", "v_new")]
+        esz_kv = host["k"].element_size()
+        kept_rows = sum(int(t) for t in eng.n_keep.tolist()) * w.n_kv_heads  # per layer
+        n_last = sum(1 for l in range(w.n_layers) if eng.group_of[l] == eng.group_of[leaders[-1]])
+        gathered = kept_rows * w.head_dim * esz_kv * (len(leaders) - 1 + 2 * (w.n_layers - len(leaders) - (n_last - 1)))
+        whole_last = (2 * n_last - 1) * host["k"][0].numel() * esz_kv  # the last group's other K and all V
+        h2d = (sum(src.numel() * src.element_size() for _, src in copies + decode_in) +
+               host_lens.numel() * 4 + gathered + whole_last)
         d2h = out_host.numel() * out_host.element_size()
         side = torch.cuda.Stream(device=dev)
+        gat = torch.cuda.Stream(device=dev)
+        # the first and the last leader are scored alone (the first starts as
+        # soon as its copies land, the last ends the chain), the others two at
+        # a time (larger grids, fewer launches)
+        mid = leaders[1:-1]
+        batches = [leaders[:1]] + [mid[i:i + 2] for i in range(0, len(mid), 2)] + [leaders[-1:]]
+        batches = [bt for bt in batches if bt]
+        last = [l for l in range(w.n_layers) if eng.group_of[l] == eng.group_of[leaders[-1]]]
+        landed = [torch.cuda.Event() for _ in batches]
+        last_landed = torch.cuda.Event()
 
         def e2e_step():
-            for dst, src in first:
-                dst.copy_(src, non_blocking=True)
             lens.copy_(host_lens, non_blocking=True)
             side.wait_stream(stream)  # the previous step is done with the inputs
+            gat.wait_stream(stream)   # ... and with the caches
             with torch.cuda.stream(side):
-                for dst, src in second:
+                for i, batch in enumerate(batches):
+                    for lead in batch:
+                        x.k[lead].copy_(host["k"][lead], non_blocking=True)
+                        x.q_win[lead].copy_(host["q_win"][lead], non_blocking=True)
+                    landed[i].record(side)
+                for dst, src in decode_in:
                     dst.copy_(src, non_blocking=True)
-            eng.static_evict(x.k, x.q_win, lens, pt, w.page_size)
+                for l in last:
+                    if l != leaders[-1]:  # the leader's keys are already there
+                        x.k[l].copy_(host["k"][l], non_blocking=True)
+                    x.v[l].copy_(host["v"][l], non_blocking=True)
+                last_landed.record(side)
+            for i, batch in enumerate(batches):
+                stream.wait_event(landed[i])
+                eng.static_evict(x.k, x.q_win, lens, pt, w.page_size, layers=batch)
+                gat.wait_stream(stream)
+                with torch.cuda.stream(gat):
+                    if i == len(batches) - 1:
+                        gat.wait_event(last_landed)
+                        eng.build_clusters(x.k, x.v, pt, w.page_size, layers=last)
+                        continue
+                    eng.build_clusters(x.k, host["v"], pt, w.page_size, layers=batch)
+                    rest = [l for lead in batch for l in members[lead]]
+                    if rest:
+                        eng.build_clusters(host["k"], host["v"], pt, w.page_size, layers=rest)
+            stream.wait_stream(gat)
             stream.wait_stream(side)
-            eng.build_clusters(x.k, x.v, pt, w.page_size)
             graph.replay()
             out_host.copy_(out_all, non_blocking=True)
 

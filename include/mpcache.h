@@ -158,7 +158,9 @@ typedef struct {
   const mpc_layer_ref* refs;   /* host [n_refs] */
   int32_t batch, n_kv_heads, head_dim, dtype;
   int32_t t_max;
-  mpc_kv_tensor k, v;          /* prompt keys and values */
+  mpc_kv_tensor k, v;          /* prompt keys and values; data may also be pinned
+                                  host memory (device-accessible under unified
+                                  addressing): only the kept rows are read */
   const int32_t* kept;         /* device [group][batch][n_kv_heads][keep_cap] */
   int32_t keep_cap;
   const int32_t* n_keep;       /* device [batch] */

@@ -468,6 +468,16 @@ MPC_API int mpc_static_evict(const mpc_static_args* args, void* workspace, size_
   return ok();
 }
 
+// True for pinned host memory reached through unified addressing.
+static bool is_host_memory(const void* ptr) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, ptr) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeHost;
+}
+
 MPC_API int mpc_build_clusters_workspace_size(const mpc_cluster_args* args, size_t* bytes) {
   if (bytes == nullptr) return fail(MPC_ERR_INVALID_ARG, "bytes is NULL");
   ClusterParams p;
@@ -488,8 +498,10 @@ MPC_API int mpc_build_clusters(const mpc_cluster_args* args, void* workspace, si
   const int gx = (clusters + 3) / 4;
   bool any_leader = false;
   for (int i = 0; i < args->n_refs; ++i) any_leader |= args->refs[i].leader != 0;
+  // sources in host memory take the grid-stride gather (few SMs, deep loads)
+  const bool host_src = is_host_memory(args->k.data) || is_host_memory(args->v.data);
   const cudaError_t e = launch_clusters(p, args->dtype, args->head_dim, units, gx > 0 ? gx : 1, any_leader,
-                                        static_cast<cudaStream_t>(stream));
+                                        host_src, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "mpc_build_clusters launch");
   return ok();
 }

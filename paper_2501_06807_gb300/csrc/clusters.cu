@@ -14,7 +14,10 @@
 
 namespace mpc {
 
-
+// CTAs of the grid-stride gather (host sources): 4 warps each, U x 2 x 512
+// bytes in flight per warp (about 2.5 MB in all, ample for the host link);
+// half the SMs, measured best beside a concurrent scoring kernel.
+constexpr int kHostGatherCtas = 76;
 
 template <typename T, int D>
 __device__ __forceinline__ const T* kv_row(const KvSrc& src, int layer, int b, int h, int t, int Hkv,
@@ -25,20 +28,21 @@ __device__ __forceinline__ const T* kv_row(const KvSrc& src, int layer, int b, i
   return base + (((int64_t)pg * Hkv + h) * src.page_size + (t % src.page_size)) * D;
 }
 
+// Gathers finest cluster c of unit (ref, b, h) with one warp.  The rows'
+// chunks are loaded U row-steps at a time before any is used, so a warp keeps
+// U x 2 x 512 bytes in flight (the sources may sit across the host link).
 template <typename T, int D>
-__global__ void __launch_bounds__(128) gather_kernel(const __grid_constant__ ClusterParams p) {
+__device__ __forceinline__ void gather_cluster(const ClusterParams& p, int unit, int c, int lane) {
   constexpr int E = 16 / (int)sizeof(T);  // elements per chunk
   constexpr int CH = D / E;               // chunks per row
   constexpr int RPW = 32 / CH;            // rows per warp step
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int unit = blockIdx.y;
+  constexpr int U = 8;                    // row steps loaded at once
   const int h = unit % p.Hkv, b = (unit / p.Hkv) % p.B, ri = unit / (p.Hkv * p.B);
   const int layer = p.refs.layer[ri], group = p.refs.group[ri];
   const bool leader = p.refs.leader[ri];
   const int s = p.pyr.s;
   const int nk = p.n_keep[b];
-  if (blockIdx.x == 0 && threadIdx.x == 0 && ri == 0 && h == 0) p.out_n_tok[b] = nk;
-  const int c = blockIdx.x * 4 + warp;
+  if (c == 0 && lane == 0 && ri == 0 && h == 0) p.out_n_tok[b] = nk;
   const int r0 = c * s;
   if (r0 >= nk) return;
   const int r1 = min(r0 + s, nk);
@@ -58,25 +62,36 @@ __global__ void __launch_bounds__(128) gather_kernel(const __grid_constant__ Clu
     mn[e] = kPosInf;
     sm[e] = 0.f;
   }
-  for (int r = r0 + ro; r < r1; r += RPW) {
-    const int t = kept[r];
-    if (t < 0 || t >= p.t_max) {  // corrupt kept set: report, skip the row
-      atomicOr(&g_mpc_status, 4);
-      continue;
-    }
-    const uint4 kv = reinterpret_cast<const uint4*>(kv_row<T, D>(p.k, layer, b, h, t, p.Hkv, p.t_max))[ch];
-    const uint4 vv = reinterpret_cast<const uint4*>(kv_row<T, D>(p.v, layer, b, h, t, p.Hkv, p.t_max))[ch];
-    const int pch = ch ^ (r & 7);
-    reinterpret_cast<uint4*>(kc + (int64_t)r * D)[pch] = kv;
-    reinterpret_cast<uint4*>(vc + (int64_t)r * D)[pch] = vv;
-    if (leader && full) {
-      const T* el = reinterpret_cast<const T*>(&kv);
+  for (int rb = r0 + ro; rb < r1; rb += U * RPW) {
+    uint4 kv[U], vv[U];
+    bool ok[U];
 #pragma unroll
-      for (int e = 0; e < E; ++e) {
-        const float x = to_float<T>(el[e]);
-        mx[e] = fmaxf(mx[e], x);
-        mn[e] = fminf(mn[e], x);
-        sm[e] += x;
+    for (int u = 0; u < U; ++u) {
+      const int r = rb + u * RPW;
+      const int t = r < r1 ? kept[r] : 0;
+      ok[u] = r < r1 && t >= 0 && t < p.t_max;
+      if (r < r1 && !ok[u]) atomicOr(&g_mpc_status, 4);  // corrupt kept set: report, skip the row
+      if (ok[u]) {
+        kv[u] = reinterpret_cast<const uint4*>(kv_row<T, D>(p.k, layer, b, h, t, p.Hkv, p.t_max))[ch];
+        vv[u] = reinterpret_cast<const uint4*>(kv_row<T, D>(p.v, layer, b, h, t, p.Hkv, p.t_max))[ch];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (!ok[u]) continue;
+      const int r = rb + u * RPW;
+      const int pch = ch ^ (r & 7);
+      reinterpret_cast<uint4*>(kc + (int64_t)r * D)[pch] = kv[u];
+      reinterpret_cast<uint4*>(vc + (int64_t)r * D)[pch] = vv[u];
+      if (leader && full) {
+        const T* el = reinterpret_cast<const T*>(&kv[u]);
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+          const float x = to_float<T>(el[e]);
+          mx[e] = fmaxf(mx[e], x);
+          mn[e] = fminf(mn[e], x);
+          sm[e] += x;
+        }
       }
     }
   }
@@ -103,6 +118,24 @@ __global__ void __launch_bounds__(128) gather_kernel(const __grid_constant__ Clu
     p.rmin[row + cc] = mn[e];
     p.rep[row + cc] = fmaf(a, mx[e], am * mn[e]);
     if (p.mean != nullptr) p.mean[row + cc] = sm[e] / (float)s;
+  }
+}
+
+// One warp per finest cluster: blockIdx.y = unit, 4 clusters per CTA.
+template <typename T, int D>
+__global__ void __launch_bounds__(128) gather_kernel(const __grid_constant__ ClusterParams p) {
+  gather_cluster<T, D>(p, blockIdx.y, blockIdx.x * 4 + (threadIdx.x >> 5), threadIdx.x & 31);
+}
+
+// Grid-stride form for sources in host memory: a few CTAs keep the host link
+// busy (every warp holds U row-steps in flight) without spreading over every
+// SM, so that concurrent kernels keep the rest of the GPU.
+template <typename T, int D>
+__global__ void __launch_bounds__(128) gather_stride_kernel(const __grid_constant__ ClusterParams p, int per_unit,
+                                                            int n_items) {
+  for (int w = blockIdx.x * 4 + (threadIdx.x >> 5); w < n_items; w += gridDim.x * 4) {
+    __syncwarp();
+    gather_cluster<T, D>(p, w / per_unit, w % per_unit, threadIdx.x & 31);
   }
 }
 
@@ -153,15 +186,22 @@ __global__ void __launch_bounds__(256) coarse_kernel(const __grid_constant__ Clu
 }
 
 cudaError_t launch_clusters(const ClusterParams& p, int dtype, int D, int n_units, int groups_x,
-                            bool any_leader, cudaStream_t st) {
+                            bool any_leader, bool host_src, cudaStream_t st) {
   const dim3 grid(groups_x, n_units);
+  const int per_unit = groups_x * 4;
+  const long long items = (long long)per_unit * n_units;
+  const int nb = (int)(items / 4 < kHostGatherCtas ? (items + 3) / 4 : kHostGatherCtas);
+#define MPC_GATHER(TT, DD)                                                           \
+  if (host_src) gather_stride_kernel<TT, DD><<<nb, 128, 0, st>>>(p, per_unit, (int)items); \
+  else gather_kernel<TT, DD><<<grid, 128, 0, st>>>(p);
   if (dtype == MPC_BF16) {
-    if (D == 64) gather_kernel<bf16, 64><<<grid, 128, 0, st>>>(p);
-    else gather_kernel<bf16, 128><<<grid, 128, 0, st>>>(p);
+    if (D == 64) { MPC_GATHER(bf16, 64) }
+    else { MPC_GATHER(bf16, 128) }
   } else {
-    if (D == 64) gather_kernel<float, 64><<<grid, 128, 0, st>>>(p);
-    else gather_kernel<float, 128><<<grid, 128, 0, st>>>(p);
+    if (D == 64) { MPC_GATHER(float, 64) }
+    else { MPC_GATHER(float, 128) }
   }
+#undef MPC_GATHER
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (p.pyr.n_levels > 1 && any_leader) {

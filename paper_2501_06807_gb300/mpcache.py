@@ -323,12 +323,22 @@ class Engine:
         self._ws = {}
 
     # --------------------------------------------------------- prefill ----
+    @staticmethod
+    def _subset(refs_list, layers):
+        """The refs of ``layers`` (all refs when None)."""
+        if layers is None:
+            return refs_list
+        keep = set(int(l) for l in layers)
+        return [r for r in refs_list if r[0] in keep]
+
     def static_args(self, k: torch.Tensor, q_win: torch.Tensor, lens: torch.Tensor,
-                    page_table: Optional[torch.Tensor] = None, page_size: int = 16) -> StaticArgs:
-        refs = _refs(self.refs_lead)
+                    page_table: Optional[torch.Tensor] = None, page_size: int = 16,
+                    layers: Optional[Sequence[int]] = None) -> StaticArgs:
+        lead = self._subset(self.refs_lead, layers)
+        refs = _refs(lead)
         a = StaticArgs()
         a.struct_size = C.sizeof(StaticArgs)
-        a.n_refs = len(self.refs_lead)
+        a.n_refs = len(lead)
         a.refs = C.cast(refs, C.POINTER(LayerRef))
         a.batch, a.n_q_heads, a.n_kv_heads, a.head_dim, a.dtype = self.B, self.Hq, self.Hkv, self.d, self.dcode
         a.t_max = self.t_max
@@ -356,20 +366,25 @@ class Engine:
             kv.max_pages = page_table.shape[1]
         return kv
 
-    def static_evict(self, k, q_win, lens, page_table=None, page_size=16):
+    def static_evict(self, k, q_win, lens, page_table=None, page_size=16, layers=None):
+        """Static eviction of the leader layers (of ``layers`` only, if given)."""
         lib = load()
-        a = self.static_args(k, q_win, lens, page_table, page_size)
+        a = self.static_args(k, q_win, lens, page_table, page_size, layers)
         n = C.c_size_t(0)
         _check(lib.mpc_static_evict_workspace_size(C.byref(a), C.byref(n)))
         ws = _ws_zero(n.value, self._ws, "static")
         _check(lib.mpc_static_evict(C.byref(a), C.c_void_p(_ptr(ws)), n.value, C.c_void_p(_stream())))
 
-    def build_clusters(self, k, v, page_table=None, page_size=16):
+    def build_clusters(self, k, v, page_table=None, page_size=16, layers=None):
+        """Gathering and clustering of every layer (of ``layers`` only, if
+        given).  k and v may be pinned host tensors: the gather then reads
+        only the kept rows across the host link."""
         lib = load()
-        refs = _refs(self.refs_all)
+        sub = self._subset(self.refs_all, layers)
+        refs = _refs(sub)
         a = ClusterArgs()
         a.struct_size = C.sizeof(ClusterArgs)
-        a.n_refs = len(self.refs_all)
+        a.n_refs = len(sub)
         a.refs = C.cast(refs, C.POINTER(LayerRef))
         a.batch, a.n_kv_heads, a.head_dim, a.dtype = self.B, self.Hkv, self.d, self.dcode
         a.t_max = self.t_max

@@ -183,6 +183,41 @@ def _off(eng, level):
     return off
 
 
+@pytest.mark.parametrize("paged", [False, True])
+def test_prefill_per_group_from_pinned_host_memory(paged):
+    """Static eviction one leader at a time and gathering per group, with the
+    keys of non-leader layers and all values read from pinned host memory
+    (only the kept rows cross the host link), equals the one-call prefill
+    from device tensors bit for bit."""
+    w = synth.C3.replace(n_layers=6, prompt_len=700, prompt_len_min=300, batch=2, n_q_heads=8, n_kv_heads=2,
+                         share_every=2)
+    if paged:
+        w = w.replace(page_size=16, paged=True)
+    x = synth.generate(w, H.window_rows_for(w), device="cpu", decode_steps=1)
+    xc = H.to_cuda(x)
+    pt = xc.page_table.cuda() if xc.page_table is not None else None
+    lens = x.prompt_lens.cuda()
+    ref = H.make_engine(w, 1)
+    ref.prefill(xc.k, xc.v, xc.q_win, lens, pt, w.page_size)
+    eng = H.make_engine(w, 1)
+    hk, hv = x.k.pin_memory(), x.v.pin_memory()
+    gat = torch.cuda.Stream()
+    for lead in eng.leaders:
+        eng.static_evict(xc.k, xc.q_win, lens, pt, w.page_size, layers=[lead])
+        gat.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(gat):
+            members = [l for l in range(w.n_layers) if eng.group_of[l] == eng.group_of[lead] and l != lead]
+            eng.build_clusters(xc.k, hv, pt, w.page_size, layers=[lead])
+            if members:
+                eng.build_clusters(hk, hv, pt, w.page_size, layers=members)
+    torch.cuda.current_stream().wait_stream(gat)
+    torch.cuda.synchronize()
+    for name in ("kept", "n_keep", "n_tok", "kc", "vc", "rmax", "rmin", "rep", "mean"):
+        assert torch.equal(getattr(eng, name), getattr(ref, name)), name
+    assert torch.equal(eng.scores, ref.scores)
+    assert mpcache.device_status() == 0
+
+
 # ------------------------------------------------- selection in isolation ----
 
 SELECT_CASES = [
