@@ -18,6 +18,9 @@ namespace mpc {
 // bytes in flight per warp (about 2.5 MB in all, ample for the host link);
 // half the SMs, measured best beside a concurrent scoring kernel.
 constexpr int kHostGatherCtas = 76;
+// Row steps loaded at once by the one-warp-per-cluster gather (device
+// sources: occupancy hides the latency).
+constexpr int kDeviceGatherSteps = 1;
 
 template <typename T, int D>
 __device__ __forceinline__ const T* kv_row(const KvSrc& src, int layer, int b, int h, int t, int Hkv,
@@ -30,13 +33,12 @@ __device__ __forceinline__ const T* kv_row(const KvSrc& src, int layer, int b, i
 
 // Gathers finest cluster c of unit (ref, b, h) with one warp.  The rows'
 // chunks are loaded U row-steps at a time before any is used, so a warp keeps
-// U x 2 x 512 bytes in flight (the sources may sit across the host link).
-template <typename T, int D>
+// U x 2 x 512 bytes in flight (U > 1 for sources across the host link).
+template <typename T, int D, int U>
 __device__ __forceinline__ void gather_cluster(const ClusterParams& p, int unit, int c, int lane) {
   constexpr int E = 16 / (int)sizeof(T);  // elements per chunk
   constexpr int CH = D / E;               // chunks per row
   constexpr int RPW = 32 / CH;            // rows per warp step
-  constexpr int U = 8;                    // row steps loaded at once
   const int h = unit % p.Hkv, b = (unit / p.Hkv) % p.B, ri = unit / (p.Hkv * p.B);
   const int layer = p.refs.layer[ri], group = p.refs.group[ri];
   const bool leader = p.refs.leader[ri];
@@ -124,7 +126,7 @@ __device__ __forceinline__ void gather_cluster(const ClusterParams& p, int unit,
 // One warp per finest cluster: blockIdx.y = unit, 4 clusters per CTA.
 template <typename T, int D>
 __global__ void __launch_bounds__(128) gather_kernel(const __grid_constant__ ClusterParams p) {
-  gather_cluster<T, D>(p, blockIdx.y, blockIdx.x * 4 + (threadIdx.x >> 5), threadIdx.x & 31);
+  gather_cluster<T, D, kDeviceGatherSteps>(p, blockIdx.y, blockIdx.x * 4 + (threadIdx.x >> 5), threadIdx.x & 31);
 }
 
 // Grid-stride form for sources in host memory: a few CTAs keep the host link
@@ -135,7 +137,7 @@ __global__ void __launch_bounds__(128) gather_stride_kernel(const __grid_constan
                                                             int n_items) {
   for (int w = blockIdx.x * 4 + (threadIdx.x >> 5); w < n_items; w += gridDim.x * 4) {
     __syncwarp();
-    gather_cluster<T, D>(p, w / per_unit, w % per_unit, threadIdx.x & 31);
+    gather_cluster<T, D, 8>(p, w / per_unit, w % per_unit, threadIdx.x & 31);
   }
 }
 
