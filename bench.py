@@ -430,8 +430,9 @@ def oracle_sample(w, E_sample=4):
     x = synth.generate(ws, R, decode_steps=E_sample)
     T = int(x.prompt_lens[0])
     G, d, s = w.group, w.head_dim, w.cluster_size
-    K = x.k[0, 0, 0, :T].double().numpy()
-    V = x.v[0, 0, 0, :T].double().numpy()
+    kd, vd = x.dense_kv(0, 0)  # dense view (paged workloads keep a page pool)
+    K = kd[0, :T].double().numpy()
+    V = vd[0, :T].double().numpy()
     wl = O.window_length(T, w.window_ppm, w.long_window_ppm, w.long_prompt_threshold)
     qw = x.q_win[0, 0, :G, R - wl:].double().numpy()
     t0 = time.perf_counter()
