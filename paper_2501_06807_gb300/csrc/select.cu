@@ -34,6 +34,12 @@ constexpr int kRankMax = 1024;  // candidates ranked by counting
 
 constexpr int kSelChunk = 8192; // bytes per bulk copy
 
+// Resident CTAs per SM asked of the 4-warp instantiation (many small units:
+// latency-bound, so residency sets the throughput).  Measured on the batch-32
+// paged workload: 4 (120 registers) 178 us per step, 5 (96) 153 us, 6 and 8
+// (80 and 64, with spills) 159 and 167 us.
+constexpr int kSelMinCtas128 = 5;
+
 __device__ __forceinline__ unsigned long long sel_key(uint32_t oscore, int id) {
   return ((unsigned long long)oscore << 32) | (unsigned long long)(0xffffffffu - (uint32_t)id);
 }
@@ -94,7 +100,7 @@ __device__ __forceinline__ void warp_copy(void* dst, const void* src, uint32_t n
 // FXP: the fixed-point metric (its own instantiation, so the fp32 metrics
 // keep their register budget).
 template <typename T, int D, int NT, bool FXP>
-__global__ void __launch_bounds__(NT, 1) select_kernel(const __grid_constant__ SelectParams p) {
+__global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_kernel(const __grid_constant__ SelectParams p) {
   constexpr int NW = NT / 32;
   constexpr int LPR = D / 4;     // lanes per representative row (one float4 each)
   constexpr int RPW = 32 / LPR;  // rows per warp-wide read
