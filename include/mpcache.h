@@ -120,7 +120,10 @@ typedef struct {
  *             (equal scores: lower position first), in ascending order.
  * Outputs: out_scores[group][b][h][t_max] (positions >= T_b undefined),
  * out_kept[group][b][h][keep_cap] (entries >= n_keep_b are -1) and
- * out_n_keep[b].  Refs must all be leaders. */
+ * out_n_keep[b].  Refs must all be leaders.  Workspace: the window rows'
+ * statistics and, for paged bf16 keys, a dense copy of the refs' keys
+ * (n_refs * batch * n_kv_heads * t_max * d * 2 bytes) gathered before the
+ * tensor-core passes. */
 typedef struct {
   uint32_t struct_size;        /* sizeof(mpc_static_args) */
   int32_t n_refs;

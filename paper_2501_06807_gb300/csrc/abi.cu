@@ -122,7 +122,7 @@ int validate_static(const mpc_static_args* a, StaticParams* p) {
   if (a->keep_cap < kb) return fail(MPC_ERR_BAD_SHAPE, "keep_cap %d < %d kept tokens at t_max", a->keep_cap, kb);
   if (a->scale < 0.f || !std::isfinite(a->scale)) return fail(MPC_ERR_BAD_SHAPE, "scale must be finite and >= 0");
   const mpc_kv_tensor& k = a->k;
-  if (a->dtype == MPC_BF16 && k.page_table == nullptr &&
+  if (a->dtype == MPC_BF16 &&
       (!aligned16(a->q_win) || !aligned16(k.data) || (a->q_win_layer_stride * 2) % 16 || (k.layer_stride * 2) % 16))
     return fail(MPC_ERR_INVALID_ARG, "bf16 q_win / k and their layer strides must be 16-byte aligned");
   if (k.page_table != nullptr && (k.page_size < 1 || k.max_pages < 1 ||
@@ -164,8 +164,12 @@ int validate_static(const mpc_static_args* a, StaticParams* p) {
 // the SIMT passes, then the same value over the log2 scale as three bf16
 // parts in a 16-byte row for the tcgen05 passes.
 int stats_ld_of(int win_rows) { return (win_rows + 127) / 128 * 128; }
-size_t static_ws(const StaticParams& p) {
+size_t static_stats_bytes(const StaticParams& p) {
   return (size_t)p.n_refs * p.B * p.Hq * stats_ld_of(p.win_rows) * (sizeof(float) + 16);
+}
+// the statistics, then (paged bf16 keys) their gathered dense copy
+size_t static_ws(const StaticParams& p, int dtype, int D) {
+  return static_stats_bytes(p) + static_dense_bytes(p, dtype, D);
 }
 
 // ------------------------------------------------------------ clusters ----
@@ -445,7 +449,7 @@ MPC_API int mpc_static_evict_workspace_size(const mpc_static_args* args, size_t*
   if (bytes == nullptr) return fail(MPC_ERR_INVALID_ARG, "bytes is NULL");
   StaticParams p;
   MPC_TRY(validate_static(args, &p));
-  *bytes = static_ws(p);
+  *bytes = static_ws(p, args->dtype, args->head_dim);
   return ok();
 }
 
@@ -454,13 +458,16 @@ MPC_API int mpc_static_evict(const mpc_static_args* args, void* workspace, size_
   MPC_TRY(validate_static(args, &p));
   if (!args->q_win || !args->k.data || !args->prompt_lens || !args->out_scores || !args->out_kept || !args->out_n_keep)
     return fail(MPC_ERR_INVALID_ARG, "a required pointer is NULL");
-  const size_t need = static_ws(p);
+  const size_t need = static_ws(p, args->dtype, args->head_dim);
   if (workspace == nullptr || workspace_bytes < need)
     return fail(MPC_ERR_WORKSPACE, "workspace of %zu bytes needed", need);
   if (!aligned16(workspace)) return fail(MPC_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
   p.stats = static_cast<float*>(workspace);
   p.stats_ld = stats_ld_of(p.win_rows);
   p.aug = static_cast<uint8_t*>(workspace) + (size_t)p.n_refs * p.B * p.Hq * p.stats_ld * sizeof(float);
+  p.k_dense = static_dense_bytes(p, args->dtype, args->head_dim) ? static_cast<uint8_t*>(workspace) +
+                                                                       static_stats_bytes(p)
+                                                                 : nullptr;
   int span = 0;
   for (int i = 0; i < args->n_refs; ++i) span = args->refs[i].layer + 1 > span ? args->refs[i].layer + 1 : span;
   const cudaError_t e = launch_static(p, args->dtype, args->head_dim, span, static_cast<cudaStream_t>(stream));

@@ -83,16 +83,13 @@ struct StaticParams {
   int stats_ld;       // win_rows rounded up to 128
   void* aug;          // [ref][b][Hq][stats_ld][8] bf16: -(m + log2 l) / scale_log2 as the sum of
                       // three bf16 parts, then five zeros (tcgen05 passes)
+  void* k_dense;      // paged bf16 keys gathered as [ref][b][Hkv][t_max][d] (tcgen05 passes)
 };
 
 // Window scoring on tcgen05 (bf16 queries and dense keys).
 struct ScoreTcParams {
   CUtensorMap map_q;  // [layer][B*Hq*win_rows][d], 128 x 64 boxes, 128B swizzle
-  CUtensorMap map_k;  // dense [layer][B*Hkv*t_max][d] (128-row boxes) or the
-                      // page pool [layer][pages*Hkv*page_size][d] (page-row boxes)
-  const int* page_table;  // null for dense keys
-  int page_size, max_pages;
-  int64_t pool_pages;     // pages per layer of the pool
+  CUtensorMap map_k;  // dense [layer or ref][B*Hkv*t_max][d] (128-row boxes)
   RefTable refs;
   int n_refs, B, Hq, Hkv, G, t_max, win_rows;
   const int* lens;
@@ -106,6 +103,7 @@ struct ScoreTcParams {
   float* stats;  // as StaticParams::stats
   int stats_ld;
   void* aug;     // as StaticParams::aug
+  int k_by_ref;  // dense keys indexed by ref (a gathered copy) rather than by layer
 };
 
 struct KvSrc {
@@ -152,6 +150,8 @@ cudaError_t launch_clusters(const ClusterParams& p, int dtype, int D, int n_unit
                             bool any_leader, bool host_src, cudaStream_t st);
 cudaError_t launch_static(const StaticParams& p, int dtype, int D, int n_layer_span, cudaStream_t st);
 cudaError_t launch_score_tc(ScoreTcParams& p, int D, int n_layer_span, cudaStream_t st);
+// Bytes of the gathered dense copy of paged bf16 keys (0 when not needed).
+size_t static_dense_bytes(const StaticParams& p, int dtype, int D);
 int static_tile_smem(int D);
 
 // Records `msg` as this thread's last error (mpc_last_error) and returns code.

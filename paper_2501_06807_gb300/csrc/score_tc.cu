@@ -1,6 +1,7 @@
 // Window scoring of look-once static eviction on the 5th-generation tensor
 // cores (Sec. 3.2; Alg. 2 Step 1): the two passes of the accumulated window
-// attention for bf16 queries and dense keys.
+// attention for bf16 queries and dense keys (paged keys arrive as a dense
+// copy gathered by the caller, indexed by ref).
 //
 //   pass 0 (row statistics): one CTA per (ref, sequence, query head, 128
 //     window rows).  A = the 128 query rows (fixed), B = 128-key tiles
@@ -276,6 +277,10 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
       }
     }
   }
+  // a CTA past its sequence's window (pass 0) or keys (pass 1) has nothing
+  // to compute or write: leave before the barriers and the TMEM allocation
+  // (ragged batches launch many of them)
+  if (n_tiles == 0) return;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStagesTc; ++s) {
@@ -318,38 +323,11 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
     const int qrow0 = (b * p.Hq) * p.win_rows + qoff;       // + hq * win_rows + i
     const int krow0 = (b * p.Hkv) * p.t_max;                 // + hk * t_max + j
     // keys [kj, kj + 128) of kv head hk: one 128-row box per 64-channel half
-    // for dense keys; for paged keys one box per page, stacked in order (a
-    // page holds whole 8-row swizzle atoms, so the stack has the layout of
-    // one 128-row box).  Pages past the sequence or outside the pool are not
-    // loaded (their keys are masked or unused).
     auto load_keys = [&](uint8_t* dst, int hk, int kj, uint64_t* bar) {
-      if (p.page_table == nullptr) {
-        mbar_arrive_expect_tx(bar, S::TILE);
-        for (int kh = 0; kh < KH; ++kh)
-          tma_load_3d(dst + kh * kBoxBytes, &p.map_k, kh * 64, krow0 + hk * p.t_max + kj, layer, bar);
-        return;
-      }
-      const int ps = p.page_size, np = 128 / ps;
-      int pg[128 / 8];
-      uint32_t bytes = 0;
-      for (int i = 0; i < np; ++i) {
-        const int pi = kj / ps + i;
-        pg[i] = -1;
-        if (pi < p.max_pages && pi * ps < T_b) {
-          const int g = __ldg(p.page_table + (int64_t)b * p.max_pages + pi);
-          if (g >= 0 && g < p.pool_pages) {
-            pg[i] = g;
-            bytes += (uint32_t)ps * 128 * KH;
-          } else {
-            atomicOr(&g_mpc_status, 4);
-          }
-        }
-      }
-      mbar_arrive_expect_tx(bar, bytes);
-      for (int i = 0; i < np; ++i)
-        if (pg[i] >= 0)
-          for (int kh = 0; kh < KH; ++kh)
-            tma_load_3d(dst + kh * kBoxBytes + i * ps * 128, &p.map_k, kh * 64, (pg[i] * p.Hkv + hk) * ps, layer, bar);
+      mbar_arrive_expect_tx(bar, S::TILE);
+      for (int kh = 0; kh < KH; ++kh)
+        tma_load_3d(dst + kh * kBoxBytes, &p.map_k, kh * 64, krow0 + hk * p.t_max + kj, p.k_by_ref ? ri : layer,
+                    bar);
     };
     if (PASS == 0) {
       mbar_arrive_expect_tx(a_full, S::TILE);
@@ -554,14 +532,13 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-// 3-D map over [layers][rows][d] bf16 with box_rows x 64-channel boxes.
-bool make_map(CUtensorMap* map, const void* base, int d, int64_t rows, int layers, int64_t layer_stride_elems,
-              int box_rows = 128) {
+// 3-D map over [layers][rows][d] bf16 with 128-row x 64-channel boxes.
+bool make_map(CUtensorMap* map, const void* base, int d, int64_t rows, int layers, int64_t layer_stride_elems) {
   auto fn = encode_fn();
   if (fn == nullptr) return false;
   const cuuint64_t dims[3] = {(cuuint64_t)d, (cuuint64_t)rows, (cuuint64_t)layers};
   const cuuint64_t strides[2] = {(cuuint64_t)d * 2, (cuuint64_t)layer_stride_elems * 2};
-  const cuuint32_t box[3] = {64, (cuuint32_t)box_rows, 1};
+  const cuuint32_t box[3] = {64, 128, 1};
   const cuuint32_t estr[3] = {1, 1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -582,14 +559,8 @@ cudaError_t launch_pass(const ScoreTcParams& p, dim3 grid, cudaStream_t st) {
 cudaError_t launch_score_tc(ScoreTcParams& p, int D, int n_layer_span, cudaStream_t st) {
   if (!make_map(&p.map_q, p.q_win, D, (int64_t)p.B * p.Hq * p.win_rows, n_layer_span, p.qw_ls))
     return cudaErrorInvalidValue;
-  if (p.page_table == nullptr) {
-    if (!make_map(&p.map_k, p.k, D, (int64_t)p.B * p.Hkv * p.t_max, n_layer_span, p.k_ls)) return cudaErrorInvalidValue;
-  } else {
-    // the pool of one layer spans layer_stride elements
-    p.pool_pages = p.k_ls / ((int64_t)p.Hkv * p.page_size * D);
-    if (!make_map(&p.map_k, p.k, D, p.pool_pages * p.Hkv * p.page_size, n_layer_span, p.k_ls, p.page_size))
-      return cudaErrorInvalidValue;
-  }
+  if (!make_map(&p.map_k, p.k, D, (int64_t)p.B * p.Hkv * p.t_max, p.k_by_ref ? p.n_refs : n_layer_span, p.k_ls))
+    return cudaErrorInvalidValue;
   const dim3 g0((p.win_rows + 127) / 128, p.n_refs * p.B * p.Hq);
   const dim3 g1((p.t_max + 127) / 128, p.n_refs * p.B * p.Hkv);
   cudaError_t e;

@@ -304,13 +304,52 @@ static cudaError_t set_smem(K kernel, int bytes) {
   return ensure_dyn_smem((const void*)kernel, bytes);
 }
 
+// Gathers the paged keys of every (ref, sequence, kv head) into a dense
+// [ref][b][Hkv][t_max][d] copy (rows [0, T_b)), so that the tensor-core
+// passes stream 128-key tiles with two TMA boxes rather than one per page
+// and half.  Page ids outside the pool are reported and their rows skipped.
+template <int D>
+__global__ void __launch_bounds__(256) densify_kernel(const __grid_constant__ StaticParams p) {
+  constexpr int CH = D * 2 / 16;  // 16-byte chunks per bf16 row
+  const int unit = blockIdx.y;
+  const int h = unit % p.Hkv, b = (unit / p.Hkv) % p.B, ri = unit / (p.Hkv * p.B);
+  const int layer = p.refs.layer[ri];
+  const int T_b = p.lens[b];
+  const int r0 = blockIdx.x * 128;
+  if (T_b < 1 || T_b > p.t_max || r0 >= T_b) return;
+  const int64_t pool_pages = p.k_ls / ((int64_t)p.Hkv * p.page_size * D);
+  const bf16* pool = (const bf16*)p.k + layer * p.k_ls;
+  bf16* dst = (bf16*)p.k_dense + (((int64_t)ri * p.B + b) * p.Hkv + h) * p.t_max * D;
+  for (int i = threadIdx.x; i < 128 * CH; i += blockDim.x) {
+    const int r = r0 + i / CH, c = i % CH;
+    if (r >= T_b) break;
+    const int pg = p.page_table[(int64_t)b * p.max_pages + r / p.page_size];
+    if (pg < 0 || pg >= pool_pages) {
+      atomicOr(&g_mpc_status, 4);
+      continue;
+    }
+    const bf16* src = pool + (((int64_t)pg * p.Hkv + h) * p.page_size + r % p.page_size) * D;
+    reinterpret_cast<uint4*>(dst + (int64_t)r * D)[c] = reinterpret_cast<const uint4*>(src)[c];
+  }
+}
+
+size_t static_dense_bytes(const StaticParams& p, int dtype, int D) {
+  if (dtype != MPC_BF16 || p.page_table == nullptr) return 0;
+  return (size_t)p.n_refs * p.B * p.Hkv * p.t_max * D * 2;
+}
+
 cudaError_t launch_static(const StaticParams& p, int dtype, int D, int n_layer_span, cudaStream_t st) {
   cudaError_t e = cudaSuccess;
-  const bool tc_pages = p.page_table == nullptr ||
-                        (p.page_size >= 8 && p.page_size <= 128 && 128 % p.page_size == 0 && p.k_ls > 0);
-  if (dtype == MPC_BF16 && tc_pages) {
-    // both score passes on the tensor cores (dense keys, or pages of 8 to
-    // 128 rows that tile a 128-key block)
+  if (dtype == MPC_BF16) {
+    // both score passes on the tensor cores; paged keys are first gathered
+    // into the dense copy in the workspace
+    const bool paged = p.page_table != nullptr;
+    if (paged) {
+      const dim3 gd((p.t_max + 127) / 128, p.n_refs * p.B * p.Hkv);
+      if (D == 64) densify_kernel<64><<<gd, 256, 0, st>>>(p);
+      else densify_kernel<128><<<gd, 256, 0, st>>>(p);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
     ScoreTcParams t;
     memset(&t, 0, sizeof(t));
     t.refs = p.refs;
@@ -324,8 +363,9 @@ cudaError_t launch_static(const StaticParams& p, int dtype, int D, int n_layer_s
     t.lens = p.lens;
     t.q_win = p.q_win;
     t.qw_ls = p.qw_ls;
-    t.k = p.k;
-    t.k_ls = p.k_ls;
+    t.k = paged ? p.k_dense : p.k;
+    t.k_ls = paged ? (int64_t)p.B * p.Hkv * p.t_max * D : p.k_ls;
+    t.k_by_ref = paged ? 1 : 0;
     t.window_ppm = p.window_ppm;
     t.long_window_ppm = p.long_window_ppm;
     t.long_threshold = p.long_threshold;
@@ -334,9 +374,6 @@ cudaError_t launch_static(const StaticParams& p, int dtype, int D, int n_layer_s
     t.stats = p.stats;
     t.stats_ld = p.stats_ld;
     t.aug = p.aug;
-    t.page_table = p.page_table;
-    t.page_size = p.page_size;
-    t.max_pages = p.max_pages;
     if ((e = launch_score_tc(t, D, n_layer_span, st)) != cudaSuccess) return e;
   } else {
     const int smem = static_tile_smem(D);

@@ -183,15 +183,19 @@ def _off(eng, level):
     return off
 
 
-@pytest.mark.parametrize("paged", [False, True])
-def test_prefill_per_group_from_pinned_host_memory(paged):
+@pytest.mark.parametrize("case", ["bf16_dense", "bf16_paged", "f32_d64"])
+def test_prefill_per_group_from_pinned_host_memory(case):
     """Static eviction one leader at a time and gathering per group, with the
     keys of non-leader layers and all values read from pinned host memory
     (only the kept rows cross the host link), equals the one-call prefill
     from device tensors bit for bit."""
-    w = synth.C3.replace(n_layers=6, prompt_len=700, prompt_len_min=300, batch=2, n_q_heads=8, n_kv_heads=2,
-                         share_every=2)
-    if paged:
+    if case == "f32_d64":
+        w = synth.C1.replace(n_layers=4, prompt_len=300, prompt_len_min=200, batch=2, n_q_heads=4, n_kv_heads=2,
+                             share_every=2, fanouts=(4,), level_keep_ppm=(250_000, 500_000))
+    else:
+        w = synth.C3.replace(n_layers=6, prompt_len=700, prompt_len_min=300, batch=2, n_q_heads=8, n_kv_heads=2,
+                             share_every=2)
+    if case == "bf16_paged":
         w = w.replace(page_size=16, paged=True)
     x = synth.generate(w, H.window_rows_for(w), device="cpu", decode_steps=1)
     xc = H.to_cuda(x)
