@@ -606,3 +606,109 @@ def test_commonality_of_unshared_selections():
             for h in range(w.n_kv_heads):
                 ref = O.commonality([list(s_cpu[l, b, h, :n_sel]) for l in range(w.n_layers)], n_sel, m)
                 assert int(total[b, h]) == round(ref * n_sel * (w.n_layers - m))
+
+
+# ------------------------------------------ full size, sampled outputs ----
+
+def _full_size_sampled(w, E, pick):
+    """Runs a workload at full size, in the launch configuration the
+    benchmark times, for E decode steps, and checks sampled (leader,
+    sequence, kv head) units against the oracle one by one: window scores and
+    the kept set, the cluster summaries, every step's selection, and the
+    attention outputs of the leader and of its group's last layer.
+    Downstream checks start from the GPU's kept set and selections, so a tie
+    at one cut does not mask the next stage.  ``pick(eng, x)`` names the
+    sampled units."""
+    R = H.window_rows_for(w)
+    x = synth.generate(w, R, device="cuda", decode_steps=E)
+    eng = H.make_engine(w, E)
+    pt = x.page_table.cuda() if x.page_table is not None else None
+    eng.prefill(x.k, x.v, x.q_win, x.prompt_lens.cuda(), pt, w.page_size)
+    torch.cuda.synchronize()
+    G, d, s = w.group, w.head_dim, w.cluster_size
+    scale = 1 / math.sqrt(d)
+    samples = pick(eng, x)
+    members = {lead: [l for l in range(w.n_layers) if eng.group_of[l] == eng.group_of[lead]] for lead, _, _ in samples}
+    watch = sorted({(l, b) for lead, b, _ in samples for l in (lead, members[lead][-1])})
+    scores = eng.scores.cpu().double().numpy()
+    kept = eng.kept.cpu().numpy()
+    rmax, rmin, rep = eng.rmax.cpu().numpy(), eng.rmin.cpu().numpy(), eng.rep.cpu().numpy()
+    sels, outs = [], []
+    for e in range(E):
+        eng.decode_step(x.q[e], x.k_new[e], x.v_new[e])
+        sels.append(eng.sel.cpu().numpy().copy())
+        outs.append({lb: eng.out[lb[0], lb[1]].cpu().double().numpy() for lb in watch})
+    assert mpcache.device_status() == 0
+    dense = {}
+
+    def kv(l, b):
+        if (l, b) not in dense:
+            k, v = x.dense_kv(l, b)
+            dense[(l, b)] = (k.double().cpu().numpy(), v.double().cpu().numpy())
+        return dense[(l, b)]
+
+    for lead, b, h in samples:
+        grp = eng.group_of[lead]
+        T = int(x.prompt_lens[b])
+        wl = O.window_length(T, w.window_ppm, w.long_window_ppm, w.long_prompt_threshold)
+        n_keep = O.kept_count(T, w.keep_ppm)
+        K = kv(lead, b)[0][h]
+        qw = x.q_win[lead, b, h * G:(h + 1) * G, R - wl:].double().cpu().numpy()
+        # static eviction
+        ref = O.accumulated_attention(qw, K, scale)
+        tau = static_band(qw, K, scale, wl, G)
+        got = scores[grp, b, h, :T]
+        assert np.all(np.abs(got - ref) <= tau * ref + 1e-30), (lead, b, h)
+        ref_kept = O.static_evict(ref, n_keep)
+        gk = kept[grp, b, h, :n_keep]
+        H.set_parity(gk, ref_kept, lambda ids: ref[ids], n_keep, band=2 * tau * ref[ref_kept].min())
+        # summaries of the GPU's kept keys, as gathered at prefill
+        levels = O.cluster_pyramid(K[gk], s, w.fanouts, w.alpha)
+        for li, lv in enumerate(levels):
+            rows = slice(_off(eng, li), _off(eng, li) + len(lv.members))
+            assert np.array_equal(rmax[grp, b, h, rows].astype(np.float64), lv.r_max), (lead, b, h, li)
+            assert np.array_equal(rmin[grp, b, h, rows].astype(np.float64), lv.r_min), (lead, b, h, li)
+            assert np.allclose(rep[grp, b, h, rows], lv.rep, rtol=4e-7, atol=4e-7 * np.abs(lv.rep).max(initial=0))
+        for e in range(E):
+            n_tok = n_keep + e  # cache rows before this step's append
+            lead_cache = np.concatenate([K[gk], x.k_new[:e, lead, b, h].double().cpu().numpy()])
+            lv_e = O.cluster_pyramid(lead_cache[:n_tok], s, w.fanouts, w.alpha)
+            qg = x.q[e, lead, b, h * G:(h + 1) * G].double().cpu().numpy()
+            tr = []
+            ref_sel = O.hierarchical_select(qg, lv_e, w.fanouts, w.level_keep_ppm, trace=tr)
+            got_sel = sels[e][grp, b, h, :len(ref_sel)]
+            C1 = n_tok // s
+            if unique_selection(tr, select_band(qg, lv_e)):
+                assert np.array_equal(got_sel, ref_sel), (lead, b, h, e)
+            else:
+                assert np.all(np.diff(got_sel) > 0) and got_sel.min(initial=0) >= 0 and got_sel.max(initial=-1) < C1
+            rows = np.concatenate([np.arange(c * s, (c + 1) * s) for c in got_sel] + [np.arange(C1 * s, n_tok)])
+            for l in (lead, members[lead][-1]):
+                Kl, Vl = kv(l, b)
+                cache_k = np.concatenate([Kl[h][gk], x.k_new[:e, l, b, h].double().cpu().numpy()])
+                cache_v = np.concatenate([Vl[h][gk], x.v_new[:e, l, b, h].double().cpu().numpy()])
+                Ka = np.concatenate([cache_k[rows], x.k_new[e, l, b, h][None].double().cpu().numpy()])
+                Va = np.concatenate([cache_v[rows], x.v_new[e, l, b, h][None].double().cpu().numpy()])
+                for g in range(G):
+                    hq = h * G + g
+                    q = x.q[e, l, b, hq].double().cpu().numpy()
+                    o_ref = O.sparse_attention(q, Ka, Va, scale)
+                    assert H.rel_err(outs[e][(l, b)][hq], o_ref) <= 2e-3, (lead, b, h, e, l, hq)
+
+
+def test_full_size_32k_sampled():
+    """The 32k-token LLaMA-3-8B GQA workload at full size (32 layers, 8 kv
+    heads, 8192 kept tokens, a three-level pyramid), three decode steps."""
+    _full_size_sampled(synth.C5, 3, lambda eng, x: [(eng.leaders[2], 0, 3), (eng.leaders[-1], 0, 7)])
+
+
+def test_full_size_batch32_paged_sampled():
+    """The batch-32 paged LLaMA-2-7B workload at full size (32 sequences of
+    1024-4096 tokens, pages of 16 with a shuffled page table, 17 leaders),
+    three decode steps; the sampled sequences are the shortest and the
+    longest of the batch."""
+    def pick(eng, x):
+        lens = x.prompt_lens.tolist()
+        bs, bl = lens.index(min(lens)), lens.index(max(lens))
+        return [(eng.leaders[3], bs, 5), (eng.leaders[-1], bl, 30)]
+    _full_size_sampled(synth.C4, 3, pick)
