@@ -712,3 +712,15 @@ def test_full_size_batch32_paged_sampled():
         bs, bl = lens.index(min(lens)), lens.index(max(lens))
         return [(eng.leaders[3], bs, 5), (eng.leaders[-1], bl, 30)]
     _full_size_sampled(synth.C4, 3, pick)
+
+
+def test_full_size_2k_mha_sampled():
+    """The 2k-token LLaMA-2-7B MHA workload at full size (32 layers, 32 kv
+    heads, a two-level pyramid, groups of two layers), three decode steps."""
+    _full_size_sampled(synth.C2, 3, lambda eng, x: [(eng.leaders[1], 0, 0), (eng.leaders[-1], 0, 31)])
+
+
+def test_full_size_8k_gqa_sampled():
+    """The 8k-token LLaMA-3-8B GQA workload at full size (32 layers, 8 kv
+    heads, a two-level pyramid, groups of four layers), three decode steps."""
+    _full_size_sampled(synth.C3, 3, lambda eng, x: [(eng.leaders[0], 0, 1), (eng.leaders[-2], 0, 6)])
