@@ -391,12 +391,14 @@ __global__ void __launch_bounds__(WPC * 32, 1) attn_bf16_persist_kernel(const __
       const int b = b0 + lane;
       int nt = 0, n = 0, k1 = 0;
       if (b < B) {
+        // both counts are requested at once (one round trip, not two)
         n = p.n_tok[b];
+        const int ns = p.sel_cap > 0 ? p.n_sel[b] : 0;
         if (n < 0 || n + 1 > p.cap_tokens) {
           atomicOr(&g_mpc_status, 2);  // no room for the append: skip the sequence
         } else {
           const int C1 = n / s;
-          k1 = p.sel_cap > 0 ? min(p.n_sel[b], min(C1, p.sel_cap)) : 0;
+          k1 = min(ns, min(C1, p.sel_cap));
           nt = (k1 * s + (n - C1 * s) + 1 + 15) / 16;
         }
       }
