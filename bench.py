@@ -366,14 +366,14 @@ def run_ours(args, rank, world, dist):
     dec_bytes = kv_bytes + rep_bytes + io_bytes
     decode_gbs = dec_bytes / (decode_ms / 1e3) / 1e9
     dominant_static = static_ms >= decode_ms
-    # bf16 keys score on tcgen05, dense or in pages of 8..128 rows dividing 128
-    tensor_path = w.dtype == "bf16" and (not w.paged or (w.page_size >= 8 and 128 % w.page_size == 0))
+    # bf16 keys score on tcgen05 (paged keys through their gathered dense copy)
+    tensor_path = w.dtype == "bf16"
     # DRAM bytes of one static-eviction call (both score passes), from ncu on
     # the 8k workload (profiles/score_tc_kernel_c3_llama3_8b_t8192.md): each
     # pass reads its inputs once, so the 32k figure is that capture scaled by
     # the input bytes (939.5 / 302.1 MB).  Valid for the kernel as captured.
-    static_traffic = {"c3_llama3_8b_gqa_t8192": 628.9e6,
-                      "c5_llama3_8b_gqa_t32768_needles": 628.9e6 * 939.5 / 302.1}.get(w.name)
+    static_traffic = {"c3_llama3_8b_gqa_t8192": 628.1e6,
+                      "c5_llama3_8b_gqa_t32768_needles": 628.1e6 * 939.5 / 302.1}.get(w.name)
     if dominant_static and tensor_path:
         # tcgen05 score passes; the kernel runs inside a long step, so the
         # sustained bf16 figure is the denominator
