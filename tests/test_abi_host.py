@@ -168,6 +168,16 @@ def test_select_and_static_validation(lib):
     assert _ws(lib, "mpc_static_evict_workspace_size", a)[0] == mpcache.MPC_ERR_BAD_SHAPE
     a.win_rows, a.keep_cap = 4916, 8191
     assert _ws(lib, "mpc_static_evict_workspace_size", a)[0] == mpcache.MPC_ERR_BAD_SHAPE
+    # paged bf16 keys: the statistics, then the dense copy of the refs' keys
+    # (n_refs * batch * n_kv_heads * t_max * d bf16) the tensor-core passes read
+    a.keep_cap = 8192
+    pt = (C.c_int32 * 1)(0)
+    a.k.page_table, a.k.page_size, a.k.max_pages = C.cast(pt, C.c_void_p), 16, 2048
+    rc, n = _ws(lib, "mpc_static_evict_workspace_size", a)
+    assert rc == 0 and n == 1 * 2 * 8 * 4992 * (4 + 16) + 1 * 2 * 2 * 32768 * 128 * 2
+    a.dtype = mpcache.MPC_F32  # fp32 keys stay paged (SIMT passes): no copy
+    rc, n = _ws(lib, "mpc_static_evict_workspace_size", a)
+    assert rc == 0 and n == 1 * 2 * 8 * 4992 * (4 + 16)
 
 
 def test_summary_rows(lib):
