@@ -395,13 +395,7 @@ def run_ours(args, rank, world, dist):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": w.dtype, "data": "synthetic (seeded generator, workload recipe in DESIGN.md)",
-        "config": {"workload": w.name, "layers": w.n_layers, "batch": w.batch, "q_heads": w.n_q_heads,
-                   "kv_heads": w.n_kv_heads, "head_dim": w.head_dim, "prompt_len": w.prompt_len,
-                   "decode_steps": E, "cluster_size": w.cluster_size, "fanouts": list(w.fanouts),
-                   "level_keep_ppm": list(w.level_keep_ppm), "keep_ppm": w.keep_ppm,
-                   "share_every": w.share_every, "parallelism": f"replicas{world}",
-                   "l2": "inputs larger than L2 (prompt KV %.1f GB per step)" % (
-                       (x.k.numel() + x.v.numel()) * x.k.element_size() / 1e9)},
+        "config": workload_config(w, E, f"replicas{world}"),
         "gpu_launches": args.steps * (3 + 1 + (1 if len(w.fanouts) else 0) + 2 * E),
         "static_scoring_path": "tcgen05" if tensor_path else "simt",
         "phases_ms": {"static_evict": static_ms, "build_clusters": build_ms, "decode_all_steps": decode_ms},
@@ -479,6 +473,17 @@ def oracle_sample(w, E_sample=4):
             "sample": sample, "seconds": t1 - t0 + t_build + t_dec, "whole_job_s_estimate": whole}
 
 
+def workload_config(w, E, parallelism):
+    """The bench line's ``config``: the workload by its sizes (both arms)."""
+    kv_gb = 2 * w.n_layers * w.batch * w.n_kv_heads * w.prompt_len * w.head_dim * (2 if w.dtype == "bf16" else 4) / 1e9
+    return {"workload": w.name, "layers": w.n_layers, "batch": w.batch, "q_heads": w.n_q_heads,
+            "kv_heads": w.n_kv_heads, "head_dim": w.head_dim, "prompt_len": w.prompt_len,
+            "decode_steps": E, "cluster_size": w.cluster_size, "fanouts": list(w.fanouts),
+            "level_keep_ppm": list(w.level_keep_ppm), "keep_ppm": w.keep_ppm,
+            "share_every": w.share_every, "paged": w.paged, "parallelism": parallelism,
+            "l2": "inputs larger than L2 (prompt KV up to %.1f GB per step)" % kv_gb}
+
+
 def run_reference(args, rank, world):
     if rank != 0:
         return None
@@ -494,7 +499,7 @@ def run_reference(args, rank, world):
     return {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": statistics.median(secs) * 1e3,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": w.name, "parallelism": "cpu"},
+            "data": "synthetic", "config": workload_config(w, args.decode_steps or w.decode_steps, "cpu"),
             "cpu_baseline": {"value": v, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
                              "sample": r["sample"]},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
