@@ -45,7 +45,7 @@ FFMA_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
 def parse_args():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=5)
+    p.add_argument("--steps", type=int, default=20)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default=synth.C5.name, choices=sorted(synth.WORKLOADS))
@@ -138,10 +138,14 @@ class ClockSampler:
         self.proc = None
 
     def start(self):
+        """Starts sampling every 50 ms and returns once the first sample is
+        out (nvidia-smi takes a while to start), so that the samples read at
+        stop() fall inside the region between the two calls."""
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", "50"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.proc.stdout.readline()
         except Exception:
             self.proc = None
 
@@ -266,9 +270,11 @@ def run_ours(args, rank, world, dist):
     # once its copies have landed.  A gather stream then builds the group's
     # caches from its kept rows (the leader's keys from the device, every
     # other key and value row straight from pinned host memory, so evicted
-    # rows never cross the host link) while the next leaders are scored; the
-    # last group, whose gather would end the prefill, gathers from its device
-    # copy.  Non-leader window queries are never read, so they are not copied.
+    # rows never cross the host link) while the next leaders are scored.
+    # When the link has time to spare during scoring, the last group, whose
+    # gather would end the prefill, is copied whole and gathers from the
+    # device.  Non-leader window queries are never read, so they are not
+    # copied.
     e2e = None
     if not args.no_e2e:
         host = {n: getattr(x, n).cpu().pin_memory() for n in ("k", "v", "q_win", "q", "k_new", "v_new")}
@@ -281,10 +287,16 @@ def run_ours(args, rank, world, dist):
         esz_kv = host["k"].element_size()
         kept_rows = sum(int(t) for t in eng.n_keep.tolist()) * w.n_kv_heads  # per layer
         n_last = sum(1 for l in range(w.n_layers) if eng.group_of[l] == eng.group_of[leaders[-1]])
-        gathered = kept_rows * w.head_dim * esz_kv * (len(leaders) - 1 + 2 * (w.n_layers - len(leaders) - (n_last - 1)))
-        whole_last = (2 * n_last - 1) * host["k"][0].numel() * esz_kv  # the last group's other K and all V
-        h2d = (sum(src.numel() * src.element_size() for _, src in copies + decode_in) +
-               host_lens.numel() * 4 + gathered + whole_last)
+        row_bytes = kept_rows * w.head_dim * esz_kv  # one layer's kept K (or V) rows
+        gathered = row_bytes * (len(leaders) + 2 * (w.n_layers - len(leaders)))
+        copied = sum(src.numel() * src.element_size() for _, src in copies + decode_in) + host_lens.numel() * 4
+        # the last group whole: its other layers' K and every V, instead of
+        # their kept rows; worth it if the link (about 200 GB/s) still idles
+        # while the leaders are scored
+        whole_last = (2 * n_last - 1) * host["k"][0].numel() * esz_kv
+        last_kept = row_bytes * (1 + 2 * (n_last - 1))
+        last_whole = (copied + gathered - last_kept + whole_last) / 200e6 < static_ms
+        h2d = copied + gathered + (whole_last - last_kept if last_whole else 0)
         d2h = out_host.numel() * out_host.element_size()
         side = torch.cuda.Stream(device=dev)
         gat = torch.cuda.Stream(device=dev)
@@ -310,17 +322,18 @@ def run_ours(args, rank, world, dist):
                     landed[i].record(side)
                 for dst, src in decode_in:
                     dst.copy_(src, non_blocking=True)
-                for l in last:
-                    if l != leaders[-1]:  # the leader's keys are already there
-                        x.k[l].copy_(host["k"][l], non_blocking=True)
-                    x.v[l].copy_(host["v"][l], non_blocking=True)
+                if last_whole:
+                    for l in last:
+                        if l != leaders[-1]:  # the leader's keys are already there
+                            x.k[l].copy_(host["k"][l], non_blocking=True)
+                        x.v[l].copy_(host["v"][l], non_blocking=True)
                 last_landed.record(side)
             for i, batch in enumerate(batches):
                 stream.wait_event(landed[i])
                 eng.static_evict(x.k, x.q_win, lens, pt, w.page_size, layers=batch)
                 gat.wait_stream(stream)
                 with torch.cuda.stream(gat):
-                    if i == len(batches) - 1:
+                    if i == len(batches) - 1 and last_whole:
                         gat.wait_event(last_landed)
                         eng.build_clusters(x.k, x.v, pt, w.page_size, layers=last)
                         continue
@@ -351,7 +364,8 @@ def run_ours(args, rank, world, dist):
         e2e_ms = max_over_ranks(statistics.median(per), dist, dev)
         e2e = {"value": job_value(attended, world, e2e_ms), "unit": UNIT, "ms_per_step": e2e_ms,
                "ms_per_step_mean": max_over_ranks(sum(per) / len(per), dist, dev),
-               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+               "last_group_copied_whole": bool(last_whole)}
 
     pk, pk_kind = peaks()
     n_lead = len(leaders)
