@@ -386,23 +386,27 @@ def test_fixed_point_ranking_survives_on_needle_workload():
 # ----------------------------------------------- static eviction alone ----
 
 STATIC_CASES = [
-    # dtype, d, Hq, Hkv, lens, keep_ppm, paged
-    (torch.float32, 64, 4, 4, (512,), 500_000, False),
-    (torch.bfloat16, 128, 8, 2, (1000,), 250_000, False),
-    (torch.bfloat16, 64, 2, 1, (129, 300, 64), 500_000, False),
-    (torch.bfloat16, 128, 4, 4, (777, 1500), 125_000, True),
-    (torch.float32, 128, 2, 2, (33,), 1_000_000, False),
-    (torch.bfloat16, 128, 4, 1, (1,), 500_000, False),
+    # dtype, d, Hq, Hkv, lens, keep_ppm, page size (0: dense keys)
+    (torch.float32, 64, 4, 4, (512,), 500_000, 0),
+    (torch.bfloat16, 128, 8, 2, (1000,), 250_000, 0),
+    (torch.bfloat16, 64, 2, 1, (129, 300, 64), 500_000, 0),
+    (torch.bfloat16, 128, 4, 4, (777, 1500), 125_000, 16),
+    (torch.float32, 128, 2, 2, (33,), 1_000_000, 0),
+    (torch.bfloat16, 128, 4, 1, (1,), 500_000, 0),
+    (torch.bfloat16, 128, 4, 2, (300, 1000), 250_000, 4),     # pages smaller than a swizzle atom
+    (torch.bfloat16, 64, 8, 2, (777, 129), 500_000, 48),      # pages that do not divide 128
+    (torch.bfloat16, 128, 2, 2, (1500,), 125_000, 256),       # pages larger than a key tile
+    (torch.float32, 64, 4, 2, (500, 333), 500_000, 32),       # fp32 keys: paged SIMT passes
 ]
 
 
-@pytest.mark.parametrize("dtype,d,Hq,Hkv,lens,keep,paged", STATIC_CASES)
-def test_static_eviction(dtype, d, Hq, Hkv, lens, keep, paged):
+@pytest.mark.parametrize("dtype,d,Hq,Hkv,lens,keep,page", STATIC_CASES)
+def test_static_eviction(dtype, d, Hq, Hkv, lens, keep, page):
     g = torch.Generator().manual_seed(sum(lens) + d)
     B, T = len(lens), max(lens)
     G = Hq // Hkv
     w = synth.Workload("t", 1, B, Hq, Hkv, d, "f32" if dtype == torch.float32 else "bf16", T, min(lens),
-                       keep, 16, (), (O.PPM,), 1, 1, "iid", paged=paged)
+                       keep, 16, (), (O.PPM,), 1, 1, "iid", paged=page > 0)
     eng = H.make_engine(w, 1)
     R = eng.win_rows
     K = torch.zeros((1, B, Hkv, T, d))
@@ -412,8 +416,8 @@ def test_static_eviction(dtype, d, Hq, Hkv, lens, keep, paged):
         Q[0, b, :, R - min(R, t):] = torch.randn((Hq, min(R, t), d), generator=g) * 1.5
     K, Q = K.to(dtype), Q.to(dtype)
     lens_t = torch.tensor(lens, dtype=torch.int32)
-    if paged:
-        P = 16
+    if page:
+        P = page
         n_pages = [(t + P - 1) // P for t in lens]
         perm = torch.randperm(sum(n_pages), generator=g).to(torch.int32)
         pt = torch.full((B, (T + P - 1) // P), -1, dtype=torch.int32)
