@@ -410,7 +410,10 @@ def run_ours(args, rank, world, dist):
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": w.dtype, "data": "synthetic (seeded generator, workload recipe in DESIGN.md)",
         "config": workload_config(w, E, f"replicas{world}"),
-        "gpu_launches": args.steps * (3 + 1 + (1 if len(w.fanouts) else 0) + 2 * E),
+        # per step: static eviction (two score passes + budget, plus the gather
+        # of paged bf16 keys), gathering (+ coarse levels), two per decode step
+        "gpu_launches": args.steps * (3 + (1 if w.paged and w.dtype == "bf16" else 0) + 1 +
+                                      (1 if len(w.fanouts) else 0) + 2 * E),
         "static_scoring_path": "tcgen05" if tensor_path else "simt",
         "phases_ms": {"static_evict": static_ms, "build_clusters": build_ms, "decode_all_steps": decode_ms},
         "decode_step_us": decode_ms / E * 1e3,
