@@ -103,8 +103,10 @@ C5 = Workload("c5_llama3_8b_gqa_t32768_needles", 32, 1, 32, 8, 128, "bf16",
               32768, 32768, 250_000, 16, (8, 8), (50_000, 250_000, 500_000), 4,
               256, "needle", seed=1005)
 
-WORKLOADS = {w.name: w for w in (C1, C2, C3, C4, C5)}
 C4_BATCHES = (1, 4, 16, 32)
+# the batched paged workload at its other batch sizes (same seed and rule)
+C4_VARIANTS = tuple(C4.replace(name=f"c4_llama2_7b_paged_b{b}", batch=b) for b in C4_BATCHES if b != C4.batch)
+WORKLOADS = {w.name: w for w in (C1, C2, C3, C4, C5) + C4_VARIANTS}
 
 
 @dataclass
