@@ -397,6 +397,7 @@ STATIC_CASES = [
     (torch.bfloat16, 64, 8, 2, (777, 129), 500_000, 48),      # pages that do not divide 128
     (torch.bfloat16, 128, 2, 2, (1500,), 125_000, 256),       # pages larger than a key tile
     (torch.float32, 64, 4, 2, (500, 333), 500_000, 32),       # fp32 keys: paged SIMT passes
+    (torch.bfloat16, 128, 2, 1, (49152,), 250_000, 0),        # the longest prompt the calls accept
 ]
 
 
@@ -728,3 +729,13 @@ def test_full_size_8k_gqa_sampled():
     """The 8k-token LLaMA-3-8B GQA workload at full size (32 layers, 8 kv
     heads, a two-level pyramid, groups of four layers), three decode steps."""
     _full_size_sampled(synth.C3, 3, lambda eng, x: [(eng.leaders[0], 0, 1), (eng.leaders[-2], 0, 6)])
+
+
+def test_pipeline_prompt_shorter_than_a_cluster():
+    """Degenerate start: 12 prompt tokens (< s = 16), so the pyramid is empty
+    and selection has no candidate; attention covers the tail alone until the
+    decode appends seal the first cluster (step 4), after which it becomes
+    selectable."""
+    w = synth.C3.replace(n_layers=2, prompt_len=12, prompt_len_min=12, n_q_heads=4, n_kv_heads=2,
+                         keep_ppm=1_000_000, fanouts=(2,), share_every=1)
+    _pipeline(w, 24, [0, 1], max_skip=0.0)
