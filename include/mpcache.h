@@ -244,6 +244,9 @@ typedef struct {
  *   3. if the tail now holds s rows it is sealed as cluster C_1: leaders
  *      write its r_max / r_min / rep and merge it into the coarser levels;
  *   4. if `advance` is nonzero, n_tok[b] += 1 once all refs are done.
+ * A sequence with no row left for the append (n + 1 > cap_tokens) is
+ * skipped on the device: nothing is written, n_tok[b] stays, and the device
+ * status word gets flag 2 (see mpc_device_status).
  * Outputs o[layer][b][n_q_heads][d] float32. */
 typedef struct {
   uint32_t struct_size;        /* sizeof(mpc_attn_args) */

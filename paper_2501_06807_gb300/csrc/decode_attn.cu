@@ -283,7 +283,11 @@ __device__ __forceinline__ void finish_grid(const AttnParams& p) {
     const int ticket = atomicAdd(p.grid_counter, 1);
     if (ticket == total - 1) {
       __threadfence();
-      for (int b = 0; b < p.B; ++b) p.n_tok[b] += 1;
+      // a sequence whose append was refused (no room left) keeps its count
+      for (int b = 0; b < p.B; ++b) {
+        const int n = p.n_tok[b];
+        if (n >= 0 && n + 1 <= p.cap_tokens) p.n_tok[b] = n + 1;
+      }
       *p.grid_counter = 0;
     }
   }

@@ -739,3 +739,26 @@ def test_pipeline_prompt_shorter_than_a_cluster():
     w = synth.C3.replace(n_layers=2, prompt_len=12, prompt_len_min=12, n_q_heads=4, n_kv_heads=2,
                          keep_ppm=1_000_000, fanouts=(2,), share_every=1)
     _pipeline(w, 24, [0, 1], max_skip=0.0)
+
+
+def test_decode_past_capacity_is_refused_and_flagged():
+    """A decode step with no cache row left for its append is refused on the
+    device: no row is written, the token count stays, and the status word
+    reports it (flag 2) until read."""
+    w = synth.C3.replace(n_layers=1, prompt_len=32, prompt_len_min=32, n_q_heads=2, n_kv_heads=1,
+                         keep_ppm=1_000_000, fanouts=(), level_keep_ppm=(500_000,), share_every=1)
+    x = H.to_cuda(synth.generate(w, H.window_rows_for(w), device="cpu", decode_steps=34))
+    eng = H.make_engine(w, 2)
+    eng.prefill(x.k, x.v, x.q_win, x.prompt_lens.cuda(), None, w.page_size)
+    cap = eng.cap_tokens
+    steps = cap - 32
+    for e in range(steps):
+        eng.decode_step(x.q[e], x.k_new[e], x.v_new[e])
+    assert mpcache.device_status() == 0
+    assert int(eng.n_tok[0]) == cap
+    kc = eng.kc.clone()
+    eng.decode_step(x.q[steps], x.k_new[steps], x.v_new[steps])
+    assert mpcache.device_status() & 2
+    assert int(eng.n_tok[0]) == cap
+    assert torch.equal(eng.kc, kc)
+    assert mpcache.device_status() == 0  # read and cleared
