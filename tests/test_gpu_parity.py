@@ -762,3 +762,28 @@ def test_decode_past_capacity_is_refused_and_flagged():
     assert int(eng.n_tok[0]) == cap
     assert torch.equal(eng.kc, kc)
     assert mpcache.device_status() == 0  # read and cleared
+
+
+def test_corrupt_indices_are_reported_not_followed():
+    """Indices outside their range (a selected cluster id past the sealed
+    clusters, a kept position past the prompt) are reported in the device
+    status word (flag 4) and never used as addresses: the outputs stay
+    finite and the status clears once read."""
+    w = synth.C3.replace(n_layers=1, prompt_len=256, prompt_len_min=256, n_q_heads=2, n_kv_heads=1,
+                         keep_ppm=1_000_000, fanouts=(), level_keep_ppm=(250_000,), share_every=1)
+    x = H.to_cuda(synth.generate(w, H.window_rows_for(w), device="cpu", decode_steps=2))
+    eng = H.make_engine(w, 2)
+    eng.prefill(x.k, x.v, x.q_win, x.prompt_lens.cuda(), None, w.page_size)
+    assert mpcache.device_status() == 0
+    # a selected id past the 16 sealed clusters
+    eng.select(x.q[0])
+    eng.sel[0, 0, 0, 0] = 1_000_000
+    eng.attend(x.q[0], x.k_new[0], x.v_new[0], advance=False)
+    assert mpcache.device_status() & 4
+    assert torch.isfinite(eng.out).all()
+    assert mpcache.device_status() == 0
+    # a kept position past the prompt
+    eng.kept[0, 0, 0, 5] = 1_000_000
+    eng.build_clusters(x.k, x.v, None, w.page_size)
+    assert mpcache.device_status() & 4
+    assert mpcache.device_status() == 0
