@@ -355,6 +355,13 @@ MPC_API const char* mpc_last_error(void);
  * device (cudaDeviceSynchronize), returns the flags and clears them. */
 MPC_API int mpc_device_status(int* flags);
 
+/* Failure-path self-test: launches one kernel whose wait is never
+ * satisfied (kind 0: an mbarrier nothing completes; kind 1: the device int
+ * never_set, which the caller keeps 0, polled with acquire loads) and gives
+ * up after limit_us microseconds (1 .. 1e6), setting flag 1 of the device
+ * status word; the context stays usable.  Asynchronous on `stream`. */
+MPC_API int mpc_selftest_wait(int32_t kind, int32_t limit_us, const int32_t* never_set, void* stream);
+
 /* MPC_ABI_VERSION of the loaded library. */
 MPC_API int mpc_abi_version(void);
 

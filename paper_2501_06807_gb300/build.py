@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(OUT_DIR, "libmpcache.so")
 SOURCES = ["abi.cu", "decode_attn.cu", "select.cu", "clusters.cu", "static_evict.cu", "score_tc.cu",
-           "no_alloc.cu", "commonality.cu"]
+           "no_alloc.cu", "commonality.cu", "selftest.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "--expt-relaxed-constexpr", "-Xcompiler", "-fPIC",
          "-Xcompiler", "-fvisibility=hidden", "-Xptxas", "-warn-spills"]

@@ -430,12 +430,23 @@ MPC_API int64_t mpc_summary_rows(int32_t cap_tokens, int32_t cluster_size, int32
   return p.rows;
 }
 
+MPC_API int mpc_selftest_wait(int32_t kind, int32_t limit_us, const int32_t* never_set, void* stream) {
+  if (kind != 0 && kind != 1) return fail(MPC_ERR_INVALID_ARG, "kind %d is not 0 (mbarrier) or 1 (flag)", kind);
+  if (limit_us < 1 || limit_us > 1000000) return fail(MPC_ERR_BAD_SHAPE, "limit_us %d not in [1, 1e6]", limit_us);
+  if (kind == 1 && never_set == nullptr) return fail(MPC_ERR_INVALID_ARG, "kind 1 needs never_set");
+  const cudaError_t e = launch_wait_selftest(kind, never_set, (uint64_t)limit_us * 1000ull,
+                                             static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "mpc_selftest_wait launch");
+  return ok();
+}
+
 MPC_API int mpc_device_status(int* flags) {
   if (flags == nullptr) return fail(MPC_ERR_INVALID_ARG, "flags is NULL");
   const cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
-  const int parts[6] = {take_status_attn(),   take_status_select(),   take_status_clusters(),
-                        take_status_static(), take_status_score_tc(), take_status_commonality()};
+  const int parts[7] = {take_status_attn(),   take_status_select(),   take_status_clusters(),
+                        take_status_static(), take_status_score_tc(), take_status_commonality(),
+                        take_status_selftest()};
   int v = 0;
   for (int x : parts) {
     if (x < 0) return fail(MPC_ERR_CUDA, "reading the device status word failed");

@@ -205,8 +205,6 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
   return true;
 }
 
-// 1-D bulk copy global -> shared (TMA engine), completion counted on `bar`.
-// dst, src 16-byte aligned; bytes a multiple of 16.
 // 16-byte asynchronous copy global -> shared (cached in L2 only), and its
 // commit / wait-group pair.
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
@@ -218,6 +216,8 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
+// 1-D bulk copy global -> shared (TMA engine), completion counted on `bar`.
+// dst, src 16-byte aligned; bytes a multiple of 16.
 __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
   asm volatile(
       "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(

@@ -157,6 +157,8 @@ int static_tile_smem(int D);
 // Records `msg` as this thread's last error (mpc_last_error) and returns code.
 int set_error(int code, const char* msg);
 int take_status_commonality();
+int take_status_selftest();
+cudaError_t launch_wait_selftest(int kind, const int* never_set, uint64_t limit_ns, cudaStream_t st);
 
 // Device status word of each translation unit: read it and clear it.
 int take_status_attn();

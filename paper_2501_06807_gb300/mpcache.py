@@ -104,7 +104,7 @@ ENTRY_POINTS = ("mpc_static_evict_workspace_size", "mpc_build_clusters_workspace
                 "mpc_select_workspace_size", "mpc_sparse_decode_attn_workspace_size",
                 "mpc_static_evict", "mpc_build_clusters", "mpc_select", "mpc_sparse_decode_attn",
                 "mpc_summary_rows", "mpc_last_error", "mpc_device_status", "mpc_abi_version",
-                "mpc_sparse_decode_attn_static_scratch", "mpc_commonality")
+                "mpc_sparse_decode_attn_static_scratch", "mpc_commonality", "mpc_selftest_wait")
 
 _LIB = None
 
@@ -139,6 +139,8 @@ def load(path: Optional[str] = None) -> C.CDLL:
     lib.mpc_sparse_decode_attn_static_scratch.argtypes = [C.c_void_p, C.c_void_p]
     lib.mpc_commonality.restype = C.c_int
     lib.mpc_commonality.argtypes = [C.c_void_p, C.c_void_p]
+    lib.mpc_selftest_wait.restype = C.c_int
+    lib.mpc_selftest_wait.argtypes = [C.c_int32, C.c_int32, C.c_void_p, C.c_void_p]
     if lib.mpc_abi_version() != ABI_VERSION:
         raise MPCError(MPC_ERR_INVALID_ARG,
                        f"libmpcache ABI {lib.mpc_abi_version()} does not match the binding's {ABI_VERSION}")
@@ -263,6 +265,13 @@ def device_status() -> int:
     v = C.c_int(0)
     _check(load().mpc_device_status(C.byref(v)))
     return v.value
+
+
+def selftest_wait(kind: int, limit_us: int, never_set: Optional[torch.Tensor] = None) -> None:
+    """Launches the failure-path self-test: a wait that is never satisfied
+    (kind 0: an mbarrier; kind 1: ``never_set``, a device int32 kept 0) gives
+    up after ``limit_us`` and sets flag 1 of the device status word."""
+    _check(load().mpc_selftest_wait(kind, limit_us, C.c_void_p(_ptr(never_set)), C.c_void_p(_stream())))
 
 
 # -------------------------------------------------------------- engine ----

@@ -202,6 +202,14 @@ def test_missing_library_fails_loudly(tmp_path):
         mpcache.load(str(tmp_path / "nope.so"))
 
 
+def test_selftest_wait_validation(lib):
+    # checked before any launch: kind, the limit's range, the flag pointer
+    assert lib.mpc_selftest_wait(2, 1000, None, None) == mpcache.MPC_ERR_INVALID_ARG
+    assert lib.mpc_selftest_wait(0, 0, None, None) == mpcache.MPC_ERR_BAD_SHAPE
+    assert lib.mpc_selftest_wait(0, 1_000_001, None, None) == mpcache.MPC_ERR_BAD_SHAPE
+    assert lib.mpc_selftest_wait(1, 1000, None, None) == mpcache.MPC_ERR_INVALID_ARG
+
+
 def test_commonality_validation(lib):
     a = mpcache.CommonalityArgs()
     a.struct_size = C.sizeof(mpcache.CommonalityArgs)

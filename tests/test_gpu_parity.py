@@ -787,3 +787,17 @@ def test_corrupt_indices_are_reported_not_followed():
     eng.build_clusters(x.k, x.v, None, w.page_size)
     assert mpcache.device_status() & 4
     assert mpcache.device_status() == 0
+
+
+@pytest.mark.parametrize("kind", [0, 1])
+def test_bounded_wait_runs_out_and_reports(kind):
+    """A wait that nothing satisfies (an mbarrier, or a flag that nothing
+    sets) gives up after its limit, sets flag 1 of the status word and
+    returns; the context stays usable for the next call."""
+    never = torch.zeros(1, dtype=torch.int32, device="cuda")
+    assert mpcache.device_status() == 0
+    mpcache.selftest_wait(kind, 2000, never)
+    assert mpcache.device_status() & 1
+    assert mpcache.device_status() == 0
+    x = torch.arange(8, device="cuda") * 2  # the context still runs work
+    assert int(x.sum()) == 56
