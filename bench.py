@@ -408,7 +408,7 @@ def run_ours(args, rank, world, dist):
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": w.dtype, "data": "synthetic (seeded generator, workload recipe in DESIGN.md)",
+        "vs_baseline": None, "dtype": w.dtype, "data": "synthetic (seeded generator shaped like the paper's models; no datasets or weights)",
         "config": workload_config(w, E, f"replicas{world}"),
         # per step: static eviction (two score passes + budget, plus the gather
         # of paged bf16 keys), gathering (+ coarse levels), two per decode step

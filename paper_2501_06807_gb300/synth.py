@@ -88,8 +88,8 @@ class Workload:
         return dataclasses.replace(self, **kw)
 
 
-# configs[0..4] of the workload table: GPT-2-small, LLaMA-2-7B, LLaMA-3-8B GQA,
-# batched paged LLaMA-2-7B, 32k-token LLaMA-3-8B GQA with needles.
+# The five workloads: GPT-2-small, LLaMA-2-7B, LLaMA-3-8B GQA, batched paged
+# LLaMA-2-7B, 32k-token LLaMA-3-8B GQA with needles.
 C1 = Workload("c1_gpt2_small_t512", 1, 1, 12, 12, 64, "f32", 512, 512,
               500_000, 16, (), (250_000,), 1, 8, "iid", seed=1001)
 C2 = Workload("c2_llama2_7b_t2048", 32, 1, 32, 32, 128, "bf16", 2048, 2048,
