@@ -431,6 +431,36 @@ def test_fxp_error_within_rounding_bound(fb):
     assert err.max() > bound.max() / 200  # and the bound not vacuous
 
 
+def test_fxp_ring_wraps_like_two_complement_int64():
+    # f = 24 and values near 2^9: products of encodings near 2^66 leave the
+    # int64 range; the ring arithmetic must equal Python big integers reduced
+    # modulo 2^64 (two's complement), with floor division for truncation
+    rng = np.random.default_rng(31)
+    G, d, C, f, a = 3, 16, 6, 24, 0.6
+    qg = rng.uniform(-600, 600, (G, d))
+    rmin = rng.uniform(-600, 0, (C, d))
+    rmax = rmin + rng.uniform(0, 600, (C, d))
+    M = 1 << 64
+
+    def wrap(v):
+        v %= M
+        return v - M if v >= 1 << 63 else v
+
+    one = 1 << f
+    q = [wrap(sum(round(float(qg[g, i]) * one) for g in range(G))) for i in range(d)]
+    ea, eb = round(a * one), round((1 - a) * one)
+    want = []
+    wrapped = False
+    for c in range(C):
+        rep = [wrap(wrap(ea * round(float(rmax[c, i]) * one)) // one + wrap(eb * round(float(rmin[c, i]) * one)) // one)
+               for i in range(d)]
+        full = sum(q[i] * rep[i] for i in range(d))
+        wrapped |= abs(full) >= 1 << 63
+        want.append(min(max(wrap(full) // one, -(1 << 31)), (1 << 31) - 1))
+    assert wrapped  # the case exercises the wrap
+    assert O.sim_fxp(qg, rmax, rmin, a, f).tolist() == want
+
+
 def test_fxp_saturates_to_int32():
     # scores beyond the int32 range of the ranking key saturate (equal keys
     # then rank the lower id first)
