@@ -259,14 +259,42 @@ __global__ void __launch_bounds__(kBudgetThreads) budget_kernel(const __grid_con
       if ((k & mask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1);
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-      int cum = 0, dg = 0;
-      for (dg = 255; dg > 0; --dg) {
-        if (cum + hist[dg] >= remaining) break;
-        cum += hist[dg];
+    if (threadIdx.x < 32) {
+      // the largest digit d whose suffix count S[d] = sum_{d' >= d} hist[d']
+      // reaches `remaining` (d = 0 if none above 0 does), and S[d + 1]:
+      // lane l holds digits 8l .. 8l + 7, the suffix runs over the lanes
+      const int lane = threadIdx.x;
+      int h[8], local = 0;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        h[i] = hist[lane * 8 + i];
+        local += h[i];
       }
-      s_digit = dg;
-      s_above = cum;
+      int incl = local;  // sum over lanes >= lane
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_down_sync(0xffffffffu, incl, o);
+        if (lane + o < 32) incl += y;
+      }
+      int run = incl - local, found = -1, above = 0;  // run = S[8 lane + 8]
+#pragma unroll
+      for (int i = 7; i >= 0; --i) {
+        if (found < 0 && lane * 8 + i > 0 && run + h[i] >= remaining) {
+          found = lane * 8 + i;
+          above = run;
+        }
+        run += h[i];
+      }
+      const unsigned bal = __ballot_sync(0xffffffffu, found >= 0);
+      if (bal != 0) {
+        if (lane == 31 - __clz(bal)) {
+          s_digit = found;
+          s_above = above;
+        }
+      } else if (lane == 0) {
+        s_digit = 0;
+        s_above = incl - h[0];  // S[1]
+      }
     }
     __syncthreads();
     remaining -= s_above;
