@@ -135,7 +135,7 @@ typedef struct {
                                   row r is prompt position T_b - win_rows + r */
   int64_t q_win_layer_stride;  /* elements */
   int32_t win_rows;            /* >= every w_b */
-  mpc_kv_tensor k;
+  mpc_kv_tensor k;             /* device memory: host memory is refused (INVALID_ARG) */
   int32_t window_ppm, long_window_ppm, long_prompt_threshold;
   int32_t keep_ppm;
   float scale;                 /* 0 selects 1/sqrt(d) */

@@ -456,6 +456,16 @@ MPC_API int mpc_device_status(int* flags) {
   return ok();
 }
 
+// True for pinned host memory reached through unified addressing.
+static bool is_host_memory(const void* ptr) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, ptr) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeHost;
+}
+
 MPC_API int mpc_static_evict_workspace_size(const mpc_static_args* args, size_t* bytes) {
   if (bytes == nullptr) return fail(MPC_ERR_INVALID_ARG, "bytes is NULL");
   StaticParams p;
@@ -469,6 +479,9 @@ MPC_API int mpc_static_evict(const mpc_static_args* args, void* workspace, size_
   MPC_TRY(validate_static(args, &p));
   if (!args->q_win || !args->k.data || !args->prompt_lens || !args->out_scores || !args->out_kept || !args->out_n_keep)
     return fail(MPC_ERR_INVALID_ARG, "a required pointer is NULL");
+  // the tensor-core passes read keys and window queries through TMA tensor maps
+  if (is_host_memory(args->k.data) || is_host_memory(args->q_win))
+    return fail(MPC_ERR_INVALID_ARG, "k and q_win must be device memory, not host memory");
   const size_t need = static_ws(p, args->dtype, args->head_dim);
   if (workspace == nullptr || workspace_bytes < need)
     return fail(MPC_ERR_WORKSPACE, "workspace of %zu bytes needed", need);
@@ -484,16 +497,6 @@ MPC_API int mpc_static_evict(const mpc_static_args* args, void* workspace, size_
   const cudaError_t e = launch_static(p, args->dtype, args->head_dim, span, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "mpc_static_evict launch");
   return ok();
-}
-
-// True for pinned host memory reached through unified addressing.
-static bool is_host_memory(const void* ptr) {
-  cudaPointerAttributes at;
-  if (cudaPointerGetAttributes(&at, ptr) != cudaSuccess) {
-    (void)cudaGetLastError();
-    return false;
-  }
-  return at.type == cudaMemoryTypeHost;
 }
 
 MPC_API int mpc_build_clusters_workspace_size(const mpc_cluster_args* args, size_t* bytes) {

@@ -168,12 +168,36 @@ def _stream() -> int:
     return torch.cuda.current_stream().cuda_stream
 
 
-def _dtype_code(t: torch.Tensor) -> int:
-    if t.dtype == torch.float32:
+def _dtype_code(dtype: torch.dtype) -> int:
+    if dtype == torch.float32:
         return MPC_F32
-    if t.dtype == torch.bfloat16:
+    if dtype == torch.bfloat16:
         return MPC_BF16
-    raise TypeError(f"unsupported dtype {t.dtype}")
+    raise TypeError(f"unsupported dtype {dtype}: the kernels take float32 or bfloat16")
+
+
+def _check_input(t: torch.Tensor, name: str, dtype: torch.dtype, shape: Sequence[Optional[int]],
+                 min_layers: int = 0, host_ok: bool = False) -> None:
+    """Refuses a tensor that the calls would misread: a dtype other than
+    ``dtype``, sizes other than ``shape`` (None: any size; with
+    ``min_layers``, dim 0 indexes layers and needs at least that many), a
+    layout that is not contiguous after dim 0 (the calls take a stride for
+    dim 0 only), or memory the call cannot read (host memory only where
+    ``host_ok``, and then pinned)."""
+    if t.dtype != dtype:
+        raise TypeError(f"{name}: dtype {t.dtype}, expected {dtype}")
+    want = tuple("*" if e is None else e for e in shape)
+    if t.dim() != len(shape) or any(e is not None and e != n for e, n in zip(shape, t.shape)):
+        raise ValueError(f"{name}: shape {tuple(t.shape)}, expected {want}")
+    if min_layers and t.shape[0] < min_layers:
+        raise ValueError(f"{name}: {t.shape[0]} layers along dim 0, the refs need {min_layers}")
+    step = 1
+    for n, st in zip(reversed(t.shape[1:]), reversed(t.stride()[1:])):
+        if n > 1 and st != step:
+            raise ValueError(f"{name}: dims after the first must be contiguous (strides {t.stride()})")
+        step *= n
+    if not t.is_cuda and not (host_ok and t.is_pinned()):
+        raise ValueError(f"{name}: must be on the GPU" + (" or in pinned host memory" if host_ok else ""))
 
 
 def _refs(refs: Sequence[tuple]):
@@ -288,7 +312,7 @@ class Engine:
         load()
         self.L, self.B, self.Hq, self.Hkv, self.d = n_layers, batch, n_q_heads, n_kv_heads, head_dim
         self.dtype = dtype
-        self.dcode = MPC_BF16 if dtype == torch.bfloat16 else MPC_F32
+        self.dcode = _dtype_code(dtype)
         self.t_max, self.keep_ppm, self.s = t_max, keep_ppm, cluster_size
         self.fanouts = tuple(fanouts)
         self.n_levels = 1 + len(self.fanouts)
@@ -344,6 +368,10 @@ class Engine:
                     page_table: Optional[torch.Tensor] = None, page_size: int = 16,
                     layers: Optional[Sequence[int]] = None) -> StaticArgs:
         lead = self._subset(self.refs_lead, layers)
+        span = 1 + max((r[0] for r in lead), default=-1)
+        self._check_kv(k, "k", page_table, page_size, span, host_ok=False)
+        _check_input(q_win, "q_win", self.dtype, (None, self.B, self.Hq, None, self.d), span)
+        _check_input(lens, "lens", torch.int32, (self.B,))
         refs = _refs(lead)
         a = StaticArgs()
         a.struct_size = C.sizeof(StaticArgs)
@@ -364,6 +392,16 @@ class Engine:
         a.out_scores, a.out_kept, a.out_n_keep = _ptr(self.scores), _ptr(self.kept), _ptr(self.n_keep)
         a._refs = refs
         return a
+
+    def _check_kv(self, t: torch.Tensor, name: str, page_table, page_size: int, span: int, host_ok: bool):
+        """Prompt keys or values: dense [layer][b][kv head][t_max][d], or a
+        page pool [layer][page][kv head][page_size][d] with its page table
+        [b][max_pages] (int32, on the GPU)."""
+        if page_table is None:
+            _check_input(t, name, self.dtype, (None, self.B, self.Hkv, self.t_max, self.d), span, host_ok)
+        else:
+            _check_input(t, name, self.dtype, (None, None, self.Hkv, page_size, self.d), span, host_ok)
+            _check_input(page_table, "page_table", torch.int32, (self.B, None))
 
     def _kv(self, t: torch.Tensor, page_table, page_size) -> KvTensor:
         kv = KvTensor()
@@ -390,6 +428,9 @@ class Engine:
         only the kept rows across the host link."""
         lib = load()
         sub = self._subset(self.refs_all, layers)
+        span = 1 + max((r[0] for r in sub), default=-1)
+        self._check_kv(k, "k", page_table, page_size, span, host_ok=True)
+        self._check_kv(v, "v", page_table, page_size, span, host_ok=True)
         refs = _refs(sub)
         a = ClusterArgs()
         a.struct_size = C.sizeof(ClusterArgs)
@@ -419,6 +460,7 @@ class Engine:
         MPC_SIM_MEAN (mean member key) or MPC_SIM_FXP (Eq. 3 in the
         fixed-point ring with ``frac_bits`` fractional bits and the cache's alpha)."""
         lib = load()
+        _check_input(q, "q", self.dtype, (None, self.B, self.Hq, self.d), 1 + max(self.leaders))
         refs = _refs(self.refs_lead)
         a = SelectArgs()
         a.struct_size = C.sizeof(SelectArgs)
@@ -436,6 +478,14 @@ class Engine:
 
     def attn_args(self, q, k_new, v_new, advance=True, refs_list=None, out=None) -> AttnArgs:
         refs_list = self.refs_all if refs_list is None else refs_list
+        out = self.out if out is None else out
+        span = 1 + max((r[0] for r in refs_list), default=-1)
+        _check_input(q, "q", self.dtype, (None, self.B, self.Hq, self.d), span)
+        _check_input(k_new, "k_new", self.dtype, (None, self.B, self.Hkv, self.d), span)
+        _check_input(v_new, "v_new", self.dtype, (None, self.B, self.Hkv, self.d), span)
+        _check_input(out, "out", torch.float32, (None, self.B, self.Hq, self.d), span)
+        if v_new.stride(0) != k_new.stride(0):
+            raise ValueError("k_new and v_new must have the same layer stride")
         refs = _refs(refs_list)
         a = AttnArgs()
         a.struct_size = C.sizeof(AttnArgs)
@@ -450,7 +500,6 @@ class Engine:
         a.mean = _ptr(self.mean)
         a.cluster_size, a.n_levels, a.fanout, a.alpha = self.s, self.n_levels, _fan(self.fanouts), self.alpha
         a.n_tok, a.advance, a.scale = _ptr(self.n_tok), int(bool(advance)), self.scale
-        out = self.out if out is None else out
         a.out, a.out_layer_stride = _ptr(out), out.stride(0)
         a._refs = refs  # keeps the host array alive as long as the args
         return a

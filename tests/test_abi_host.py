@@ -228,3 +228,37 @@ def test_commonality_validation(lib):
 def test_choose_share_every():
     assert mpcache.choose_share_every({1: 0.95, 2: 0.9, 3: 0.6}, 0.85) == 3   # groups of 3 layers
     assert mpcache.choose_share_every({1: 0.5}, 0.85) == 1                     # no sharing
+
+
+def test_engine_rejects_unsupported_dtype():
+    """The kernels take float32 or bfloat16 only; any other dtype is refused
+    before any buffer is allocated, not passed on under the float32 code."""
+    with pytest.raises(TypeError):
+        mpcache.Engine(n_layers=2, batch=1, n_q_heads=2, n_kv_heads=1, head_dim=64, dtype=torch.float16,
+                       t_max=64, keep_ppm=500_000, cluster_size=16, fanouts=(), level_keep_ppm=(500_000,),
+                       share_every=2, max_decode_steps=4)
+
+
+def test_input_checks_refuse_what_the_calls_would_misread():
+    chk = mpcache._check_input
+    t = torch.zeros((3, 2, 4, 8), dtype=torch.bfloat16)
+    # host memory only where allowed, and then pinned (checked last, so the
+    # layout checks below run on CPU tensors)
+    with pytest.raises(ValueError, match="on the GPU"):
+        chk(t, "q", torch.bfloat16, (None, 2, 4, 8))
+    with pytest.raises(TypeError, match="dtype"):
+        chk(t, "q", torch.float32, (None, 2, 4, 8))
+    with pytest.raises(ValueError, match="shape"):
+        chk(t, "q", torch.bfloat16, (None, 2, 4, 16))
+    with pytest.raises(ValueError, match="shape"):
+        chk(t[0], "q", torch.bfloat16, (None, 2, 4, 8))
+    with pytest.raises(ValueError, match="layers"):
+        chk(t, "q", torch.bfloat16, (None, 2, 4, 8), min_layers=4)
+    # a transposed view has the right sizes but not the layout
+    u = torch.zeros((3, 2, 8, 4), dtype=torch.bfloat16).transpose(2, 3)
+    with pytest.raises(ValueError, match="contiguous"):
+        chk(u, "q", torch.bfloat16, (None, 2, 4, 8))
+    # a layer stride of its own is fine (a slice along dim 0 of a larger buffer)
+    big = torch.zeros((6, 2, 4, 8), dtype=torch.bfloat16)
+    with pytest.raises(ValueError, match="on the GPU"):   # layout accepted, only the memory refused
+        chk(big[::2], "q", torch.bfloat16, (None, 2, 4, 8), min_layers=3)

@@ -11,6 +11,7 @@ Tolerances:
   the oracle's unless the oracle's margin at a cut is inside the band (a tie
   at the kernel's precision), in which case only its validity is checked.
 """
+import ctypes as C
 import math
 
 import numpy as np
@@ -219,6 +220,17 @@ def test_prefill_per_group_from_pinned_host_memory(case):
     for name in ("kept", "n_keep", "n_tok", "kc", "vc", "rmax", "rmin", "rep", "mean"):
         assert torch.equal(getattr(eng, name), getattr(ref, name)), name
     assert torch.equal(eng.scores, ref.scores)
+    assert mpcache.device_status() == 0
+    # static eviction reads keys through TMA tensor maps: host keys are
+    # refused by the binding and, below it, by the C call before any launch
+    with pytest.raises(ValueError, match="on the GPU"):
+        eng.static_evict(hk, xc.q_win, lens, pt, w.page_size)
+    a = eng.static_args(xc.k, xc.q_win, lens, pt, w.page_size)
+    a.k.data = hk.data_ptr()
+    lib = mpcache.load()
+    rc = lib.mpc_static_evict(C.byref(a), None, 0, C.c_void_p(torch.cuda.current_stream().cuda_stream))
+    assert rc == mpcache.MPC_ERR_INVALID_ARG, lib.mpc_last_error()
+    assert b"host memory" in lib.mpc_last_error()
     assert mpcache.device_status() == 0
 
 
