@@ -417,6 +417,8 @@ def run_ours(args, rank, world, dist):
         "static_scoring_path": "tcgen05" if tensor_path else "simt",
         "phases_ms": {"static_evict": static_ms, "build_clusters": build_ms, "decode_all_steps": decode_ms},
         "decode_step_us": decode_ms / E * 1e3,
+        # one launch pair covers every layer, so a layer's share is the mean
+        "decode_step_us_per_layer": decode_ms / E * 1e3 / w.n_layers,
         "decode": {"bytes_per_step": dec_bytes / E, "achieved_gbs": round(decode_gbs, 1),
                    "frac_of_measured_hbm": round(decode_gbs / pk["hbm_gbs"], 4),
                    "frac_of_8tbs": round(decode_gbs / 8000.0, 4)},
