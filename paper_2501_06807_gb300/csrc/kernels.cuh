@@ -104,6 +104,7 @@ struct ScoreTcParams {
   int stats_ld;
   void* aug;     // as StaticParams::aug
   int k_by_ref;  // dense keys indexed by ref (a gathered copy) rather than by layer
+  int items_per_cta;  // 1: one CTA per (unit, 128-block) item; > 1: consecutive items per CTA
 };
 
 struct KvSrc {

@@ -36,6 +36,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "kernels.cuh"
@@ -49,6 +50,7 @@ constexpr int kTcThreads = 64 + kTcEpiThreads;
 constexpr int kStagesTc = 2;
 constexpr int kStatSlots = 4;  // row-statistics ring of pass 1 (tiles in flight ahead of the epilogue)
 constexpr int kBoxBytes = 128 * 128;  // 128 rows x 64 bf16 channels
+constexpr int kTilesPerCta = 32;      // below this many tiles per item, a CTA takes several items
 
 template <int D>
 struct TcSmem {
@@ -59,8 +61,8 @@ struct TcSmem {
   static constexpr int STAGE = TILE;                // one streamed B tile
   static constexpr int AUG_OFF = B_OFF + kStagesTc * STAGE;    // pass 1: kStatSlots x 128 rows x 16 B
   static constexpr int ONE_OFF = AUG_OFF + kStatSlots * 2048;   // pass 1: constant K-side core matrices
-  static constexpr int XCH_OFF = ONE_OFF + 256;                 // halves' partials, 128 x float2
-  static constexpr int BAR_OFF = XCH_OFF + 128 * 8;
+  static constexpr int XCH_OFF = ONE_OFF + 256;                 // halves' partials, 2 x 128 x float2
+  static constexpr int BAR_OFF = XCH_OFF + 2 * 128 * 8;
   static constexpr int USED = BAR_OFF + 256 + 1024;  // + alignment slack
   // at least 80 KB so that at most two CTAs (2 x 256 TMEM columns) share an SM
   static constexpr int TOTAL = USED > 80 * 1024 ? USED : 80 * 1024;
@@ -515,6 +517,354 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
   }
 }
 
+// Several consecutive items per CTA, for items of few tiles (short prompts,
+// one query head per group), where the one-item kernel spends much of a
+// CTA's life on setup and on filling and draining its pipeline.
+template <int PASS, int D>
+__global__ void __launch_bounds__(kTcThreads, 2) score_tc_items_kernel(const __grid_constant__ ScoreTcParams p) {
+  using S = TcSmem<D>;
+  constexpr int KH = S::KH;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::BAR_OFF);
+  uint64_t* empty = full + kStagesTc;
+  uint64_t* a_full = empty + kStagesTc;
+  uint64_t* a_empty = a_full + 1;
+  uint64_t* acc_full = a_empty + 1;
+  uint64_t* acc_empty = acc_full + 2;
+  uint64_t* stats_full = acc_empty + 2;
+  uint64_t* stats_empty = stats_full + kStatSlots;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(stats_empty + kStatSlots);
+  volatile int* abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // ---- work items: (unit, block) pairs.  CTA c takes the contiguous items
+  // [c * per_cta, (c + 1) * per_cta) (consecutive blocks of one unit share
+  // their other operand through L2); every role walks them in the same
+  // order and skips the items with nothing to compute.  The stage ring, the two accumulators and the statistics ring
+  // run on tile counters that continue across items, so TMEM and the
+  // barriers are set up once per CTA.
+  const int HEADS = PASS == 0 ? p.Hq : p.Hkv;
+  const int n_blk = PASS == 0 ? (p.win_rows + 127) / 128 : (p.t_max + 127) / 128;
+  const int64_t n_items = (int64_t)n_blk * p.n_refs * p.B * HEADS;
+  const int64_t x_begin = (int64_t)blockIdx.x * p.items_per_cta;
+  const int64_t x_end = min(n_items, x_begin + p.items_per_cta);
+  struct Item {
+    int head, b, ri, layer, group, T_b, w, qoff, base, i0, j0, i_start, tiles_per_g, n_tiles;
+  };
+  auto item_at = [&](int64_t x) {
+    Item it;
+    const int unit = (int)(x / n_blk), blk = (int)(x % n_blk);
+    it.head = unit % HEADS;
+    it.b = (unit / HEADS) % p.B;
+    it.ri = unit / (HEADS * p.B);
+    it.layer = p.refs.layer[it.ri];
+    it.group = p.refs.group[it.ri];
+    it.T_b = p.lens[it.b];
+    const bool valid_len = it.T_b >= 1 && it.T_b <= p.t_max;
+    it.w = valid_len ? win_rows_of(p, it.T_b) : 0;
+    it.qoff = p.win_rows - it.w;
+    it.base = it.T_b - it.w;  // position of window row 0
+    it.n_tiles = it.i0 = it.j0 = it.i_start = it.tiles_per_g = 0;
+    if (valid_len && it.w <= p.win_rows) {
+      if (PASS == 0) {
+        it.i0 = blk * 128;  // window rows of this item
+        if (it.i0 < it.w) {
+          const int pos_last = it.base + min(it.i0 + 127, it.w - 1);
+          it.n_tiles = pos_last / 128 + 1;  // key tiles 0 .. pos_last
+        }
+      } else {
+        it.j0 = blk * 128;  // keys of this item
+        if (it.j0 < it.T_b) {
+          const int i_first = max(0, it.j0 - it.base);  // first row that sees key j0
+          it.i_start = (i_first / 128) * 128;
+          it.tiles_per_g = (it.w - it.i_start + 127) / 128;
+          it.n_tiles = p.G * it.tiles_per_g;
+        }
+      }
+    }
+    return it;
+  };
+  // the first item is worked out once, before the setup, and reused by
+  // every role; a CTA whose items are all empty (past its sequences'
+  // windows or keys) leaves before the barriers and the TMEM allocation
+  const Item first = item_at(x_begin);
+  {
+    bool any = first.n_tiles > 0;
+    for (int64_t x = x_begin + 1; x < x_end && !any; ++x) any = item_at(x).n_tiles > 0;
+    if (!any) return;
+  }
+  auto item_of = [&](int64_t x) { return x == x_begin ? first : item_at(x); };
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStagesTc; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(a_full, 1);
+    mbar_init(a_empty, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], kTcEpiWarps);
+    }
+    for (int i = 0; i < kStatSlots; ++i) {
+      mbar_init(&stats_full[i], 1);
+      mbar_init(&stats_empty[i], 1);  // released by the MMA that read the slot
+    }
+    *abort = 0;
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 256);
+    tmem_relinquish();
+  }
+  if (PASS == 1 && threadIdx.x >= 64 && threadIdx.x < 80) {
+    // K-side operand of the statistic step: one 8-row core matrix whose rows
+    // are (1, 1, 1, 0, 0, 0, 0, 0) (every 8-row group reuses it), then a zero
+    // core matrix for channels 8..15
+    const int i = threadIdx.x - 64;
+    reinterpret_cast<uint4*>(smem + S::ONE_OFF)[i] =
+        i < 8 ? make_uint4(0x3F803F80u, 0x00003F80u, 0u, 0u) : make_uint4(0u, 0u, 0u, 0u);
+    fence_proxy_async_smem();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0 && lane == 0) {
+    // ---------------------------------------------------- TMA producer
+    int64_t gt = 0;  // B tiles issued (all items)
+    int n_a = 0;     // A tiles issued
+    for (int64_t x = x_begin; x < x_end && !*abort; ++x) {
+      const Item it = item_of(x);
+      if (it.n_tiles == 0) continue;
+      const int qrow0 = (it.b * p.Hq) * p.win_rows + it.qoff;  // + hq * win_rows + i
+      const int krow0 = (it.b * p.Hkv) * p.t_max;              // + hk * t_max + j
+      const int kcoord = p.k_by_ref ? it.ri : it.layer;
+      // A: once the previous item's MMAs have read it
+      if (n_a > 0 && !wait_or_abort(a_empty, (n_a - 1) & 1, abort)) break;
+      mbar_arrive_expect_tx(a_full, S::TILE);
+      for (int kh = 0; kh < KH; ++kh) {
+        if (PASS == 0)
+          tma_load_3d(smem + S::A_OFF + kh * kBoxBytes, &p.map_q, kh * 64, qrow0 + it.head * p.win_rows + it.i0,
+                      it.layer, a_full);
+        else  // keys [j0, j0 + 128) of this kv head: one 128-row box per 64-channel half
+          tma_load_3d(smem + S::A_OFF + kh * kBoxBytes, &p.map_k, kh * 64, krow0 + it.head * p.t_max + it.j0,
+                      kcoord, a_full);
+      }
+      ++n_a;
+      for (int t = 0; t < it.n_tiles; ++t, ++gt) {
+        const int s = (int)(gt % kStagesTc);
+        if (gt >= kStagesTc && !wait_or_abort(&empty[s], (int)((gt / kStagesTc) - 1) & 1, abort)) break;
+        uint8_t* st = smem + S::B_OFF + s * S::STAGE;
+        mbar_arrive_expect_tx(&full[s], S::TILE);
+        if (PASS == 0) {
+          for (int kh = 0; kh < KH; ++kh)
+            tma_load_3d(st + kh * kBoxBytes, &p.map_k, kh * 64, krow0 + (it.head / p.G) * p.t_max + t * 128, kcoord,
+                        &full[s]);
+        } else {
+          const int g = t / it.tiles_per_g, ir = it.i_start + (t % it.tiles_per_g) * 128;
+          const int hq = it.head * p.G + g;
+          for (int kh = 0; kh < KH; ++kh)
+            tma_load_3d(st + kh * kBoxBytes, &p.map_q, kh * 64, qrow0 + hq * p.win_rows + ir, it.layer, &full[s]);
+          // the rows' statistic (16 bytes per row) into its ring slot, once
+          // the MMA that read the slot before has completed
+          const int sb = (int)(gt % kStatSlots);
+          if (gt >= kStatSlots && !wait_or_abort(&stats_empty[sb], (int)((gt / kStatSlots) - 1) & 1, abort)) {
+            ++gt;
+            break;
+          }
+          const uint8_t* src = static_cast<const uint8_t*>(p.aug) +
+                               ((((int64_t)it.ri * p.B + it.b) * p.Hq + hq) * p.stats_ld + ir) * 16;
+          mbar_arrive_expect_tx(&stats_full[sb], 2048);
+          bulk_g2s(smem + S::AUG_OFF + sb * 2048, src, 2048, &stats_full[sb]);
+        }
+      }
+    }
+    // leave no copy in flight: wait (bounded) for the last copies issued
+    for (int64_t t = gt > kStagesTc ? gt - kStagesTc : 0; t < gt; ++t) {
+      int never = 0;
+      wait_or_abort(&full[t % kStagesTc], (int)(t / kStagesTc) & 1, &never);
+    }
+    if (PASS == 1)
+      for (int64_t t = gt > kStatSlots ? gt - kStatSlots : 0; t < gt; ++t) {
+        int never = 0;
+        wait_or_abort(&stats_full[t % kStatSlots], (int)(t / kStatSlots) & 1, &never);
+      }
+    if (n_a > 0) {
+      int never = 0;
+      wait_or_abort(a_full, (n_a - 1) & 1, &never);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ---------------------------------------------------- MMA issuer
+    int64_t gt = 0;  // B tiles consumed (all items)
+    int n_a = 0;
+    bool any = false;
+    for (int64_t x = x_begin; x < x_end && !*abort; ++x) {
+      const Item it = item_of(x);
+      if (it.n_tiles == 0) continue;
+      if (!wait_or_abort(a_full, n_a & 1, abort)) break;
+      ++n_a;
+      const uint32_t a_base = smem_u32(smem + S::A_OFF);
+      bool ok = true;
+      for (int t = 0; t < it.n_tiles; ++t, ++gt) {
+        const int s = (int)(gt % kStagesTc), buf = (int)(gt & 1);
+        if (!wait_or_abort(&full[s], (int)(gt / kStagesTc) & 1, abort) ||
+            (gt >= 2 && !wait_or_abort(&acc_empty[buf], (int)((gt >> 1) - 1) & 1, abort)) ||
+            (PASS == 1 && !wait_or_abort(&stats_full[gt % kStatSlots], (int)(gt / kStatSlots) & 1, abort))) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t b_base = smem_u32(smem + S::B_OFF + s * S::STAGE);
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * kBoxBytes + (kk & 3) * 32;
+          umma_bf16(tmem + buf * 128, sw128_desc(a_base + off), sw128_desc(b_base + off), kIdesc, kk > 0);
+        }
+        if (PASS == 1) {
+          // one more K step adds the rows' statistic: S^T + (x1 + x2 + x3)
+          const int sb = (int)(gt % kStatSlots);
+          umma_bf16(tmem + buf * 128, plain_desc(smem_u32(smem + S::ONE_OFF), 128, 0),
+                    plain_desc(smem_u32(smem + S::AUG_OFF + sb * 2048), 0, 128), kIdesc, 1);
+          umma_commit(&stats_empty[sb]);
+        }
+        umma_commit(&empty[s]);
+        umma_commit(&acc_full[buf]);
+        any = true;
+      }
+      umma_commit(a_empty);  // A is free once this item's MMAs are done
+      if (!ok) break;
+    }
+    // leave no MMA in flight before TMEM is released (bounded)
+    if (any) {
+      int never = 0;
+      wait_or_abort(&acc_full[(gt - 1) & 1], (int)((gt - 1) >> 1) & 1, &never);
+    }
+  } else if (warp >= 2) {
+    // ---------------------------------------------------- epilogue
+    const int quarter = warp & 3;               // TMEM lanes 32*quarter ..
+    const int half = (warp - 2) >> 2;           // columns 64*half .. +63
+    const int col0 = half * 64;
+    const int r = quarter * 32 + lane;          // this thread's TMEM lane
+    const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16) + col0;
+    const uint64_t sc2 = pk2(p.scale_log2, p.scale_log2);
+    int64_t gt = 0;
+    int n_done = 0;
+    for (int64_t x = x_begin; x < x_end; ++x) {
+      const Item it = item_of(x);
+      if (it.n_tiles == 0) continue;
+      float m = kNegInf, l = 0.f, acc = 0.f;
+      const int i_row = it.i0 + r;                // pass 0: window row
+      const int pos_row = it.base + i_row;
+      const int j_key = it.j0 + r;                // pass 1: key
+      int t = 0;
+      for (; t < it.n_tiles; ++t, ++gt) {
+        const int buf = (int)(gt & 1);
+        const bool ok = wait_or_abort(&acc_full[buf], (int)(gt >> 1) & 1, abort);
+        if (!epilogue_all(ok)) break;
+        tc_fence_after();
+        if (PASS == 0) {
+          const int kj = t * 128 + col0;                     // first key of this thread's columns
+          const bool need_mask = kj + 63 > it.base + it.i0;  // crosses some row's diagonal
+#pragma unroll 1
+          for (int c = 0; c < 2; ++c) {
+            float v[32];
+            tmem_ld32(lane_addr + buf * 128 + c * 32, v);
+            if (need_mask) {
+#pragma unroll
+              for (int k = 0; k < 32; ++k)
+                if (kj + c * 32 + k > pos_row) v[k] = kNegInf;
+            }
+            const float mnew = fmaxf(m, max32(v) * p.scale_log2);
+            if (mnew != kNegInf) {
+              const uint64_t nm2 = pk2(-mnew, -mnew);
+              uint64_t s2 = pk2(0.f, 0.f);
+#pragma unroll
+              for (int k = 0; k < 32; k += 2) {
+                const uint64_t x2 = ffma2(pk2(v[k], v[k + 1]), sc2, nm2);
+                s2 = fadd2(s2, exp2_mufu2(x2));
+              }
+              float s0, s1;
+              upk2(s2, s0, s1);
+              const float sum = s0 + s1;
+              l = (m == kNegInf) ? sum : l * fast_exp2(m - mnew) + sum;
+              m = mnew;
+            }
+          }
+        } else {
+          const int ir = it.i_start + (t % it.tiles_per_g) * 128 + col0;  // first row of this thread's columns
+          // the accumulator already holds s + statistic / scale_log2 (about
+          // -3e38 past the window); row i sees key j when j <= base + i
+          const bool need_mask = it.j0 + 127 > it.base + ir;
+          const uint64_t zero2 = pk2(0.f, 0.f);
+          uint64_t s2 = pk2(0.f, 0.f);
+#pragma unroll 1
+          for (int c = 0; c < 2; ++c) {
+            float v[32];
+            tmem_ld32(lane_addr + buf * 128 + c * 32, v);
+            if (need_mask) {
+#pragma unroll
+              for (int k = 0; k < 32; ++k)
+                if (j_key > it.base + ir + c * 32 + k) v[k] = kNegInf;
+            }
+#pragma unroll
+            for (int k = 0; k < 32; k += 2) s2 = fadd2(s2, exp2_mufu2(ffma2(pk2(v[k], v[k + 1]), sc2, zero2)));
+          }
+          float s0, s1;
+          upk2(s2, s0, s1);
+          acc += s0 + s1;
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acc_empty[buf]);
+      }
+      if (t < it.n_tiles) break;  // aborted (every epilogue warp takes this branch)
+      // combine the two column halves of every lane (fixed order: half 0 +
+      // half 1), through a buffer that alternates between items
+      float2* xch = reinterpret_cast<float2*>(smem + S::XCH_OFF) + (n_done & 1) * 128;
+      if (half == 1) xch[r] = PASS == 0 ? make_float2(m, l) : make_float2(acc, 0.f);
+      epilogue_sync();
+      if (half == 0 && !*abort) {
+        const float2 o = xch[r];
+        if (PASS == 0) {
+          const float M = fmaxf(m, o.x);
+          const float L =
+              (m == kNegInf ? 0.f : l * fast_exp2(m - M)) + (o.x == kNegInf ? 0.f : o.y * fast_exp2(o.x - M));
+          // the statistic over the log2 scale, split into three bf16 parts
+          // (x1 + x2 + x3 = x to fp32 precision), so pass 1's extra MMA step
+          // adds it to every score of the row.  Rows past the window get a
+          // large finite negative value (ex2 of it is 0): -inf would meet
+          // the zero channels of the step's other operand and give
+          // 0 x inf = NaN
+          uint4* ar = reinterpret_cast<uint4*>(p.aug) +
+                      (((int64_t)it.ri * p.B + it.b) * p.Hq + it.head) * p.stats_ld + i_row;
+          if (i_row < it.w) {
+            const float xv = -(M + log2f(L)) / p.scale_log2;
+            const bf16 x1 = __float2bfloat16_rn(xv);
+            const float r1 = xv - __bfloat162float(x1);
+            const bf16 x2 = __float2bfloat16_rn(r1);
+            const bf16 x3 = __float2bfloat16_rn(r1 - __bfloat162float(x2));
+            *ar = make_uint4(pack_bf16_pair(x1, x2), pack_bf16_pair(x3, __float2bfloat16_rn(0.f)), 0u, 0u);
+          } else if (i_row < (it.w + 127) / 128 * 128) {
+            *ar = make_uint4(pack_bf16_pair(__float2bfloat16_rn(-3.0e38f), __float2bfloat16_rn(0.f)), 0u, 0u, 0u);
+          }
+        } else if (j_key < it.T_b) {
+          p.scores[((int64_t)(it.group * p.B + it.b) * p.Hkv + it.head) * p.t_max + j_key] = acc + o.x;
+        }
+      }
+      ++n_done;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 256);
+  }
+}
+
 // ------------------------------------------------------------- host side ----
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -548,11 +898,23 @@ bool make_map(CUtensorMap* map, const void* base, int d, int64_t rows, int layer
 template <int PASS, int D>
 cudaError_t launch_pass(const ScoreTcParams& p, dim3 grid, cudaStream_t st) {
   const int smem = TcSmem<D>::TOTAL;
+  if (p.items_per_cta > 1) {
+    cudaError_t e = ensure_dyn_smem((const void*)score_tc_items_kernel<PASS, D>, smem);
+    if (e != cudaSuccess) return e;
+    score_tc_items_kernel<PASS, D><<<grid, kTcThreads, smem, st>>>(p);
+    return cudaGetLastError();
+  }
   cudaError_t e = ensure_dyn_smem((const void*)score_tc_kernel<PASS, D>, smem);
   if (e != cudaSuccess) return e;
   score_tc_kernel<PASS, D><<<grid, kTcThreads, smem, st>>>(p);
   return cudaGetLastError();
 }
+
+// Items per CTA of a pass: one while an item has kTilesPerCta tiles or more
+// (the one-item kernel, one CTA per item on a 2-D grid), else enough items
+// for about that many tiles (the items kernel, 1-D grid).  `tiles` is the
+// most tiles one item of the pass can have.
+int items_per_cta(int tiles) { return std::max(1, kTilesPerCta / std::max(1, tiles)); }
 
 }  // namespace
 
@@ -561,15 +923,23 @@ cudaError_t launch_score_tc(ScoreTcParams& p, int D, int n_layer_span, cudaStrea
     return cudaErrorInvalidValue;
   if (!make_map(&p.map_k, p.k, D, (int64_t)p.B * p.Hkv * p.t_max, p.k_by_ref ? p.n_refs : n_layer_span, p.k_ls))
     return cudaErrorInvalidValue;
-  const dim3 g0((p.win_rows + 127) / 128, p.n_refs * p.B * p.Hq);
-  const dim3 g1((p.t_max + 127) / 128, p.n_refs * p.B * p.Hkv);
+  const int row_blks = (p.win_rows + 127) / 128, key_blks = (p.t_max + 127) / 128;
+  ScoreTcParams p0 = p, p1 = p;
+  p0.items_per_cta = items_per_cta(key_blks);        // pass 0 item: key tiles up to t_max
+  p1.items_per_cta = items_per_cta(p.G * row_blks);  // pass 1 item: row tiles of the group's heads
+  auto grid_of = [](const ScoreTcParams& q, int blks, int heads) {
+    const long long units = (long long)q.n_refs * q.B * heads;
+    if (q.items_per_cta == 1) return dim3(blks, (unsigned)units);
+    return dim3((unsigned)((units * blks + q.items_per_cta - 1) / q.items_per_cta));
+  };
+  const dim3 g0 = grid_of(p0, row_blks, p.Hq), g1 = grid_of(p1, key_blks, p.Hkv);
   cudaError_t e;
   if (D == 64) {
-    if ((e = launch_pass<0, 64>(p, g0, st)) != cudaSuccess) return e;
-    return launch_pass<1, 64>(p, g1, st);
+    if ((e = launch_pass<0, 64>(p0, g0, st)) != cudaSuccess) return e;
+    return launch_pass<1, 64>(p1, g1, st);
   }
-  if ((e = launch_pass<0, 128>(p, g0, st)) != cudaSuccess) return e;
-  return launch_pass<1, 128>(p, g1, st);
+  if ((e = launch_pass<0, 128>(p0, g0, st)) != cudaSuccess) return e;
+  return launch_pass<1, 128>(p1, g1, st);
 }
 
 int take_status_score_tc() { return take_status(); }
