@@ -16,7 +16,7 @@
  *                           (Sec. 3.3-3.4, Alg. 2 Step 2)
  *   mpc_sparse_decode_attn  per decode step: append the new k, v, then
  *                           softmax(q K'^T / sqrt(d)) V' over the selected
- *                           clusters and the tail (Alg. 1 line 4)
+ *                           clusters and the tail (Alg. 1)
  *
  * Conventions shared by every call
  * --------------------------------
@@ -234,7 +234,7 @@ typedef struct {
 } mpc_select_args;
 
 /* ---- mpc_sparse_decode_attn ----------------------------------------------
- * One decode step of attention for every ref (Alg. 1 line 4; Alg. 2 Step 2,
+ * One decode step of attention for every ref (Alg. 1; Alg. 2 Step 2,
  * gather + sparse attention; App. A decode append).  With n = n_tok_b and
  * C_1 = floor(n / s):
  *   1. k_new, v_new are written to row n of the layer's cache (append);

@@ -13,7 +13,7 @@ Step 1 (prefill, once):
     per key column; the highest-scoring tokens are kept, the rest dropped;
   * leader layers score, the other layers of a sharing group reuse the
     leader's kept set (cross-layer index sharing, Sec. 3.4);
-  * the kept keys/values are gathered (token gathering, Alg. 1 line 3).
+  * the kept keys/values are gathered (token gathering, Alg. 1).
 Step 2 (every decode step e, every layer l):
   * append k, v to the cache (decoding stage, App. A);
   * leader layers: cluster similarity Sim(q, K_c) = q . (alpha r_max +
@@ -22,7 +22,7 @@ Step 2 (every decode step e, every layer l):
     top-k from the coarsest to the finest level among the children of the kept
     parents (Sec. 3.3 "Hierarchical KV cache clustering"); other layers reuse
     the leader's ids (Sec. 3.4);
-  * softmax(q K'^T / sqrt(d)) V' over the gathered tokens (Alg. 1 line 4).
+  * softmax(q K'^T / sqrt(d)) V' over the gathered tokens (Alg. 1).
 
 Readings of points the paper leaves open (each follows the numbered reading in
 the design notes):
@@ -295,7 +295,7 @@ def hierarchical_select(q_group: np.ndarray, levels: List[Level],
 
 def sparse_attention(q: np.ndarray, k_sel: np.ndarray, v_sel: np.ndarray,
                      scale: float) -> np.ndarray:
-    """softmax(q K'^T * scale) V' over the gathered tokens (Alg. 1 line 4)."""
+    """softmax(q K'^T * scale) V' over the gathered tokens (Alg. 1)."""
     q = np.asarray(q, dtype=np.float64)
     logits = (np.asarray(k_sel, dtype=np.float64) @ q) * scale
     logits -= logits.max()

@@ -1,5 +1,5 @@
 // Sparse decode attention over the selected clusters and the tail, with the
-// decode-step append and the tail seal (Alg. 1 line 4; Alg. 2 Step 2; App. A).
+// decode-step append and the tail seal (Alg. 1; Alg. 2 Step 2; App. A).
 //
 // Work decomposition: one unit = (ref, sequence b, kv head h).  The rows a
 // unit attends are listed in order: the s rows of every selected cluster,
