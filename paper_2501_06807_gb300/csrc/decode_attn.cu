@@ -299,8 +299,8 @@ __device__ __forceinline__ void finish_grid(const AttnParams& p) {
 // cluster row tile, tail and appended row of every (layer, sequence, kv
 // head)) form one list, cut into contiguous, equal ranges, one per warp slot
 // (slots interleaved over the CTAs, at most one slot per tile).  Every warp
-// streams its range through its own ring of shared-memory stages (1-D bulk
-// copies of K and V tile rows), so every SM moves the same amount of KV.
+// streams its range through its own ring of shared-memory stages (K and V
+// tile rows), so every SM moves the same amount of KV.
 //
 // Tiles are staged with cp.async (16 bytes per lane, committed as one group
 // per tile, so a warp keeps NST tiles in flight at the cost of a few
