@@ -21,6 +21,10 @@
 //     epilogue needs one multiply, one ex2 and one add per score and no
 //     shared-memory loads (every lane would need every row's value, and
 //     broadcast loads were this pass's bound).
+//   An item is one such 128-row block.  When an item has fewer than 32
+//   tiles (short prompts, one query head per group), score_tc_items_kernel
+//   gives each CTA several consecutive items instead of one, so that setup
+//   and the filling and draining of its pipeline are paid once per CTA.
 
 // Roles: warp 0 issues TMA tile loads (128B-swizzled, K-major boxes of
 // 128 rows x 64 channels), warp 1 allocates TMEM and issues tcgen05.mma
