@@ -24,8 +24,8 @@ Step 2 (every decode step e, every layer l):
     the leader's ids (Sec. 3.4);
   * softmax(q K'^T / sqrt(d)) V' over the gathered tokens (Alg. 1).
 
-Readings of points the paper leaves open (each follows the numbered reading in
-the design notes):
+Readings of points the paper leaves open (the same readings as the CUDA
+path's, each implemented here on its own):
   * the static map uses the model's own 1/sqrt(d) scale and a causal mask;
   * window w = ceil(rho_w T), rho_w = 0.2, or 0.1 when T > 24576;
   * one kept set per (sequence, kv head); GQA sums the group's query heads;
