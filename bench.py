@@ -382,10 +382,12 @@ def run_ours(args, rank, world, dist):
     dominant_static = static_ms >= decode_ms
     # bf16 keys score on tcgen05 (paged keys through their gathered dense copy)
     tensor_path = w.dtype == "bf16"
-    # DRAM bytes of one static-eviction call (both score passes), from ncu on
-    # the 8k workload (profiles/score_tc_kernel_c3_llama3_8b_t8192.md): each
-    # pass reads its inputs once, so the 32k figure is that capture scaled by
-    # the input bytes (939.5 / 302.1 MB).  Valid for the kernel as captured.
+    # DRAM bytes of one static-eviction call (both score passes), from an ncu
+    # capture of the 8k workload (dram__bytes_read.sum + dram__bytes_write.sum
+    # of the two score_tc_kernel launches: 302.1 + 10.0 + 310.6 + 5.5 MB):
+    # each pass reads its inputs once, so the 32k figure is that capture
+    # scaled by the input bytes (939.5 / 302.1 MB).  Valid for the kernel as
+    # captured.
     static_traffic = {"c3_llama3_8b_gqa_t8192": 628.1e6,
                       "c5_llama3_8b_gqa_t32768_needles": 628.1e6 * 939.5 / 302.1}.get(w.name)
     if dominant_static and tensor_path:
