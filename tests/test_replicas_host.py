@@ -36,7 +36,7 @@ def _worker(rank, world, port, out):
 
 def test_two_replicas_aggregate_over_gloo():
     world = 2
-    out = mp.Manager().dict()
+    out = mp.get_context("spawn").Manager().dict()  # no fork of a threaded process
     mp.spawn(_worker, args=(world, _free_port(), out), nprocs=world, join=True)
     for r in range(world):
         t, v, seeds = out[r]
