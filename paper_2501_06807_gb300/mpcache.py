@@ -367,6 +367,12 @@ class Engine:
     def static_args(self, k: torch.Tensor, q_win: torch.Tensor, lens: torch.Tensor,
                     page_table: Optional[torch.Tensor] = None, page_size: int = 16,
                     layers: Optional[Sequence[int]] = None) -> StaticArgs:
+        # the kernels skip a sequence whose window has more rows than q_win
+        # holds; the engine's bound (the window of a t_max-token prompt)
+        # covers every sequence
+        if q_win.dim() == 5 and q_win.shape[3] < self.win_rows:
+            raise ValueError(f"q_win: {q_win.shape[3]} window rows, the engine's prompts need up to "
+                             f"{self.win_rows}")
         lead = self._subset(self.refs_lead, layers)
         span = 1 + max((r[0] for r in lead), default=-1)
         self._check_kv(k, "k", page_table, page_size, span, host_ok=False)

@@ -262,3 +262,12 @@ def test_input_checks_refuse_what_the_calls_would_misread():
     big = torch.zeros((6, 2, 4, 8), dtype=torch.bfloat16)
     with pytest.raises(ValueError, match="on the GPU"):   # layout accepted, only the memory refused
         chk(big[::2], "q", torch.bfloat16, (None, 2, 4, 8), min_layers=3)
+
+
+def test_static_args_need_the_engines_window_rows():
+    """Window queries with fewer rows than the longest window the engine's
+    prompts can have are refused (the kernels would skip such a sequence)."""
+    eng = mpcache.Engine.__new__(mpcache.Engine)   # no device buffers needed
+    eng.win_rows = 52
+    with pytest.raises(ValueError, match="window rows"):
+        eng.static_args(torch.zeros(1), torch.zeros((1, 1, 2, 51, 64), dtype=torch.bfloat16), torch.zeros(1))
