@@ -367,9 +367,8 @@ class Engine:
     def static_args(self, k: torch.Tensor, q_win: torch.Tensor, lens: torch.Tensor,
                     page_table: Optional[torch.Tensor] = None, page_size: int = 16,
                     layers: Optional[Sequence[int]] = None) -> StaticArgs:
-        # the kernels skip a sequence whose window has more rows than q_win
-        # holds; the engine's bound (the window of a t_max-token prompt)
-        # covers every sequence
+        # the C call refuses fewer window rows than the longest window of a
+        # t_max-token prompt too; this names the tensor in the message
         if q_win.dim() == 5 and q_win.shape[3] < self.win_rows:
             raise ValueError(f"q_win: {q_win.shape[3]} window rows, the engine's prompts need up to "
                              f"{self.win_rows}")

@@ -266,7 +266,7 @@ def test_input_checks_refuse_what_the_calls_would_misread():
 
 def test_static_args_need_the_engines_window_rows():
     """Window queries with fewer rows than the longest window the engine's
-    prompts can have are refused (the kernels would skip such a sequence)."""
+    prompts can have are refused before the C call (which refuses them too)."""
     eng = mpcache.Engine.__new__(mpcache.Engine)   # no device buffers needed
     eng.win_rows = 52
     with pytest.raises(ValueError, match="window rows"):
