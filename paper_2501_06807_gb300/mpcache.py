@@ -34,15 +34,18 @@ PPM = 1_000_000
 
 
 class LayerRef(C.Structure):
+    """mpc_layer_ref: a processed layer's index, its sharing group and whether it leads."""
     _fields_ = [("layer", C.c_int32), ("group", C.c_int32), ("leader", C.c_int32)]
 
 
 class KvTensor(C.Structure):
+    """mpc_kv_tensor: prompt keys or values, dense or as a page pool with its page table."""
     _fields_ = [("data", C.c_void_p), ("layer_stride", C.c_int64), ("page_table", C.c_void_p),
                 ("page_size", C.c_int32), ("max_pages", C.c_int32)]
 
 
 class StaticArgs(C.Structure):
+    """mpc_static_args: the arguments of mpc_static_evict, field for field."""
     _fields_ = [("struct_size", C.c_uint32), ("n_refs", C.c_int32), ("refs", C.POINTER(LayerRef)),
                 ("batch", C.c_int32), ("n_q_heads", C.c_int32), ("n_kv_heads", C.c_int32),
                 ("head_dim", C.c_int32), ("dtype", C.c_int32), ("t_max", C.c_int32),
@@ -54,6 +57,7 @@ class StaticArgs(C.Structure):
 
 
 class ClusterArgs(C.Structure):
+    """mpc_cluster_args: the arguments of mpc_build_clusters, field for field."""
     _fields_ = [("struct_size", C.c_uint32), ("n_refs", C.c_int32), ("refs", C.POINTER(LayerRef)),
                 ("batch", C.c_int32), ("n_kv_heads", C.c_int32), ("head_dim", C.c_int32),
                 ("dtype", C.c_int32), ("t_max", C.c_int32), ("k", KvTensor), ("v", KvTensor),
@@ -66,6 +70,7 @@ class ClusterArgs(C.Structure):
 
 
 class SelectArgs(C.Structure):
+    """mpc_select_args: the arguments of mpc_select, field for field."""
     _fields_ = [("struct_size", C.c_uint32), ("n_refs", C.c_int32), ("refs", C.POINTER(LayerRef)),
                 ("batch", C.c_int32), ("n_q_heads", C.c_int32), ("n_kv_heads", C.c_int32),
                 ("head_dim", C.c_int32), ("dtype", C.c_int32), ("q", C.c_void_p),
@@ -79,6 +84,7 @@ class SelectArgs(C.Structure):
 
 
 class CommonalityArgs(C.Structure):
+    """mpc_commonality_args: the arguments of mpc_commonality, field for field."""
     _fields_ = [("struct_size", C.c_uint32), ("n_layers", C.c_int32), ("batch", C.c_int32),
                 ("n_kv_heads", C.c_int32), ("sel", C.c_void_p), ("sel_layer_stride", C.c_int64),
                 ("sel_cap", C.c_int32), ("n_clusters", C.c_int32), ("k", C.c_int32), ("m", C.c_int32),
@@ -86,6 +92,7 @@ class CommonalityArgs(C.Structure):
 
 
 class AttnArgs(C.Structure):
+    """mpc_attn_args: the arguments of mpc_sparse_decode_attn, field for field."""
     _fields_ = [("struct_size", C.c_uint32), ("n_refs", C.c_int32), ("refs", C.POINTER(LayerRef)),
                 ("batch", C.c_int32), ("n_q_heads", C.c_int32), ("n_kv_heads", C.c_int32),
                 ("head_dim", C.c_int32), ("dtype", C.c_int32), ("q", C.c_void_p),
@@ -110,6 +117,7 @@ _LIB = None
 
 
 def library_path() -> str:
+    """Path of the in-tree libmpcache.so."""
     return _build.LIB
 
 
@@ -150,6 +158,8 @@ def load(path: Optional[str] = None) -> C.CDLL:
 
 
 class MPCError(RuntimeError):
+    """A call returned a negative MPC_ERR_* code; ``code`` holds it, the message is the library's."""
+
     def __init__(self, code: int, msg: str):
         super().__init__(f"mpcache error {code}: {msg}")
         self.code = code
@@ -278,6 +288,7 @@ def choose_share_every(scores: dict, threshold: float) -> int:
 
 
 def summary_rows(cap_tokens: int, s: int, fanouts: Sequence[int]) -> int:
+    """Rows of one summary pyramid (all levels) for ``cap_tokens`` cache rows."""
     arr = (C.c_int32 * MAX_LEVELS)(*([int(f) for f in fanouts] + [0] * (MAX_LEVELS - len(fanouts))))
     r = load().mpc_summary_rows(cap_tokens, s, 1 + len(fanouts), arr)
     if r < 0:
@@ -286,6 +297,9 @@ def summary_rows(cap_tokens: int, s: int, fanouts: Sequence[int]) -> int:
 
 
 def device_status() -> int:
+    """Synchronizes the device, then reads and clears the device status word
+    (1: a bounded wait gave up, 2: a decode step had no row left, 4: an index
+    out of range was skipped)."""
     v = C.c_int(0)
     _check(load().mpc_device_status(C.byref(v)))
     return v.value
@@ -367,6 +381,8 @@ class Engine:
     def static_args(self, k: torch.Tensor, q_win: torch.Tensor, lens: torch.Tensor,
                     page_table: Optional[torch.Tensor] = None, page_size: int = 16,
                     layers: Optional[Sequence[int]] = None) -> StaticArgs:
+        """The checked mpc_static_args of the leader layers (of ``layers``
+        only, if given); the returned struct keeps its refs array alive."""
         # the C call refuses fewer window rows than the longest window of a
         # t_max-token prompt too; this names the tensor in the message
         if q_win.dim() == 5 and q_win.shape[3] < self.win_rows:
@@ -482,6 +498,8 @@ class Engine:
         _check(lib.mpc_select(C.byref(a), None, 0, C.c_void_p(_stream())))
 
     def attn_args(self, q, k_new, v_new, advance=True, refs_list=None, out=None) -> AttnArgs:
+        """The checked mpc_attn_args of one decode step for ``refs_list``
+        (default: every processed layer); the struct keeps its refs array alive."""
         refs_list = self.refs_all if refs_list is None else refs_list
         out = self.out if out is None else out
         span = 1 + max((r[0] for r in refs_list), default=-1)
