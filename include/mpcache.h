@@ -70,7 +70,7 @@ extern "C" {
 
 #define MPC_API __attribute__((visibility("default")))
 
-#define MPC_ABI_VERSION 5
+#define MPC_ABI_VERSION 6
 #define MPC_MAX_LEVELS 4
 #define MPC_MAX_REFS 128
 
@@ -295,6 +295,52 @@ MPC_API int mpc_select(const mpc_select_args* args, void* workspace,
                        size_t workspace_bytes, void* stream);
 MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace,
                                    size_t workspace_bytes, void* stream);
+
+/* ---- mpc_decode_step -----------------------------------------------------
+ * One whole decode step (Alg. 2 Step 2) in one call: for every leader ref the
+ * hierarchical selection of mpc_select, then for every ref the append and
+ * sparse attention of mpc_sparse_decode_attn over the selection of its group
+ * (Sec. 3.4: the leader computes the indices, the other layers of the group
+ * reuse them).  The selections and outputs are those of mpc_select followed
+ * by mpc_sparse_decode_attn with the same arguments: the same similarity
+ * arithmetic and ranking, so the same ids; the attention sums the same rows
+ * in another order, so o agrees to fp32 rounding.
+ * - attn: the arguments of mpc_sparse_decode_attn (attn.struct_size =
+ *   sizeof(mpc_attn_args)); attn.sel / attn.n_sel are OUTPUTS here, written
+ *   like mpc_select's out_sel / out_n_sel for every group of the call.  Every
+ *   ref's group must have its leader among the refs (one leader per group),
+ *   and the summary pyramid the metric reads must be given (rep for
+ *   MPC_SIM_EQ3, mean for MPC_SIM_MEAN, r_max / r_min for MPC_SIM_BOUND and
+ *   MPC_SIM_FXP; r_max, r_min and rep are also updated by the seal).
+ * - level_keep_ppm, metric, frac_bits: as in mpc_select_args (alpha is
+ *   attn.alpha).
+ * - chunk_tiles: 16-row tiles per unit of attention work a warp claims at a
+ *   time (1 .. 64; 0 picks one from the sizes).
+ * - speculate: -1 automatic, 0 or 1: whether the selection's first round
+ *   also scores every cluster of the level below the coarsest (one
+ *   dependent round fewer, more rows read).
+ * With bf16 caches and the EQ3 / BOUND / MEAN metrics the step is one
+ * persistent kernel: selection teams publish each unit's ids (release store
+ * of a ready flag in the workspace) and the attention warps wait for them
+ * (bounded, 1 s; a wait that gives up sets flag 1 of mpc_device_status and
+ * the call's outputs are undefined).  Otherwise (fp32 caches, MPC_SIM_FXP,
+ * more than 1024 candidates at a level) it is mpc_select's kernel followed
+ * by mpc_sparse_decode_attn's.
+ * Workspace: mpc_decode_step_workspace_size bytes, zero-filled once; the
+ * call leaves its counters zero (also after a wait that gave up). */
+typedef struct {
+  uint32_t struct_size;        /* sizeof(mpc_decode_args) */
+  mpc_attn_args attn;
+  int32_t level_keep_ppm[MPC_MAX_LEVELS]; /* finest level first */
+  int32_t metric;              /* MPC_SIM_EQ3, _BOUND, _MEAN or _FXP */
+  int32_t frac_bits;           /* MPC_SIM_FXP only */
+  int32_t chunk_tiles;         /* 0 = automatic */
+  int32_t speculate;           /* -1 = automatic */
+} mpc_decode_args;
+
+MPC_API int mpc_decode_step_workspace_size(const mpc_decode_args* args, size_t* bytes);
+MPC_API int mpc_decode_step(const mpc_decode_args* args, void* workspace, size_t workspace_bytes,
+                            void* stream);
 
 /* ---- mpc_sparse_decode_attn_static_scratch --------------------------------
  * The same decode step as mpc_sparse_decode_attn, for callers that cannot

@@ -17,7 +17,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(OUT_DIR, "libmpcache.so")
-SOURCES = ["abi.cu", "decode_attn.cu", "select.cu", "clusters.cu", "static_evict.cu", "score_tc.cu",
+SOURCES = ["abi.cu", "decode_attn.cu", "decode_step.cu", "select.cu", "clusters.cu", "static_evict.cu", "score_tc.cu",
            "no_alloc.cu", "commonality.cu", "selftest.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "--expt-relaxed-constexpr", "-Xcompiler", "-fPIC",

@@ -404,6 +404,149 @@ int validate_attn(const mpc_attn_args* a, AttnParams* p, AttnPlan* plan) {
   return MPC_OK;
 }
 
+// --------------------------------------------------------- decode step ----
+struct StepPlan {
+  AttnPlan attn;   // the two-launch path (mpc_select's and mpc_sparse_decode_attn's kernels)
+  bool fused;      // one decode_step_kernel launch
+  int sel_units;
+  size_t part_off, ucnt_off, ready_off, cnt_off, ctl_off, bytes;
+};
+
+int validate_step(const mpc_decode_args* a, StepParams* sp, SelectParams* sel, StepPlan* plan) {
+  if (a == nullptr) return fail(MPC_ERR_INVALID_ARG, "args is NULL");
+  if (a->struct_size != sizeof(mpc_decode_args))
+    return fail(MPC_ERR_INVALID_ARG, "struct_size %u != %zu", a->struct_size, sizeof(mpc_decode_args));
+  memset(sp, 0, sizeof(*sp));
+  memset(plan, 0, sizeof(*plan));
+  const mpc_attn_args& t = a->attn;
+  MPC_TRY(validate_attn(&t, &sp->a, &plan->attn));
+  // one leader per group, and every ref's group led in this call
+  mpc_layer_ref lead[kMaxRefs];
+  int nl = 0;
+  for (int i = 0; i < t.n_refs; ++i) {
+    if (!t.refs[i].leader) continue;
+    for (int k = 0; k < nl; ++k)
+      if (lead[k].group == t.refs[i].group)
+        return fail(MPC_ERR_INVALID_ARG, "refs[%d] is a second leader of group %d", i, t.refs[i].group);
+    sp->lead_ref[nl] = (int16_t)i;
+    lead[nl++] = t.refs[i];
+  }
+  for (int i = 0; i < t.n_refs; ++i) {
+    int k = 0;
+    while (k < nl && lead[k].group != t.refs[i].group) ++k;
+    if (k == nl)
+      return fail(MPC_ERR_INVALID_ARG,
+                  "the leader of refs[%d]'s group %d is not among the refs (use mpc_sparse_decode_attn)", i,
+                  t.refs[i].group);
+    sp->lead_of[i] = (int16_t)k;
+  }
+  mpc_select_args sa;
+  memset(&sa, 0, sizeof(sa));
+  sa.struct_size = sizeof(sa);
+  sa.n_refs = nl;
+  sa.refs = lead;
+  sa.batch = t.batch;
+  sa.n_q_heads = t.n_q_heads;
+  sa.n_kv_heads = t.n_kv_heads;
+  sa.head_dim = t.head_dim;
+  sa.dtype = t.dtype;
+  sa.q = t.q;
+  sa.q_layer_stride = t.q_layer_stride;
+  sa.rep = t.rep;
+  sa.summary_rows = t.summary_rows;
+  sa.cap_tokens = t.cap_tokens;
+  sa.n_tok = t.n_tok;
+  sa.cluster_size = t.cluster_size;
+  sa.n_levels = t.n_levels;
+  for (int l = 0; l < kMaxLevels; ++l) {
+    sa.fanout[l] = t.fanout[l];
+    sa.level_keep_ppm[l] = a->level_keep_ppm[l];
+  }
+  sa.sel_cap = t.sel_cap;
+  sa.out_sel = const_cast<int32_t*>(t.sel);
+  sa.out_n_sel = const_cast<int32_t*>(t.n_sel);
+  sa.metric = a->metric;
+  sa.r_max = t.r_max;
+  sa.r_min = t.r_min;
+  sa.mean = t.mean;
+  sa.alpha = t.alpha;
+  sa.frac_bits = a->frac_bits;
+  MPC_TRY(validate_select(&sa, sel));
+  if (a->chunk_tiles < 0 || a->chunk_tiles > 64) return fail(MPC_ERR_BAD_SHAPE, "chunk_tiles %d not in [0, 64]", a->chunk_tiles);
+  if (a->speculate < -1 || a->speculate > 1) return fail(MPC_ERR_BAD_SHAPE, "speculate %d not in {-1, 0, 1}", a->speculate);
+
+  const int D = t.head_dim, G = sp->a.G, B = t.batch, s = t.cluster_size;
+  const int units = plan->attn.units;
+  plan->sel_units = nl * B * t.n_kv_heads;
+  const int n_src = select_n_src(a->metric);
+  int wpc = 0, nst = 0;
+  step_shape(D, G, B, &wpc, &nst);
+  plan->fused = t.dtype == MPC_BF16 && a->metric != MPC_SIM_FXP && sel->max_cand <= 1024 &&
+                step_smem_bytes(D, G, B) <= kSmemOptin;
+  int tw = 1, rb = 0;
+  if (plan->fused) {
+    // the largest team (divisor of the CTA's warps) that still gives every
+    // selection unit its own team, grown while its scratch stages few rows
+    const int ctas = kStepCtasMax;
+    for (int d = 1; d <= wpc; ++d)
+      if (wpc % d == 0 && (long long)ctas * (wpc / d) >= plan->sel_units) tw = d;
+    rb = step_row_buf(D, G, B, tw, sel->max_cand, n_src);
+    for (int d = tw + 1; d <= wpc && rb < 32; ++d)
+      if (wpc % d == 0) {
+        tw = d;
+        rb = step_row_buf(D, G, B, tw, sel->max_cand, n_src);
+      }
+    if (rb < 8) plan->fused = false;
+  }
+  if (!plan->fused) {
+    plan->bytes = plan->attn.bytes;
+    return MPC_OK;
+  }
+  // tiles per chunk: about three chunks per warp of the grid over the
+  // longest lists the capacities allow, at least two tiles
+  const long long tt_max = (s + 15) / 16;  // the tail rows and the appended row
+  const long long ntm = tt_max + ((long long)t.sel_cap * s + 15) / 16;
+  int ct = a->chunk_tiles;
+  if (ct == 0) {
+    const long long warps = (long long)kStepCtasMax * wpc;
+    const long long want = ((long long)units * ntm + 3 * warps - 1) / (3 * warps);
+    ct = (int)(want < 2 ? 2 : (want > 32 ? 32 : want));
+  }
+  if (s < 16) {  // a chunk's selected ids must fit a warp's staging buffer
+    const int lim = (kStepSelIds - 2) * s / 16;
+    if (ct > lim) ct = lim < 1 ? 1 : lim;
+  }
+  const long long chunks = (long long)units * ((ntm + ct - 1) / ct);
+  if (chunks >= (1ll << 31)) return fail(MPC_ERR_BAD_SHAPE, "%lld attention chunks exceed one call", chunks);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off += (bytes + 255) & ~size_t(255);
+    return o;
+  };
+  plan->part_off = take((size_t)chunks * G * (D + 4) * sizeof(float));
+  plan->ucnt_off = take((size_t)units * sizeof(int));
+  plan->ready_off = take((size_t)plan->sel_units * sizeof(unsigned));
+  plan->cnt_off = take((size_t)plan->sel_units * sizeof(int));
+  plan->ctl_off = take(8 * sizeof(int));
+  plan->bytes = off;
+
+  sp->sel_out = const_cast<int*>(t.sel);
+  sp->n_sel_out = const_cast<int*>(t.n_sel);
+  sp->n_sel_units = plan->sel_units;
+  for (int l = 0; l < kMaxLevels; ++l) sp->keep_ppm[l] = sel->keep_ppm[l];
+  sp->metric = a->metric;
+  sp->src0 = a->metric == MPC_SIM_MEAN ? t.mean : (n_src == 2 ? t.r_max : t.rep);
+  sp->src1 = t.r_min;
+  sp->n_src = n_src;
+  sp->max_cand = sel->max_cand;
+  sp->row_buf = rb;
+  sp->spec = a->speculate < 0 ? select_spec_first(plan->sel_units) : a->speculate;
+  sp->team_warps = tw;
+  sp->chunk_tiles = ct;
+  return MPC_OK;
+}
+
 int cuda_fail(cudaError_t e, const char* what) {
   return fail(MPC_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
 }
@@ -444,9 +587,9 @@ MPC_API int mpc_device_status(int* flags) {
   if (flags == nullptr) return fail(MPC_ERR_INVALID_ARG, "flags is NULL");
   const cudaError_t e = cudaDeviceSynchronize();
   if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
-  const int parts[7] = {take_status_attn(),   take_status_select(),   take_status_clusters(),
+  const int parts[8] = {take_status_attn(),   take_status_select(),   take_status_clusters(),
                         take_status_static(), take_status_score_tc(), take_status_commonality(),
-                        take_status_selftest()};
+                        take_status_selftest(), take_status_step()};
   int v = 0;
   for (int x : parts) {
     if (x < 0) return fail(MPC_ERR_CUDA, "reading the device status word failed");
@@ -575,6 +718,52 @@ MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace, s
   p.grid_counter = reinterpret_cast<int*>(ws + plan.gcnt_off);
   const cudaError_t e = launch_attn(p, args->dtype, args->head_dim, plan.units, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "mpc_sparse_decode_attn launch");
+  return ok();
+}
+
+MPC_API int mpc_decode_step_workspace_size(const mpc_decode_args* args, size_t* bytes) {
+  if (bytes == nullptr) return fail(MPC_ERR_INVALID_ARG, "bytes is NULL");
+  StepParams sp;
+  SelectParams sel;
+  StepPlan plan;
+  MPC_TRY(validate_step(args, &sp, &sel, &plan));
+  *bytes = plan.bytes;
+  return ok();
+}
+
+MPC_API int mpc_decode_step(const mpc_decode_args* args, void* workspace, size_t workspace_bytes, void* stream) {
+  StepParams sp;
+  SelectParams sel;
+  StepPlan plan;
+  MPC_TRY(validate_step(args, &sp, &sel, &plan));
+  const mpc_attn_args& t = args->attn;
+  if (!t.q || !t.k_new || !t.v_new || !t.kc || !t.vc || !t.n_tok || !t.out || !t.sel || !t.n_sel)
+    return fail(MPC_ERR_INVALID_ARG, "a required pointer is NULL");
+  if (!t.rep || !t.r_max || !t.r_min) return fail(MPC_ERR_INVALID_ARG, "the summary pyramid (r_max, r_min, rep) is required");
+  if (args->metric == MPC_SIM_MEAN && !t.mean) return fail(MPC_ERR_INVALID_ARG, "MPC_SIM_MEAN needs mean");
+  if (workspace == nullptr || workspace_bytes < plan.bytes)
+    return fail(MPC_ERR_WORKSPACE, "workspace of %zu bytes needed", plan.bytes);
+  if (!aligned16(workspace)) return fail(MPC_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (plan.fused) {
+    sp.a.part = reinterpret_cast<float*>(ws + plan.part_off);
+    sp.a.unit_counter = reinterpret_cast<int*>(ws + plan.ucnt_off);
+    sp.ready = reinterpret_cast<unsigned*>(ws + plan.ready_off);
+    sp.sel_cnt = reinterpret_cast<int*>(ws + plan.cnt_off);
+    sp.ctl = reinterpret_cast<int*>(ws + plan.ctl_off);
+    e = launch_step(sp, t.head_dim, st);
+    if (e != cudaSuccess) return cuda_fail(e, "mpc_decode_step launch");
+    return ok();
+  }
+  e = launch_select(sel, t.dtype, t.head_dim, plan.sel_units, st);
+  if (e != cudaSuccess) return cuda_fail(e, "mpc_decode_step select launch");
+  sp.a.part = reinterpret_cast<float*>(ws + plan.attn.part_off);
+  sp.a.unit_counter = reinterpret_cast<int*>(ws + plan.attn.ucnt_off);
+  sp.a.grid_counter = reinterpret_cast<int*>(ws + plan.attn.gcnt_off);
+  e = launch_attn(sp.a, t.dtype, t.head_dim, plan.attn.units, st);
+  if (e != cudaSuccess) return cuda_fail(e, "mpc_decode_step attention launch");
   return ok();
 }
 

@@ -16,6 +16,7 @@
 #include <mutex>
 
 #include "kernels.cuh"
+#include "seal.cuh"
 
 namespace mpc {
 
@@ -206,72 +207,12 @@ __device__ void merge_and_store(const AttnParams& p, const Unit& u, float* mw, i
   if (tid == 0) p.unit_counter[unit] = 0;
 }
 
-// Writes the appended row of this unit into the cache (and into the stage
-// buffers when `sK` is given) and, when the tail fills up, seals it as a new
-// finest-level cluster of a leader's pyramid.
+// Seals a full tail as a new finest-level cluster of a leader's pyramid
+// (the pyramid update itself is seal_cluster in seal.cuh).
 template <typename T, int D>
 __device__ void seal_tail(const AttnParams& p, const Unit& u, const T* kcache) {
-  const int s = p.pyr.s;
-  if (!(u.leader && u.tail + 1 == s && p.rmax != nullptr)) return;
-  const int lane = threadIdx.x & 31;  // called by one warp
-  const int c_new = u.C1;
-  if (c_new >= p.pyr.cap[0]) {
-    if (lane == 0) atomicOr(&g_mpc_status, 2);
-    return;
-  }
-  constexpr int PER = D / 32;
-  float mx[PER], mn[PER], sm[PER];
-#pragma unroll
-  for (int i = 0; i < PER; ++i) {
-    mx[i] = kNegInf;
-    mn[i] = -kNegInf;
-    sm[i] = 0.f;
-  }
-#pragma unroll 8
-  for (int r = c_new * s; r < c_new * s + s; ++r) {
-    const T* row = kcache + (int64_t)r * D;
-#pragma unroll
-    for (int i = 0; i < PER; ++i) {
-      const int c = lane * PER + i;
-      const float v = to_float<T>(row[swz<T>(r, c)]);
-      mx[i] = fmaxf(mx[i], v);
-      mn[i] = fminf(mn[i], v);
-      sm[i] += v;
-    }
-  }
-  const int64_t ubase = ((int64_t)(u.group * p.B + u.b) * p.Hkv + u.h) * p.pyr.rows;
-  const float a = p.alpha, am = 1.f - p.alpha;
-  int prod = 1;
-  for (int l = 0; l < p.pyr.n_levels; ++l) {
-    if (l > 0) prod *= p.pyr.fanout[l - 1];
-    const int node = c_new / prod;
-    const bool fresh = (c_new % prod) == 0;
-    if (node >= p.pyr.cap[l]) {
-      if (lane == 0) atomicOr(&g_mpc_status, 2);
-      return;
-    }
-    float* Rx = p.rmax + (ubase + p.pyr.off[l] + node) * D;
-    float* Rn = p.rmin + (ubase + p.pyr.off[l] + node) * D;
-    float* Rp = p.rep + (ubase + p.pyr.off[l] + node) * D;
-    float* Rm = p.mean ? p.mean + (ubase + p.pyr.off[l] + node) * D : nullptr;
-    const int n_old = c_new - node * prod;  // finest clusters the node held before
-#pragma unroll
-    for (int i = 0; i < PER; ++i) {
-      const int c = lane * PER + i;
-      float x = mx[i], n = mn[i];
-      if (!fresh) {
-        x = fmaxf(x, Rx[c]);
-        n = fminf(n, Rn[c]);
-      }
-      Rx[c] = x;
-      Rn[c] = n;
-      Rp[c] = fmaf(a, x, am * n);
-      if (Rm) {  // running mean over the node's finest clusters
-        const float m_new = sm[i] / (float)s;
-        Rm[c] = fresh ? m_new : fmaf((float)n_old, Rm[c], m_new) / (float)(n_old + 1);
-      }
-    }
-  }
+  if (!(u.leader && u.tail + 1 == p.pyr.s && p.rmax != nullptr)) return;
+  seal_cluster<T, D>(p, u.group, u.b, u.h, u.C1, kcache);
 }
 
 __device__ __forceinline__ void finish_grid(const AttnParams& p) {

@@ -39,6 +39,30 @@ struct AttnParams {
   int* grid_counter;  // [1]
 };
 
+// Fused decode step: the leaders' hierarchical selection and every ref's
+// append + sparse attention in one persistent launch (decode_step.cu).
+struct StepParams {
+  AttnParams a;                // attention part; a.sel / a.n_sel are the selections
+  int* sel_out;                // written by the in-call selection (the same array as a.sel)
+  int* n_sel_out;              // [B]
+  int n_sel_units;             // leader refs x B x Hkv; 0 = attention only (selections are inputs)
+  int16_t lead_ref[kMaxRefs];  // ref index of the i-th leader ref
+  int16_t lead_of[kMaxRefs];   // for each ref: index among the leader refs of its group's leader
+  int keep_ppm[kMaxLevels];
+  int metric;                  // MPC_SIM_EQ3, _BOUND or _MEAN
+  const float* src0;           // staged summary rows: rep (Eq. 3), mean, or r_max (Eq. 2)
+  const float* src1;           // r_min (Eq. 2)
+  int n_src;
+  int max_cand;                // power of two, capacity of a team's candidate arrays
+  int row_buf;                 // summary rows a team stages at once
+  int spec;                    // the first round also stages the level below the coarsest
+  int team_warps;              // warps per selection team (divides the CTA's warps)
+  int chunk_tiles;             // tiles per attention chunk
+  unsigned* ready;             // [n_sel_units]: epoch + 1 once the unit's ids are published
+  int* sel_cnt;                // [n_sel_units]: selected clusters of each unit
+  int* ctl;                    // [8]: claim counters, grid ticket, epoch, abort flag
+};
+
 struct SelectParams {
   RefTable refs;
   int n_refs, B, Hq, Hkv, G;
@@ -144,6 +168,17 @@ cudaError_t launch_attn(const AttnParams& p, int dtype, int D, int n_units, cuda
 int attn_smem_bytes(int dtype, int D, int G, int B);
 int attn_persist_ctas_max();
 int attn_persist_batch_max();
+cudaError_t launch_step(const StepParams& p, int D, cudaStream_t st);
+int step_smem_bytes(int D, int G, int B);
+// CTA shape of the fused step kernel: warps per CTA and ring stages per warp
+void step_shape(int D, int G, int B, int* wpc, int* nst);
+// Summary rows a selection team of team_warps warps stages at once (0 if
+// its scratch cannot hold the candidate arrays).
+int step_row_buf(int D, int G, int B, int team_warps, int max_cand, int n_src);
+constexpr int kStepSelIds = 256;  // selected ids a warp of the step kernel stages per chunk
+constexpr int kStepCtasMax = 152;
+int step_ctas();
+int take_status_step();
 cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cudaStream_t st);
 int select_smem_bytes(int D, int max_cand, int row_buf, int n_src);
 int select_spec_first(int units);

@@ -27,6 +27,7 @@
 //   3. the block writes the kept clusters' children as the next level's
 //      keys, with their scores when the first round computed them.
 #include "kernels.cuh"
+#include "sel_score.cuh"
 
 namespace mpc {
 
@@ -39,10 +40,6 @@ constexpr int kSelChunk = 8192; // bytes per bulk copy
 // paged workload: 4 (120 registers) 178 us per step, 5 (96) 153 us, 6 and 8
 // (80 and 64, with spills) 159 and 167 us.
 constexpr int kSelMinCtas128 = 5;
-
-__device__ __forceinline__ unsigned long long sel_key(uint32_t oscore, int id) {
-  return ((unsigned long long)oscore << 32) | (unsigned long long)(0xffffffffu - (uint32_t)id);
-}
 
 // Fixed-point Eq. 3 (ring Z_{2^64}, f fractional bits) of four channels:
 // sum_j q_j rep_j with rep_j = tr(a enc(r_max_j)) + tr(b enc(r_min_j)), the
@@ -68,9 +65,6 @@ __device__ __forceinline__ uint32_t fxp_oscore(unsigned long long acc, int f) {
   long long v = (long long)acc >> f;
   v = v > 2147483647ll ? 2147483647ll : (v < -2147483648ll ? -2147483648ll : v);
   return (uint32_t)(int32_t)v ^ 0x80000000u;
-}
-__device__ __forceinline__ int key_id(unsigned long long key) {
-  return (int)(0xffffffffu - (uint32_t)(key & 0xffffffffull));
 }
 
 // Shared-memory layout of one select CTA (host and device): n_src staged
@@ -178,39 +172,20 @@ __global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_ker
       }
     } else {
       // 4 lanes per row, each with a quarter of the channels and that
-      // quarter of q in registers: chunk ql + 4 ((j + rot) % V4) of the row
-      // for j < V4, rotated by the row's parity so that the 32 lanes of a
-      // read hit 8 distinct 16-byte bank groups (4 wavefronts, the minimum)
+      // quarter of q in registers (row_partial: reads rotated by the row's
+      // parity against bank conflicts, products summed in channel order)
       constexpr int V4 = D / 16;  // float4 chunks per lane
       const int ql = lane & 3, rs = lane >> 2, rot = rs & 1;
       float4 qv[V4];
 #pragma unroll
-      for (int jj = 0; jj < V4; ++jj) qv[jj] = reinterpret_cast<const float4*>(qsum)[ql + 4 * ((jj + rot) % V4)];
+      for (int jj = 0; jj < V4; ++jj) qv[jj] = reinterpret_cast<const float4*>(qsum)[ql + 4 * jj];
       for (int r0 = warp * 8; r0 < nrows; r0 += NW * 8) {
         const int r = r0 + rs;
-        float ax = 0.f, ay = 0.f, az = 0.f, aw = 0.f;
+        float a = 0.f;
         if (r < nrows) {
-          const float4* rp = reinterpret_cast<const float4*>(rows + (size_t)r * D);
-          const float4* rp2 = reinterpret_cast<const float4*>(rows2 + (size_t)r * D);
-#pragma unroll
-          for (int jj = 0; jj < V4; ++jj) {
-            const int c = ql + 4 * ((jj + rot) % V4);
-            const float4 v = rp[c];
-            if (NSRC == 1) {
-              ax = fmaf(v.x, qv[jj].x, ax);
-              ay = fmaf(v.y, qv[jj].y, ay);
-              az = fmaf(v.z, qv[jj].z, az);
-              aw = fmaf(v.w, qv[jj].w, aw);
-            } else {
-              const float4 m = rp2[c];
-              ax += fmaxf(qv[jj].x * v.x, qv[jj].x * m.x);
-              ay += fmaxf(qv[jj].y * v.y, qv[jj].y * m.y);
-              az += fmaxf(qv[jj].z * v.z, qv[jj].z * m.z);
-              aw += fmaxf(qv[jj].w * v.w, qv[jj].w * m.w);
-            }
-          }
+          a = NSRC == 1 ? row_partial<D, false>(rows + (size_t)r * D, nullptr, qv, ql, rot)
+                        : row_partial<D, true>(rows + (size_t)r * D, rows2 + (size_t)r * D, qv, ql, rot);
         }
-        float a = (ax + ay) + (az + aw);
         a += __shfl_xor_sync(0xffffffffu, a, 1);
         a += __shfl_xor_sync(0xffffffffu, a, 2);
         if (ql == 0 && r < nrows) put(r, orderable(a));
@@ -282,7 +257,7 @@ __global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_ker
     const int nC = top > 0 ? C[top - 1] : 0;
     const int own = n < nT0 ? n : nT0;
     score_rows(spec0 ? capT + nC : own, [&](int r, uint32_t sc) {
-      if (r < own) keysA[r] = sel_key(sc, r);
+      if (r < own) keysA[r] = cand_key(sc, r);
       else if (r >= capT) cs[r - capT] = sc;
     });
     __syncthreads();
@@ -296,7 +271,7 @@ __global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_ker
           warp_copy(rows + (size_t)w * RB * D, src0[w] + offT + (int64_t)x0 * D, (uint32_t)nb * ROWB, &s_bar, lane);
       }
       wait_rows();
-      score_rows(nb, [&](int r, uint32_t sc) { keysA[x0 + r] = sel_key(sc, x0 + r); });
+      score_rows(nb, [&](int r, uint32_t sc) { keysA[x0 + r] = cand_key(sc, x0 + r); });
       __syncthreads();
     }
   }
@@ -317,13 +292,13 @@ __global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_ker
         const int x1 = min(n, x0 + RB);
         for (int c = tid; c < (x1 - x0) * CPR; c += NT) {
           const int r = c / CPR, part = c - r * CPR;
-          const int64_t srow = offL + (int64_t)key_id(keysA[x0 + r]) * D + part * 4;
+          const int64_t srow = offL + (int64_t)cand_id(keysA[x0 + r]) * D + part * 4;
           for (int w = 0; w < NSRC; ++w) cp_async16(rows + ((size_t)w * RB + r) * D + part * 4, src0[w] + srow);
         }
         cp_async_commit();
         cp_async_wait<0>();
         __syncthreads();
-        score_rows(x1 - x0, [&](int r, uint32_t sc) { keysA[x0 + r] = sel_key(sc, key_id(keysA[x0 + r])); });
+        score_rows(x1 - x0, [&](int r, uint32_t sc) { keysA[x0 + r] = cand_key(sc, cand_id(keysA[x0 + r])); });
         __syncthreads();
       }
     }
@@ -356,18 +331,18 @@ __global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_ker
           const unsigned bal = __ballot_sync(0xffffffffu, keep);
           if (keep) {
             const int pos = __popc(bal & lt);
-            const int id = key_id(ki);
+            const int id = cand_id(ki);
             if (lw == 0) {
               if (pos < p.sel_cap) out[pos] = id;
             } else {
               for (int j = 0; j < fw; ++j) {
                 const int cid = id * fw + j;
-                if (cid < nCw) kb[pos * fw + j] = hc ? sel_key(cs[lane * fw + j], cid) : sel_key(0u, cid);
+                if (cid < nCw) kb[pos * fw + j] = hc ? cand_key(cs[lane * fw + j], cid) : cand_key(0u, cid);
               }
             }
           }
           const int base = __popc(bal);
-          const int last = bal ? __shfl_sync(0xffffffffu, key_id(ki), 31 - __clz(bal)) : -1;
+          const int last = bal ? __shfl_sync(0xffffffffu, cand_id(ki), 31 - __clz(bal)) : -1;
           nkw = base;
           if (lw == 0) {
             flags |= 8;
@@ -451,7 +426,7 @@ __global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_ker
       int nn = 0;
       if (l > 0 && total > 0) {
         const int wl = 31 - __clz(has);
-        const int last = key_id(keysA[wl * C + 31 - __clz(s_wmask[wl])]);
+        const int last = cand_id(keysA[wl * C + 31 - __clz(s_wmask[wl])]);
         nn = (total - 1) * f + min(f, nC - last * f);
       }
       const bool fits = l == 0 || nn <= MC;
@@ -459,13 +434,13 @@ __global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_ker
         const int c = __ffs(mk) - 1;
         const int pos = before + __popc(wmask & ((1u << c) - 1u));
         const int i = c0 + c;
-        const int id = key_id(keysA[i]);
+        const int id = cand_id(keysA[i]);
         if (l == 0) {
           if (lane == 0 && pos < p.sel_cap) out[pos] = id;
         } else {
           for (int j = lane; j < f; j += 32) {
             const int cid = id * f + j;
-            if (cid < nC) keysB[pos * f + j] = have_child ? sel_key(cs[i * f + j], cid) : sel_key(0u, cid);
+            if (cid < nC) keysB[pos * f + j] = have_child ? cand_key(cs[i * f + j], cid) : cand_key(0u, cid);
           }
         }
       }
@@ -554,7 +529,7 @@ __global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_ker
           if (fl4[c]) {
             const int pos = nkw + __popc(bal[c] & lt);
             kept[pos] = i0 + 32 * c + lane;
-            if (l == 0 && pos < p.sel_cap) out[pos] = key_id(keysA[i0 + 32 * c + lane]);
+            if (l == 0 && pos < p.sel_cap) out[pos] = cand_id(keysA[i0 + 32 * c + lane]);
           }
           nkw += __popc(bal[c]);
         }
@@ -566,7 +541,7 @@ __global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_ker
         // cluster of the level, which can only be the last kept one
         int nxt = 0;
         if (l > 0 && nkw > 0) {
-          const int last = key_id(keysA[kept[nkw - 1]]);
+          const int last = cand_id(keysA[kept[nkw - 1]]);
           nxt = (nkw - 1) * f + min(f, nC - last * f);
         }
         s_next = nxt;
@@ -585,8 +560,8 @@ __global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_ker
     for (int x = tid; x < nn; x += NT) {
       const int kk = x / f, j = x - kk * f;
       const int i = kept[kk];
-      const int id = key_id(keysA[i]) * f + j;
-      keysB[x] = have_child ? sel_key(cs[i * f + j], id) : sel_key(0u, id);
+      const int id = cand_id(keysA[i]) * f + j;
+      keysB[x] = have_child ? cand_key(cs[i * f + j], id) : cand_key(0u, id);
     }
     need_score = !have_child;
     have_child = false;

@@ -28,7 +28,7 @@ MPC_F32, MPC_BF16 = 0, 1
 MPC_SIM_EQ3, MPC_SIM_BOUND, MPC_SIM_MEAN, MPC_SIM_FXP = 0, 1, 2, 3
 FXP_FRAC_BITS = 18
 MAX_LEVELS = 4
-ABI_VERSION = 5
+ABI_VERSION = 6
 MAX_REFS = 128
 PPM = 1_000_000
 
@@ -107,11 +107,19 @@ class AttnArgs(C.Structure):
                 ("mean", C.c_void_p)]
 
 
+class DecodeArgs(C.Structure):
+    """mpc_decode_args: the arguments of mpc_decode_step (attention arguments plus selection settings)."""
+    _fields_ = [("struct_size", C.c_uint32), ("attn", AttnArgs), ("level_keep_ppm", C.c_int32 * MAX_LEVELS),
+                ("metric", C.c_int32), ("frac_bits", C.c_int32), ("chunk_tiles", C.c_int32),
+                ("speculate", C.c_int32)]
+
+
 ENTRY_POINTS = ("mpc_static_evict_workspace_size", "mpc_build_clusters_workspace_size",
                 "mpc_select_workspace_size", "mpc_sparse_decode_attn_workspace_size",
                 "mpc_static_evict", "mpc_build_clusters", "mpc_select", "mpc_sparse_decode_attn",
                 "mpc_summary_rows", "mpc_last_error", "mpc_device_status", "mpc_abi_version",
-                "mpc_sparse_decode_attn_static_scratch", "mpc_commonality", "mpc_selftest_wait")
+                "mpc_sparse_decode_attn_static_scratch", "mpc_commonality", "mpc_selftest_wait",
+                "mpc_decode_step_workspace_size", "mpc_decode_step")
 
 _LIB = None
 
@@ -131,10 +139,12 @@ def load(path: Optional[str] = None) -> C.CDLL:
         raise OSError(f"libmpcache.so not found at {p}; run paper_2501_06807_gb300.build.build()")
     lib = C.CDLL(p)
     for name in ("mpc_static_evict_workspace_size", "mpc_build_clusters_workspace_size",
-                 "mpc_select_workspace_size", "mpc_sparse_decode_attn_workspace_size"):
+                 "mpc_select_workspace_size", "mpc_sparse_decode_attn_workspace_size",
+                 "mpc_decode_step_workspace_size"):
         getattr(lib, name).restype = C.c_int
         getattr(lib, name).argtypes = [C.c_void_p, C.POINTER(C.c_size_t)]
-    for name in ("mpc_static_evict", "mpc_build_clusters", "mpc_select", "mpc_sparse_decode_attn"):
+    for name in ("mpc_static_evict", "mpc_build_clusters", "mpc_select", "mpc_sparse_decode_attn",
+                 "mpc_decode_step"):
         getattr(lib, name).restype = C.c_int
         getattr(lib, name).argtypes = [C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]
     lib.mpc_summary_rows.restype = C.c_int64
@@ -537,8 +547,34 @@ class Engine:
         ws = _ws_zero(n.value, self._ws, "attn")
         _check(lib.mpc_sparse_decode_attn(C.byref(a), C.c_void_p(_ptr(ws)), n.value, C.c_void_p(_stream())))
 
-    def decode_step(self, q, k_new, v_new, out=None):
-        """One decode step of every layer: q [L][B][Hq][d], k_new / v_new
-        [L][B][Hkv][d] (layer index = position along dim 0)."""
+    def step_args(self, q, k_new, v_new, advance=True, out=None, metric: int = MPC_SIM_EQ3,
+                  frac_bits: int = FXP_FRAC_BITS, chunk_tiles: int = 0, speculate: int = -1) -> DecodeArgs:
+        """The checked mpc_decode_args of one whole decode step of every
+        processed layer (selection of the leaders, then attention)."""
+        a = DecodeArgs()
+        a.struct_size = C.sizeof(DecodeArgs)
+        att = self.attn_args(q, k_new, v_new, advance, out=out)
+        a.attn = att  # copied into the struct; its refs pointer still names att's array
+        a._refs = att._refs  # which stays alive as long as the args
+        a.level_keep_ppm = _fan(self.level_keep_ppm)
+        a.metric, a.frac_bits, a.chunk_tiles, a.speculate = metric, frac_bits, chunk_tiles, speculate
+        return a
+
+    def decode_step(self, q, k_new, v_new, out=None, metric: int = MPC_SIM_EQ3, chunk_tiles: int = 0,
+                    speculate: int = -1):
+        """One decode step of every layer in one call (mpc_decode_step):
+        q [L][B][Hq][d], k_new / v_new [L][B][Hkv][d] (layer index = position
+        along dim 0).  Same selections and outputs as ``select`` followed by
+        ``attend``."""
+        lib = load()
+        a = self.step_args(q, k_new, v_new, True, out, metric, chunk_tiles=chunk_tiles, speculate=speculate)
+        n = C.c_size_t(0)
+        _check(lib.mpc_decode_step_workspace_size(C.byref(a), C.byref(n)))
+        ws = _ws_zero(n.value, self._ws, "step")
+        _check(lib.mpc_decode_step(C.byref(a), C.c_void_p(_ptr(ws)), n.value, C.c_void_p(_stream())))
+
+    def decode_step_two_calls(self, q, k_new, v_new, out=None):
+        """The same decode step as two calls: ``select`` (leaders), then
+        ``attend`` (every layer)."""
         self.select(q)
         self.attend(q, k_new, v_new, advance=True, out=out)

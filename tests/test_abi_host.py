@@ -33,14 +33,14 @@ def test_exports_every_declared_symbol(lib):
                          capture_output=True, text=True).stdout
     exported = set(re.findall(r"\b(mpc_\w+)\b", out))
     assert set(names) <= exported
-    assert lib.mpc_abi_version() == mpcache.ABI_VERSION == 5
+    assert lib.mpc_abi_version() == mpcache.ABI_VERSION == 6
 
 
 def test_struct_layout_matches_c(tmp_path):
     structs = {"mpc_layer_ref": mpcache.LayerRef, "mpc_kv_tensor": mpcache.KvTensor,
                "mpc_static_args": mpcache.StaticArgs, "mpc_cluster_args": mpcache.ClusterArgs,
                "mpc_select_args": mpcache.SelectArgs, "mpc_attn_args": mpcache.AttnArgs,
-               "mpc_commonality_args": mpcache.CommonalityArgs}
+               "mpc_commonality_args": mpcache.CommonalityArgs, "mpc_decode_args": mpcache.DecodeArgs}
     lines = ['#include <stdio.h>', '#include <stddef.h>', '#include "mpcache.h"', 'int main(void){']
     for cname, py in structs.items():
         lines.append(f'printf("{cname} size %zu\\n", sizeof({cname}));')
@@ -271,3 +271,53 @@ def test_static_args_need_the_engines_window_rows():
     eng.win_rows = 52
     with pytest.raises(ValueError, match="window rows"):
         eng.static_args(torch.zeros(1), torch.zeros((1, 1, 2, 51, 64), dtype=torch.bfloat16), torch.zeros(1))
+
+
+def _step_args(**over):
+    a = mpcache.DecodeArgs()
+    a.struct_size = C.sizeof(mpcache.DecodeArgs)
+    att = _attn_args()
+    a.attn = att
+    a._refs = att._refs
+    a.level_keep_ppm[0], a.level_keep_ppm[1] = 125_000, 500_000
+    a.metric, a.speculate = mpcache.MPC_SIM_EQ3, -1
+    for k, v in over.items():
+        setattr(a, k, v)
+    return a
+
+
+def test_decode_step_validation(lib):
+    """mpc_decode_step checks the attention arguments like
+    mpc_sparse_decode_attn, the selection settings like mpc_select, and that
+    every ref's group is led by a ref of the call, before any CUDA call."""
+    rc, n = _ws(lib, "mpc_decode_step_workspace_size", _step_args())
+    assert rc == 0 and n > 0, lib.mpc_last_error()
+    cases = [
+        (dict(struct_size=8), mpcache.MPC_ERR_INVALID_ARG),
+        (dict(chunk_tiles=65), mpcache.MPC_ERR_BAD_SHAPE),
+        (dict(chunk_tiles=-1), mpcache.MPC_ERR_BAD_SHAPE),
+        (dict(speculate=2), mpcache.MPC_ERR_BAD_SHAPE),
+        (dict(metric=9), mpcache.MPC_ERR_INVALID_ARG),
+    ]
+    for over, code in cases:
+        rc, _ = _ws(lib, "mpc_decode_step_workspace_size", _step_args(**over))
+        assert rc == code, (over, rc, lib.mpc_last_error())
+    a = _step_args()
+    a.level_keep_ppm[1] = 0
+    assert _ws(lib, "mpc_decode_step_workspace_size", a)[0] == mpcache.MPC_ERR_BAD_SHAPE
+    a = _step_args()
+    a.attn.head_dim = 96  # the embedded attention arguments are checked too
+    assert _ws(lib, "mpc_decode_step_workspace_size", a)[0] == mpcache.MPC_ERR_BAD_SHAPE
+    # a group whose leader is not among the refs, and a group with two leaders
+    for pairs in (((1, 0, 0), (2, 0, 0)), ((0, 0, 1), (1, 0, 1))):
+        a = _step_args()
+        refs = (mpcache.LayerRef * 2)(*[mpcache.LayerRef(*p) for p in pairs])
+        a.attn.refs = C.cast(refs, C.POINTER(mpcache.LayerRef))
+        assert _ws(lib, "mpc_decode_step_workspace_size", a)[0] == mpcache.MPC_ERR_INVALID_ARG
+        assert b"leader" in lib.mpc_last_error()
+    # the call rejects a missing workspace before launching anything
+    a = _step_args()
+    a.attn.n_tok = a.attn.out = a.attn.sel = a.attn.n_sel = 8192
+    a.attn.rep = a.attn.r_max = a.attn.r_min = 16384
+    assert lib.mpc_decode_step(C.byref(a), None, 0, None) == mpcache.MPC_ERR_WORKSPACE
+    assert lib.mpc_decode_step(None, None, 0, None) == mpcache.MPC_ERR_INVALID_ARG
