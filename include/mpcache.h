@@ -314,27 +314,25 @@ MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace,
  *   MPC_SIM_FXP; r_max, r_min and rep are also updated by the seal).
  * - level_keep_ppm, metric, frac_bits: as in mpc_select_args (alpha is
  *   attn.alpha).
- * - chunk_tiles: 16-row tiles per unit of attention work a warp claims at a
- *   time (1 .. 64; 0 picks one from the sizes).
  * - speculate: -1 automatic, 0 or 1: whether the selection's first round
  *   also scores every cluster of the level below the coarsest (one
  *   dependent round fewer, more rows read).
  * With bf16 caches and the EQ3 / BOUND / MEAN metrics the step is one
- * persistent kernel: selection teams publish each unit's ids (release store
- * of a ready flag in the workspace) and the attention warps wait for them
- * (bounded, 1 s; a wait that gives up sets flag 1 of mpc_device_status and
- * the call's outputs are undefined).  Otherwise (fp32 caches, MPC_SIM_FXP,
+ * persistent kernel: selection teams publish each unit's ids in the
+ * workspace (each word tagged with the call) and the attention warps wait
+ * for them (bounded, 1 s; a wait that gives up sets flag 1 of
+ * mpc_device_status and the call's outputs are undefined).  Otherwise (fp32 caches, MPC_SIM_FXP,
  * more than 1024 candidates at a level) it is mpc_select's kernel followed
  * by mpc_sparse_decode_attn's.
  * Workspace: mpc_decode_step_workspace_size bytes, zero-filled once; the
- * call leaves its counters zero (also after a wait that gave up). */
+ * call leaves it ready for the next call, except after a wait that gave up
+ * (flag 1 of mpc_device_status): zero-fill it again before the next call. */
 typedef struct {
   uint32_t struct_size;        /* sizeof(mpc_decode_args) */
   mpc_attn_args attn;
   int32_t level_keep_ppm[MPC_MAX_LEVELS]; /* finest level first */
   int32_t metric;              /* MPC_SIM_EQ3, _BOUND, _MEAN or _FXP */
   int32_t frac_bits;           /* MPC_SIM_FXP only */
-  int32_t chunk_tiles;         /* 0 = automatic */
   int32_t speculate;           /* -1 = automatic */
 } mpc_decode_args;
 

@@ -409,7 +409,7 @@ struct StepPlan {
   AttnPlan attn;   // the two-launch path (mpc_select's and mpc_sparse_decode_attn's kernels)
   bool fused;      // one decode_step_kernel launch
   int sel_units;
-  size_t part_off, ucnt_off, ready_off, cnt_off, ctl_off, bytes;
+  size_t part_off, ucnt_off, pub_off, ctl_off, bytes;
 };
 
 int validate_step(const mpc_decode_args* a, StepParams* sp, SelectParams* sel, StepPlan* plan) {
@@ -472,7 +472,6 @@ int validate_step(const mpc_decode_args* a, StepParams* sp, SelectParams* sel, S
   sa.alpha = t.alpha;
   sa.frac_bits = a->frac_bits;
   MPC_TRY(validate_select(&sa, sel));
-  if (a->chunk_tiles < 0 || a->chunk_tiles > 64) return fail(MPC_ERR_BAD_SHAPE, "chunk_tiles %d not in [0, 64]", a->chunk_tiles);
   if (a->speculate < -1 || a->speculate > 1) return fail(MPC_ERR_BAD_SHAPE, "speculate %d not in {-1, 0, 1}", a->speculate);
 
   const int D = t.head_dim, G = sp->a.G, B = t.batch, s = t.cluster_size;
@@ -481,8 +480,9 @@ int validate_step(const mpc_decode_args* a, StepParams* sp, SelectParams* sel, S
   const int n_src = select_n_src(a->metric);
   int wpc = 0, nst = 0;
   step_shape(D, G, B, &wpc, &nst);
+  // published ids and counts are 16-bit values
   plan->fused = t.dtype == MPC_BF16 && a->metric != MPC_SIM_FXP && sel->max_cand <= 1024 &&
-                step_smem_bytes(D, G, B) <= kSmemOptin;
+                step_smem_bytes(D, G, B) <= kSmemOptin && t.cap_tokens / s < 65535 && t.sel_cap < 65535;
   int tw = 1, rb = 0;
   if (plan->fused) {
     // the largest team (divisor of the CTA's warps) that still gives every
@@ -502,32 +502,16 @@ int validate_step(const mpc_decode_args* a, StepParams* sp, SelectParams* sel, S
     plan->bytes = plan->attn.bytes;
     return MPC_OK;
   }
-  // tiles per chunk: about three chunks per warp of the grid over the
-  // longest lists the capacities allow, at least two tiles
-  const long long tt_max = (s + 15) / 16;  // the tail rows and the appended row
-  const long long ntm = tt_max + ((long long)t.sel_cap * s + 15) / 16;
-  int ct = a->chunk_tiles;
-  if (ct == 0) {
-    const long long warps = (long long)kStepCtasMax * wpc;
-    const long long want = ((long long)units * ntm + 3 * warps - 1) / (3 * warps);
-    ct = (int)(want < 2 ? 2 : (want > 32 ? 32 : want));
-  }
-  if (s < 16) {  // a chunk's selected ids must fit a warp's staging buffer
-    const int lim = (kStepSelIds - 2) * s / 16;
-    if (ct > lim) ct = lim < 1 ? 1 : lim;
-  }
-  const long long chunks = (long long)units * ((ntm + ct - 1) / ct);
-  if (chunks >= (1ll << 31)) return fail(MPC_ERR_BAD_SHAPE, "%lld attention chunks exceed one call", chunks);
   size_t off = 0;
   auto take = [&](size_t bytes) {
     const size_t o = off;
     off += (bytes + 255) & ~size_t(255);
     return o;
   };
-  plan->part_off = take((size_t)chunks * G * (D + 4) * sizeof(float));
+  // two partial records per warp slot (a later piece's, an owner's)
+  plan->part_off = take((size_t)2 * kStepCtasMax * wpc * G * (D + 4) * sizeof(float));
   plan->ucnt_off = take((size_t)units * sizeof(int));
-  plan->ready_off = take((size_t)plan->sel_units * sizeof(unsigned));
-  plan->cnt_off = take((size_t)plan->sel_units * sizeof(int));
+  plan->pub_off = take((size_t)plan->sel_units * (1 + t.sel_cap) * sizeof(unsigned));
   plan->ctl_off = take(8 * sizeof(int));
   plan->bytes = off;
 
@@ -543,7 +527,6 @@ int validate_step(const mpc_decode_args* a, StepParams* sp, SelectParams* sel, S
   sp->row_buf = rb;
   sp->spec = a->speculate < 0 ? select_spec_first(plan->sel_units) : a->speculate;
   sp->team_warps = tw;
-  sp->chunk_tiles = ct;
   return MPC_OK;
 }
 
@@ -750,8 +733,7 @@ MPC_API int mpc_decode_step(const mpc_decode_args* args, void* workspace, size_t
   if (plan.fused) {
     sp.a.part = reinterpret_cast<float*>(ws + plan.part_off);
     sp.a.unit_counter = reinterpret_cast<int*>(ws + plan.ucnt_off);
-    sp.ready = reinterpret_cast<unsigned*>(ws + plan.ready_off);
-    sp.sel_cnt = reinterpret_cast<int*>(ws + plan.cnt_off);
+    sp.sel_pub = reinterpret_cast<unsigned*>(ws + plan.pub_off);
     sp.ctl = reinterpret_cast<int*>(ws + plan.ctl_off);
     e = launch_step(sp, t.head_dim, st);
     if (e != cudaSuccess) return cuda_fail(e, "mpc_decode_step launch");

@@ -42,7 +42,7 @@ struct AttnParams {
 // Fused decode step: the leaders' hierarchical selection and every ref's
 // append + sparse attention in one persistent launch (decode_step.cu).
 struct StepParams {
-  AttnParams a;                // attention part; a.sel / a.n_sel are the selections
+  AttnParams a;                // attention part; a.part holds two records per warp slot
   int* sel_out;                // written by the in-call selection (the same array as a.sel)
   int* n_sel_out;              // [B]
   int n_sel_units;             // leader refs x B x Hkv; 0 = attention only (selections are inputs)
@@ -57,10 +57,8 @@ struct StepParams {
   int row_buf;                 // summary rows a team stages at once
   int spec;                    // the first round also stages the level below the coarsest
   int team_warps;              // warps per selection team (divides the CTA's warps)
-  int chunk_tiles;             // tiles per attention chunk
-  unsigned* ready;             // [n_sel_units]: epoch + 1 once the unit's ids are published
-  int* sel_cnt;                // [n_sel_units]: selected clusters of each unit
-  int* ctl;                    // [8]: claim counters, grid ticket, epoch, abort flag
+  unsigned* sel_pub;           // [n_sel_units][1 + sel_cap]: count, then ids, each tagged with the call
+  int* ctl;                    // [8]: claim counter, grid ticket, call counter, abort flag
 };
 
 struct SelectParams {

@@ -110,8 +110,7 @@ class AttnArgs(C.Structure):
 class DecodeArgs(C.Structure):
     """mpc_decode_args: the arguments of mpc_decode_step (attention arguments plus selection settings)."""
     _fields_ = [("struct_size", C.c_uint32), ("attn", AttnArgs), ("level_keep_ppm", C.c_int32 * MAX_LEVELS),
-                ("metric", C.c_int32), ("frac_bits", C.c_int32), ("chunk_tiles", C.c_int32),
-                ("speculate", C.c_int32)]
+                ("metric", C.c_int32), ("frac_bits", C.c_int32), ("speculate", C.c_int32)]
 
 
 ENTRY_POINTS = ("mpc_static_evict_workspace_size", "mpc_build_clusters_workspace_size",
@@ -548,7 +547,7 @@ class Engine:
         _check(lib.mpc_sparse_decode_attn(C.byref(a), C.c_void_p(_ptr(ws)), n.value, C.c_void_p(_stream())))
 
     def step_args(self, q, k_new, v_new, advance=True, out=None, metric: int = MPC_SIM_EQ3,
-                  frac_bits: int = FXP_FRAC_BITS, chunk_tiles: int = 0, speculate: int = -1) -> DecodeArgs:
+                  frac_bits: int = FXP_FRAC_BITS, speculate: int = -1) -> DecodeArgs:
         """The checked mpc_decode_args of one whole decode step of every
         processed layer (selection of the leaders, then attention)."""
         a = DecodeArgs()
@@ -557,17 +556,16 @@ class Engine:
         a.attn = att  # copied into the struct; its refs pointer still names att's array
         a._refs = att._refs  # which stays alive as long as the args
         a.level_keep_ppm = _fan(self.level_keep_ppm)
-        a.metric, a.frac_bits, a.chunk_tiles, a.speculate = metric, frac_bits, chunk_tiles, speculate
+        a.metric, a.frac_bits, a.speculate = metric, frac_bits, speculate
         return a
 
-    def decode_step(self, q, k_new, v_new, out=None, metric: int = MPC_SIM_EQ3, chunk_tiles: int = 0,
-                    speculate: int = -1):
+    def decode_step(self, q, k_new, v_new, out=None, metric: int = MPC_SIM_EQ3, speculate: int = -1):
         """One decode step of every layer in one call (mpc_decode_step):
         q [L][B][Hq][d], k_new / v_new [L][B][Hkv][d] (layer index = position
         along dim 0).  Same selections and outputs as ``select`` followed by
         ``attend``."""
         lib = load()
-        a = self.step_args(q, k_new, v_new, True, out, metric, chunk_tiles=chunk_tiles, speculate=speculate)
+        a = self.step_args(q, k_new, v_new, True, out, metric, speculate=speculate)
         n = C.c_size_t(0)
         _check(lib.mpc_decode_step_workspace_size(C.byref(a), C.byref(n)))
         ws = _ws_zero(n.value, self._ws, "step")

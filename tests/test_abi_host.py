@@ -294,8 +294,6 @@ def test_decode_step_validation(lib):
     assert rc == 0 and n > 0, lib.mpc_last_error()
     cases = [
         (dict(struct_size=8), mpcache.MPC_ERR_INVALID_ARG),
-        (dict(chunk_tiles=65), mpcache.MPC_ERR_BAD_SHAPE),
-        (dict(chunk_tiles=-1), mpcache.MPC_ERR_BAD_SHAPE),
         (dict(speculate=2), mpcache.MPC_ERR_BAD_SHAPE),
         (dict(metric=9), mpcache.MPC_ERR_INVALID_ARG),
     ]

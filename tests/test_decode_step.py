@@ -82,11 +82,10 @@ CASES = [
     ("token_wise_s1", synth.C3.replace(n_layers=2, prompt_len=1024, prompt_len_min=1024, n_q_heads=8,
                                        n_kv_heads=2, keep_ppm=1_000_000, cluster_size=1, fanouts=(16,),
                                        level_keep_ppm=(50_000, 250_000), share_every=1), 6, {}),
-    ("one_tile_chunks_no_spec", synth.C3.replace(n_layers=5, prompt_len=2048, prompt_len_min=2048,
-                                                 n_q_heads=8, n_kv_heads=2), 17,
-     dict(chunk_tiles=1, speculate=0)),
-    ("long_chunks_spec", synth.C3.replace(n_layers=5, prompt_len=2048, prompt_len_min=2048,
-                                          n_q_heads=8, n_kv_heads=2), 17, dict(chunk_tiles=7, speculate=1)),
+    ("no_speculative_round", synth.C3.replace(n_layers=5, prompt_len=2048, prompt_len_min=2048,
+                                              n_q_heads=8, n_kv_heads=2), 17, dict(speculate=0)),
+    ("speculative_round", synth.C3.replace(n_layers=5, prompt_len=2048, prompt_len_min=2048,
+                                           n_q_heads=8, n_kv_heads=2), 17, dict(speculate=1)),
     ("bound_metric", synth.C3.replace(n_layers=3, prompt_len=2048, prompt_len_min=2048, n_q_heads=8,
                                       n_kv_heads=2), 17, dict(metric=mpcache.MPC_SIM_BOUND)),
     ("mean_metric", synth.C3.replace(n_layers=3, prompt_len=2048, prompt_len_min=2048, n_q_heads=8,
@@ -108,8 +107,9 @@ def test_fused_step_equals_two_calls(name, w, E, kw):
 
 def test_fused_step_is_one_launch_in_a_graph():
     """The fused step replays inside a CUDA graph (one kernel per step, the
-    ready flags and counters of the workspace carried from replay to replay)
-    and gives the eager run's outputs."""
+    published selections and counters of the workspace carried from replay to
+    replay) and gives the eager run's outputs bit for bit (the static split
+    and the canonical merge order make them deterministic)."""
     w = synth.C3.replace(n_layers=6, prompt_len=2048, prompt_len_min=2048, n_q_heads=8, n_kv_heads=2)
     E = 20
     x = H.to_cuda(synth.generate(w, H.window_rows_for(w), device="cpu", decode_steps=E))
@@ -129,7 +129,9 @@ def test_fused_step_is_one_launch_in_a_graph():
             graphed.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=outs_g[e])
     g.replay()
     torch.cuda.synchronize()
-    assert torch.equal(outs_g, outs_e)
+    diff = (outs_g - outs_e).abs().amax(dim=(2, 3, 4))  # [step][layer]
+    bad = [(e, l, float(diff[e, l])) for e, l in zip(*torch.nonzero(diff).T.tolist())]
+    assert not bad, bad[:12]
     assert torch.equal(graphed.kc, eager.kc) and torch.equal(graphed.rep, eager.rep)
     assert mpcache.device_status() == 0
 
