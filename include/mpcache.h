@@ -350,12 +350,12 @@ MPC_API int mpc_decode_step(const mpc_decode_args* args, void* workspace, size_t
  *   GPU that loads the library until the process exits.  A call whose
  *   workspace (mpc_sparse_decode_attn_workspace_size) exceeds 4 MiB is
  *   rejected with MPC_ERR_WORKSPACE and nothing is launched.
- * - The first call on each device looks up the array's device address (with
- *   that device current); make that first call before any stream capture.
- * - Each call clears the part of the array it uses (an asynchronous memset
- *   on `stream`) and then runs the regular kernels.  Every call shares the
- *   one array: calls that overlap on the GPU (different streams, no
- *   ordering between them) race and corrupt each other's results.
+ * - Every call looks up the array's device address in the current device's
+ *   context (cudaGetSymbolAddress), clears the counters it keeps in the
+ *   array (an asynchronous memset on `stream`) and then runs the regular
+ *   kernels.  Every call shares the one array: calls that overlap on the GPU
+ *   (different streams, no ordering between them) race and corrupt each
+ *   other's results.
  * - Allocates nothing (no cudaMalloc / cudaFree). */
 MPC_API int mpc_sparse_decode_attn_static_scratch(const mpc_attn_args* args, void* stream);
 

@@ -305,7 +305,7 @@ int validate_select(const mpc_select_args* a, SelectParams* p) {
 // ---------------------------------------------------------- attention ----
 struct AttnPlan {
   int units, n_split, tps;
-  size_t part_off, ucnt_off, gcnt_off, bytes;
+  size_t part_off, ucnt_off, gcnt_off, ctl_off, bytes;
 };
 
 int validate_attn(const mpc_attn_args* a, AttnParams* p, AttnPlan* plan) {
@@ -359,14 +359,18 @@ int validate_attn(const mpc_attn_args* a, AttnParams* p, AttnPlan* plan) {
   };
   if (a->dtype == MPC_BF16) {
     // persistent kernel: two partial records per warp of the grid
-    if (a->batch > attn_persist_batch_max())
-      return fail(MPC_ERR_BAD_SHAPE, "batch %d > %d sequences per call", a->batch, attn_persist_batch_max());
-    plan->part_off = take((size_t)2 * attn_persist_ctas_max() * 4 * G * (a->head_dim + 4) * sizeof(float));
+    if (a->batch > kStepBatchMax)
+      return fail(MPC_ERR_BAD_SHAPE, "batch %d > %d sequences per call", a->batch, kStepBatchMax);
+    // the step kernel with no selection units: two partial records per warp slot
+    int wpc = 0, nst = 0;
+    step_shape(a->head_dim, G, a->batch, &wpc, &nst);
+    plan->part_off = take((size_t)2 * kStepCtasMax * wpc * G * (a->head_dim + 4) * sizeof(float));
   } else {
     plan->part_off = take(n_split > 1 ? (size_t)units * n_split * G * (a->head_dim + 4) * sizeof(float) : 0);
   }
   plan->ucnt_off = take((size_t)units * sizeof(int));
   plan->gcnt_off = take(sizeof(int));
+  plan->ctl_off = take(8 * sizeof(int));
   plan->bytes = off;
 
   p->n_refs = a->n_refs;
@@ -538,6 +542,19 @@ int cuda_fail(cudaError_t e, const char* what) {
 
 int set_error(int code, const char* msg) { return fail(code, "%s", msg); }
 
+// Byte range [off, off + bytes) of the workspace of mpc_sparse_decode_attn
+// that must be zero before a call (its counters); the rest is written before
+// it is read.
+int attn_counter_range(const mpc_attn_args* args, size_t* off, size_t* bytes) {
+  AttnParams p;
+  AttnPlan plan;
+  MPC_TRY(validate_attn(args, &p, &plan));
+  *off = plan.ucnt_off;
+  *bytes = plan.bytes - plan.ucnt_off;
+  return MPC_OK;
+}
+
+
 }  // namespace mpc
 
 using namespace mpc;
@@ -699,7 +716,17 @@ MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace, s
   p.part = reinterpret_cast<float*>(ws + plan.part_off);
   p.unit_counter = reinterpret_cast<int*>(ws + plan.ucnt_off);
   p.grid_counter = reinterpret_cast<int*>(ws + plan.gcnt_off);
-  const cudaError_t e = launch_attn(p, args->dtype, args->head_dim, plan.units, static_cast<cudaStream_t>(stream));
+  cudaError_t e;
+  if (args->dtype == MPC_BF16) {
+    // the decode step kernel with every selection an input (no selection units)
+    StepParams sp;
+    memset(&sp, 0, sizeof(sp));
+    sp.a = p;
+    sp.ctl = reinterpret_cast<int*>(ws + plan.ctl_off);
+    e = launch_step(sp, args->head_dim, static_cast<cudaStream_t>(stream));
+  } else {
+    e = launch_attn(p, args->dtype, args->head_dim, plan.units, static_cast<cudaStream_t>(stream));
+  }
   if (e != cudaSuccess) return cuda_fail(e, "mpc_sparse_decode_attn launch");
   return ok();
 }
@@ -744,7 +771,15 @@ MPC_API int mpc_decode_step(const mpc_decode_args* args, void* workspace, size_t
   sp.a.part = reinterpret_cast<float*>(ws + plan.attn.part_off);
   sp.a.unit_counter = reinterpret_cast<int*>(ws + plan.attn.ucnt_off);
   sp.a.grid_counter = reinterpret_cast<int*>(ws + plan.attn.gcnt_off);
-  e = launch_attn(sp.a, t.dtype, t.head_dim, plan.attn.units, st);
+  if (t.dtype == MPC_BF16) {  // the step kernel with the selections as inputs
+    StepParams ap;
+    memset(&ap, 0, sizeof(ap));
+    ap.a = sp.a;
+    ap.ctl = reinterpret_cast<int*>(ws + plan.attn.ctl_off);
+    e = launch_step(ap, t.head_dim, st);
+  } else {
+    e = launch_attn(sp.a, t.dtype, t.head_dim, plan.attn.units, st);
+  }
   if (e != cudaSuccess) return cuda_fail(e, "mpc_decode_step attention launch");
   return ok();
 }

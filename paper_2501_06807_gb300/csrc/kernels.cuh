@@ -162,10 +162,8 @@ __host__ __device__ inline int select_n_src(int metric) {
   return metric == MPC_SIM_BOUND || metric == MPC_SIM_FXP ? 2 : 1;
 }
 
+// fp32 attention (split grid, last-CTA merge)
 cudaError_t launch_attn(const AttnParams& p, int dtype, int D, int n_units, cudaStream_t st);
-int attn_smem_bytes(int dtype, int D, int G, int B);
-int attn_persist_ctas_max();
-int attn_persist_batch_max();
 cudaError_t launch_step(const StepParams& p, int D, cudaStream_t st);
 int step_smem_bytes(int D, int G, int B);
 // CTA shape of the fused step kernel: warps per CTA and ring stages per warp
@@ -175,6 +173,7 @@ void step_shape(int D, int G, int B, int* wpc, int* nst);
 int step_row_buf(int D, int G, int B, int team_warps, int max_cand, int n_src);
 constexpr int kStepSelIds = 256;  // selected ids a warp of the step kernel stages per chunk
 constexpr int kStepCtasMax = 152;
+constexpr int kStepBatchMax = 512;  // sequences per call (the per-sequence table lives in shared memory)
 int step_ctas();
 int take_status_step();
 cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cudaStream_t st);
@@ -187,6 +186,10 @@ cudaError_t launch_score_tc(ScoreTcParams& p, int D, int n_layer_span, cudaStrea
 // Bytes of the gathered dense copy of paged bf16 keys (0 when not needed).
 size_t static_dense_bytes(const StaticParams& p, int dtype, int D);
 int static_tile_smem(int D);
+
+// The counters of mpc_sparse_decode_attn's workspace: the byte range that
+// must be zero before a call.
+int attn_counter_range(const mpc_attn_args* args, size_t* off, size_t* bytes);
 
 // Records `msg` as this thread's last error (mpc_last_error) and returns code.
 int set_error(int code, const char* msg);

@@ -9,11 +9,8 @@
 // image, so the caller passes only inputs and outputs.
 //
 // The array is a file-scope __device__ variable.  Host code cannot use its
-// name as a device address, so the address is looked up with
-// cudaGetSymbolAddress, once per device, the first time the entry point runs
-// on that device (with that device current).
-#include <mutex>
-
+// name as a device address, so every call looks the address up with
+// cudaGetSymbolAddress in the current device's context.
 #include "kernels.cuh"
 
 namespace mpc {
@@ -23,25 +20,15 @@ constexpr size_t kStaticScratchBytes = size_t(4) << 20;  // 4 MiB per device
 
 static __device__ __align__(256) unsigned char g_attn_scratch[kStaticScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_scratch_mu;
-void* g_scratch_addr[kMaxDevices] = {};
-
-// Device address of g_attn_scratch on the current device.
+// Device address of g_attn_scratch in the current device's context, looked
+// up on every call (a cached address would dangle after a device reset or a
+// switch of context on the same ordinal).
 int scratch_address(void** out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return set_error(MPC_ERR_CUDA, cudaGetErrorString(e));
-  if (dev < 0 || dev >= kMaxDevices) return set_error(MPC_ERR_INVALID_ARG, "device ordinal out of range");
-  std::lock_guard<std::mutex> lk(g_scratch_mu);
-  if (g_scratch_addr[dev] == nullptr) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_attn_scratch);
-    if (e != cudaSuccess || p == nullptr)
-      return set_error(MPC_ERR_CUDA, "cudaGetSymbolAddress of the static scratch array failed");
-    g_scratch_addr[dev] = p;
-  }
-  *out = g_scratch_addr[dev];
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_attn_scratch);
+  if (e != cudaSuccess || p == nullptr)
+    return set_error(MPC_ERR_CUDA, "cudaGetSymbolAddress of the static scratch array failed");
+  *out = p;
   return MPC_OK;
 }
 
@@ -60,9 +47,13 @@ extern "C" MPC_API int mpc_sparse_decode_attn_static_scratch(const mpc_attn_args
   void* ws = nullptr;
   rc = scratch_address(&ws);
   if (rc != MPC_OK) return rc;
-  // the split counters must start at zero; the array keeps the previous
-  // call's contents, so clear the part this call uses
-  const cudaError_t e = cudaMemsetAsync(ws, 0, need, static_cast<cudaStream_t>(stream));
+  // the counters must start at zero; the array keeps the previous call's
+  // contents, so clear them (the partial records are written before they
+  // are read)
+  size_t coff = 0, cbytes = 0;
+  rc = attn_counter_range(args, &coff, &cbytes);
+  if (rc != MPC_OK) return rc;
+  const cudaError_t e = cudaMemsetAsync(static_cast<uint8_t*>(ws) + coff, 0, cbytes, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return set_error(MPC_ERR_CUDA, cudaGetErrorString(e));
   return mpc_sparse_decode_attn(args, ws, need, stream);
 }
