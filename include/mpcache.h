@@ -317,6 +317,11 @@ MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace,
  * - speculate: -1 automatic, 0 or 1: whether the selection's first round
  *   also scores every cluster of the level below the coarsest (one
  *   dependent round fewer, more rows read).
+ * - static_ppm, slice_tiles: the attention's tile list is cut into one
+ *   contiguous range per warp for its first static_ppm parts per million,
+ *   the rest into slices of slice_tiles tiles that warps claim once their
+ *   range is done (a balance for SMs that stream slower); 1e6 keeps every
+ *   tile static; 0 picks either.
  * With bf16 caches and the EQ3 / BOUND / MEAN metrics the step is one
  * persistent kernel: selection teams publish each unit's ids in the
  * workspace (each word tagged with the call) and the attention warps wait
@@ -334,6 +339,8 @@ typedef struct {
   int32_t metric;              /* MPC_SIM_EQ3, _BOUND, _MEAN or _FXP */
   int32_t frac_bits;           /* MPC_SIM_FXP only */
   int32_t speculate;           /* -1 = automatic */
+  int32_t static_ppm;          /* share of the attention tiles in static warp ranges; 0 = automatic */
+  int32_t slice_tiles;         /* tiles per dynamically claimed slice of the rest; 0 = automatic */
 } mpc_decode_args;
 
 MPC_API int mpc_decode_step_workspace_size(const mpc_decode_args* args, size_t* bytes);

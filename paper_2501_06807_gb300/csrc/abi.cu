@@ -103,6 +103,21 @@ int window_bound(int t_max, int wppm, int lppm, int thr) {
   return a > b ? a : b;
 }
 
+// The split of the attention tile list (static warp ranges, then dynamic
+// slices) and the range slots the partial-record arrays need, for a call of
+// `units` units of at most ntm tiles each.
+void step_balance(int units, long long ntm, int wpc, int static_ppm, int slice_tiles, StepParams* sp) {
+  // measured: slices of 2-8 tiles after a 30-80% static share were 12-50%
+  // slower than all-static ranges on the 2k, 8k and 32k workloads (each slice
+  // drains and refills its warp's ring and merges through a fenced ticket)
+  sp->static_ppm = static_ppm > 0 ? static_ppm : 1000000;
+  sp->slice_tiles = slice_tiles > 0 ? slice_tiles : 4;
+  if (sp->static_ppm >= 1000000) sp->slice_tiles = 0;  // all static
+  const long long tiles = (long long)units * ntm;
+  const long long nb = sp->slice_tiles > 0 ? (tiles + sp->slice_tiles - 1) / sp->slice_tiles + 1 : 0;
+  sp->rec_slots = (int)((long long)kStepCtasMax * wpc + nb);
+}
+
 // -------------------------------------------------------------- static ----
 int validate_static(const mpc_static_args* a, StaticParams* p) {
   if (a == nullptr) return fail(MPC_ERR_INVALID_ARG, "args is NULL");
@@ -305,6 +320,7 @@ int validate_select(const mpc_select_args* a, SelectParams* p) {
 // ---------------------------------------------------------- attention ----
 struct AttnPlan {
   int units, n_split, tps;
+  int rec_slots, static_ppm, slice_tiles;  // bf16: the step kernel's split
   size_t part_off, ucnt_off, gcnt_off, ctl_off, bytes;
 };
 
@@ -361,10 +377,16 @@ int validate_attn(const mpc_attn_args* a, AttnParams* p, AttnPlan* plan) {
     // persistent kernel: two partial records per warp of the grid
     if (a->batch > kStepBatchMax)
       return fail(MPC_ERR_BAD_SHAPE, "batch %d > %d sequences per call", a->batch, kStepBatchMax);
-    // the step kernel with no selection units: two partial records per warp slot
+    // the step kernel with no selection units: two partial records per range slot
     int wpc = 0, nst = 0;
     step_shape(a->head_dim, G, a->batch, &wpc, &nst);
-    plan->part_off = take((size_t)2 * kStepCtasMax * wpc * G * (a->head_dim + 4) * sizeof(float));
+    StepParams bal;
+    const long long ntm = (a->cluster_size + 15) / 16 + ((long long)a->sel_cap * a->cluster_size + 15) / 16;
+    step_balance(units, ntm, wpc, 0, 0, &bal);
+    plan->rec_slots = bal.rec_slots;
+    plan->static_ppm = bal.static_ppm;
+    plan->slice_tiles = bal.slice_tiles;
+    plan->part_off = take((size_t)2 * bal.rec_slots * G * (a->head_dim + 4) * sizeof(float));
   } else {
     plan->part_off = take(n_split > 1 ? (size_t)units * n_split * G * (a->head_dim + 4) * sizeof(float) : 0);
   }
@@ -512,8 +534,12 @@ int validate_step(const mpc_decode_args* a, StepParams* sp, SelectParams* sel, S
     off += (bytes + 255) & ~size_t(255);
     return o;
   };
-  // two partial records per warp slot (a later piece's, an owner's)
-  plan->part_off = take((size_t)2 * kStepCtasMax * wpc * G * (D + 4) * sizeof(float));
+  // two partial records per range slot (a later piece's, an owner's)
+  if (a->static_ppm < 0 || a->static_ppm > 1000000 || a->slice_tiles < 0 || a->slice_tiles > 64)
+    return fail(MPC_ERR_BAD_SHAPE, "static_ppm %d / slice_tiles %d out of range", a->static_ppm, a->slice_tiles);
+  const long long ntm = (s + 15) / 16 + ((long long)t.sel_cap * s + 15) / 16;
+  step_balance(units, ntm, wpc, a->static_ppm, a->slice_tiles, sp);
+  plan->part_off = take((size_t)2 * sp->rec_slots * G * (D + 4) * sizeof(float));
   plan->ucnt_off = take((size_t)units * sizeof(int));
   plan->pub_off = take((size_t)plan->sel_units * (1 + t.sel_cap) * sizeof(unsigned));
   plan->ctl_off = take(8 * sizeof(int));
@@ -723,6 +749,9 @@ MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace, s
     memset(&sp, 0, sizeof(sp));
     sp.a = p;
     sp.ctl = reinterpret_cast<int*>(ws + plan.ctl_off);
+    sp.rec_slots = plan.rec_slots;
+    sp.static_ppm = plan.static_ppm;
+    sp.slice_tiles = plan.slice_tiles;
     e = launch_step(sp, args->head_dim, static_cast<cudaStream_t>(stream));
   } else {
     e = launch_attn(p, args->dtype, args->head_dim, plan.units, static_cast<cudaStream_t>(stream));
@@ -776,6 +805,9 @@ MPC_API int mpc_decode_step(const mpc_decode_args* args, void* workspace, size_t
     memset(&ap, 0, sizeof(ap));
     ap.a = sp.a;
     ap.ctl = reinterpret_cast<int*>(ws + plan.attn.ctl_off);
+    ap.rec_slots = plan.attn.rec_slots;
+    ap.static_ppm = plan.attn.static_ppm;
+    ap.slice_tiles = plan.attn.slice_tiles;
     e = launch_step(ap, t.head_dim, st);
   } else {
     e = launch_attn(sp.a, t.dtype, t.head_dim, plan.attn.units, st);

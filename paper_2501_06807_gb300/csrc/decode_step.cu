@@ -43,7 +43,8 @@ namespace {
 constexpr int kSelIds = kStepSelIds;  // selected ids a warp stages at once
 constexpr int kMaxStepCtas = kStepCtasMax;
 // control words of the workspace
-constexpr int kCtlSelClaim = 0, kCtlTeamsDone = 1, kCtlStarted = 2, kCtlEpoch = 3;
+constexpr int kCtlSelClaim = 0, kCtlTeamsDone = 1, kCtlStarted = 2, kCtlEpoch = 3, kCtlSliceClaim = 4,
+              kCtlWarpsDone = 5;
 constexpr uint64_t kWaitNs = 1000000000ull;  // bound of every wait (1 s)
 
 __device__ __forceinline__ void named_bar(int id, int nthreads) {
@@ -555,10 +556,20 @@ __global__ void __launch_bounds__(WPC * 32, 1) decode_step_kernel(const __grid_c
   const int64_t TPR = (int64_t)Hkv * s_pre[B];
   const int64_t NT = TPR * p.n_refs;
   const int64_t NW_all = (int64_t)gridDim.x * WPC;
-  const int NW = (int)(NW_all < NT ? NW_all : NT);
+  // the list's first xA tiles are cut into equal contiguous ranges, one per
+  // warp slot (slots [0, NW), interleaved over the CTAs); the other tiles
+  // into NB equal slices (slots NW + k) that warps claim once their range is
+  // done, so that warps on slower SMs take fewer of them
+  const int64_t xA = sp.slice_tiles > 0 ? NT * (int64_t)sp.static_ppm / 1000000 : NT;
+  const int NW = (int)(NW_all < xA ? NW_all : xA);
+  const int NB = NT > xA ? (int)((NT - xA + sp.slice_tiles - 1) / sp.slice_tiles) : 0;
   const int gw = warp * gridDim.x + blockIdx.x;
-  const int64_t x0 = gw < NW ? NT * gw / NW : 0, x1 = gw < NW ? NT * (gw + 1) / NW : 0;
-  auto warp_of = [&](int64_t x) { return (int)((x * NW + NW - 1) / NT); };
+  auto slot_of = [&](int64_t x) {  // the range slot holding list tile x
+    if (x < xA) return (int)((x * NW + NW - 1) / xA);
+    return NW + (int)(((x - xA) * NB + NB - 1) / (NT - xA));
+  };
+  int64_t x0 = gw < NW ? xA * gw / NW : 0, x1 = gw < NW ? xA * (gw + 1) / NW : 0;
+  int slot = gw;  // of the current range
   bool abort = false;
 
   struct Unit {
@@ -761,8 +772,8 @@ __global__ void __launch_bounds__(WPC * 32, 1) decode_step_kernel(const __grid_c
   const int r_tok = lane >> 2;       // token row of S^T (and +8)
   const int h_off = 2 * (lane & 3);  // first of this thread's two heads in an n-tile
   const int REC = G * (D + 4);       // record: per head max (log2), sum, 2 pad, o[D]
-  float* recA = p.part;                          // [warp slot]: a later piece's record
-  float* recB = p.part + (int64_t)NW_all * REC;  // [warp slot]: an owner's record
+  float* recA = p.part;                               // [range slot]: a later piece's record
+  float* recB = p.part + (int64_t)sp.rec_slots * REC;  // [range slot]: an owner's record
 
   // folds record rec (max, sum, o) into the registers by log-sum-exp
   auto fold = [&](const float* rec, bool staged, float (&lq)[HN][2]) {
@@ -847,8 +858,8 @@ __global__ void __launch_bounds__(WPC * 32, 1) decode_step_kernel(const __grid_c
     const bool later = u.ustart < x0, owner = !later && uend > x1;
     bool write = !later && !owner;  // the whole unit is in this warp's range
     if (later || owner) {
-      const int w0 = warp_of(u.ustart);
-      const int nother = warp_of(uend - 1) - w0;  // pieces besides the owner's
+      const int w0 = slot_of(u.ustart);
+      const int nother = slot_of(uend - 1) - w0;  // pieces besides the owner's
       int* cnt = p.unit_counter + ((int64_t)u.ri * B + u.b) * Hkv + u.h;
       if (owner) {
         int done = 0;
@@ -856,11 +867,11 @@ __global__ void __launch_bounds__(WPC * 32, 1) decode_step_kernel(const __grid_c
         done = __shfl_sync(0xffffffffu, done, 0);
         if (done == nother) {
           // every later piece has published: this piece is the last; stage
-          // the later pieces' records (warps gw + 1 .. gw + nother, contiguous)
-          // in the idle ring with one batch of copies and fold them
+          // the later pieces' records (slots slot + 1 .. slot + nother,
+          // contiguous) in the idle ring with one batch of copies and fold them
           if (lane == 0) *cnt = 0;
           const bool staged = nother * REC * 4 <= NST * STAGE;
-          const float* recs = recA + (int64_t)(gw + 1) * REC;
+          const float* recs = recA + (int64_t)(slot + 1) * REC;
           if (staged) {
             const uint8_t* src = reinterpret_cast<const uint8_t*>(recs);
             for (int i = lane; i < nother * REC / 4; i += 32) cp_async16(ring + i * 16, src + i * 16);
@@ -872,18 +883,18 @@ __global__ void __launch_bounds__(WPC * 32, 1) decode_step_kernel(const __grid_c
           for (int k = 0; k < nother; ++k) fold(recs + (int64_t)k * REC, staged, lq);
           write = true;
         } else {
-          write_rec(recB + (int64_t)gw * REC, lq);
+          write_rec(recB + (int64_t)slot * REC, lq);
           __syncwarp();
           int t = 0;
           if (lane == 0) t = atom_add_acq_rel(cnt, 1);
           if (__shfl_sync(0xffffffffu, t, 0) == nother) {  // the later pieces finished meanwhile
             if (lane == 0) *cnt = 0;
-            for (int k = 1; k <= nother; ++k) fold(recA + (int64_t)(gw + k) * REC, false, lq);
+            for (int k = 1; k <= nother; ++k) fold(recA + (int64_t)(slot + k) * REC, false, lq);
             write = true;
           }
         }
       } else {
-        write_rec(recA + (int64_t)gw * REC, lq);
+        write_rec(recA + (int64_t)slot * REC, lq);
         __syncwarp();
         int t = 0;
         if (lane == 0) t = atom_add_acq_rel(cnt, 1);
@@ -924,12 +935,17 @@ __global__ void __launch_bounds__(WPC * 32, 1) decode_step_kernel(const __grid_c
     }
   };
 
+  while (true) {  // the warp's static range, then the slices it claims
   const int nj = (int)(x1 - x0);
+  ix = x0;
+  seq_i = 0;
+  iu.ustart = -1;
+  iu.nt = 0;
+  bool have = false;
   for (int j = 0; j < NST; ++j) {
     issue_one();
     cp_async_commit();
   }
-  bool have = false;
   for (int j = 0; j < nj && !abort; ++j) {
     const int slot = j % NST;
     uint8_t* sK = ring + slot * STAGE;
@@ -1075,6 +1091,21 @@ __global__ void __launch_bounds__(WPC * 32, 1) decode_step_kernel(const __grid_c
   cp_async_wait<0>();
   __syncwarp();
   if (have && !abort) flush();
+  if (abort || NB == 0) break;
+  int k = 0;
+  if (lane == 0) k = atomicAdd(&sp.ctl[kCtlSliceClaim], 1);
+  k = __shfl_sync(0xffffffffu, k, 0);
+  if (k >= NB) break;
+  x0 = xA + (NT - xA) * k / NB;
+  x1 = xA + (NT - xA) * (k + 1) / NB;
+  slot = NW + k;
+  }
+  // every slice is claimed; the last warp to leave resets the counter
+  if (NB > 0 && lane == 0 && atomicAdd(&sp.ctl[kCtlWarpsDone], 1) == (int)(gridDim.x * WPC) - 1) {
+    sp.ctl[kCtlSliceClaim] = 0;
+    sp.ctl[kCtlWarpsDone] = 0;
+  }
+
 
 }
 

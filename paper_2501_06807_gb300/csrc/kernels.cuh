@@ -57,6 +57,9 @@ struct StepParams {
   int row_buf;                 // summary rows a team stages at once
   int spec;                    // the first round also stages the level below the coarsest
   int team_warps;              // warps per selection team (divides the CTA's warps)
+  int static_ppm;              // share of the tile list cut into static warp ranges
+  int slice_tiles;             // tiles per dynamic slice of the rest (0: all static)
+  int rec_slots;               // range slots the partial-record arrays hold
   unsigned* sel_pub;           // [n_sel_units][1 + sel_cap]: count, then ids, each tagged with the call
   int* ctl;                    // [8]: claim counter, grid ticket, call counter, abort flag
 };

@@ -86,6 +86,14 @@ CASES = [
                                               n_q_heads=8, n_kv_heads=2), 17, dict(speculate=0)),
     ("speculative_round", synth.C3.replace(n_layers=5, prompt_len=2048, prompt_len_min=2048,
                                            n_q_heads=8, n_kv_heads=2), 17, dict(speculate=1)),
+    ("all_static_ranges", synth.C3.replace(n_layers=5, prompt_len=2048, prompt_len_min=2048,
+                                           n_q_heads=8, n_kv_heads=2), 17, dict(static_ppm=1_000_000)),
+    ("half_dynamic_one_tile_slices", synth.C3.replace(n_layers=5, prompt_len=2048, prompt_len_min=2048,
+                                                      n_q_heads=8, n_kv_heads=2), 17,
+     dict(static_ppm=500_000, slice_tiles=1)),
+    ("all_dynamic_slices", synth.C5.replace(n_layers=6, prompt_len=4096, prompt_len_min=4096, n_q_heads=8,
+                                            n_kv_heads=2, level_keep_ppm=(100_000, 250_000, 500_000)), 20,
+     dict(static_ppm=1, slice_tiles=3)),
     ("bound_metric", synth.C3.replace(n_layers=3, prompt_len=2048, prompt_len_min=2048, n_q_heads=8,
                                       n_kv_heads=2), 17, dict(metric=mpcache.MPC_SIM_BOUND)),
     ("mean_metric", synth.C3.replace(n_layers=3, prompt_len=2048, prompt_len_min=2048, n_q_heads=8,
