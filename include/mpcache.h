@@ -392,6 +392,29 @@ typedef struct {
 
 MPC_API int mpc_commonality(const mpc_commonality_args* args, void* stream);
 
+/* ---- mpc_layer_refs ---------------------------------------------------------
+ * Cross-layer index sharing (Sec. 3.4): the refs of a call over layers
+ * 0 .. n_layers - 1.  The first two layers are left unshared (each leads
+ * itself); from layer 2 on, consecutive groups of share_every layers reuse
+ * the indices of the group's first layer, so layer l's leader is
+ * 2 + share_every * floor((l - 2) / share_every).  share_every = 1: every
+ * layer leads.  out_refs[l] = {layer l, the group of its leader (groups
+ * numbered in layer order from 0), 1 if l leads its group}.
+ * Host only: writes n_layers entries of out_refs (host memory) and returns
+ * the number of groups, or MPC_ERR_INVALID_ARG (out_refs NULL, n_layers not
+ * in 1 .. MPC_MAX_REFS, share_every < 1). */
+MPC_API int mpc_layer_refs(int32_t n_layers, int32_t share_every, mpc_layer_ref* out_refs);
+
+/* ---- mpc_choose_share_every --------------------------------------------------
+ * The adaptive sharing-group size (Sec. 2, Observation 3; Sec. 3.4): score[m - 1]
+ * is the commonality score of windows of m + 1 adjacent layers
+ * (mpc_commonality's out_score for that m, e.g. averaged over sequences and
+ * kv heads), for m = 1 .. n.  Returns the largest m + 1 whose score reaches
+ * `threshold` (groups of that many layers selected nearly the same clusters,
+ * so one leader can serve them), else 1 (no sharing).  Host only; returns
+ * MPC_ERR_INVALID_ARG for score NULL, n < 1 or a threshold outside [0, 1]. */
+MPC_API int mpc_choose_share_every(int32_t n, const float* score, float threshold);
+
 /* Rows of the summary pyramid for a cache of cap_tokens rows (the sum of the
  * level capacities above), or a negative MPC_ERR_* code. */
 MPC_API int64_t mpc_summary_rows(int32_t cap_tokens, int32_t cluster_size,

@@ -591,6 +591,32 @@ MPC_API int mpc_abi_version(void) { return MPC_ABI_VERSION; }
 
 MPC_API const char* mpc_last_error(void) { return g_err.c_str(); }
 
+MPC_API int mpc_layer_refs(int32_t n_layers, int32_t share_every, mpc_layer_ref* out_refs) {
+  if (out_refs == nullptr) return fail(MPC_ERR_INVALID_ARG, "out_refs is NULL");
+  if (n_layers < 1 || n_layers > kMaxRefs) return fail(MPC_ERR_INVALID_ARG, "n_layers %d not in [1, %d]", n_layers, kMaxRefs);
+  if (share_every < 1) return fail(MPC_ERR_INVALID_ARG, "share_every %d < 1", share_every);
+  int groups = 0;
+  for (int l = 0; l < n_layers; ++l) {
+    // the first two layers lead themselves; later layers form groups of share_every
+    const int lead = (share_every == 1 || l < 2) ? l : 2 + share_every * ((l - 2) / share_every);
+    if (lead == l) ++groups;
+    out_refs[l].layer = l;
+    out_refs[l].group = groups - 1;
+    out_refs[l].leader = lead == l ? 1 : 0;
+  }
+  return groups;
+}
+
+MPC_API int mpc_choose_share_every(int32_t n, const float* score, float threshold) {
+  if (score == nullptr) return fail(MPC_ERR_INVALID_ARG, "score is NULL");
+  if (n < 1) return fail(MPC_ERR_INVALID_ARG, "n %d < 1", n);
+  if (!(threshold >= 0.f && threshold <= 1.f)) return fail(MPC_ERR_INVALID_ARG, "threshold %g not in [0, 1]", threshold);
+  int best = 1;
+  for (int m = 1; m <= n; ++m)
+    if (score[m - 1] >= threshold && m + 1 > best) best = m + 1;
+  return best;
+}
+
 MPC_API int64_t mpc_summary_rows(int32_t cap_tokens, int32_t cluster_size, int32_t n_levels, const int32_t* fanout) {
   Pyramid p;
   int32_t none[kMaxLevels] = {0, 0, 0, 0};

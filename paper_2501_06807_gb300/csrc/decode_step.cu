@@ -177,8 +177,10 @@ __global__ void __launch_bounds__(WPC * 32, 1) decode_step_kernel(const __grid_c
     // the last CTA to get here (every CTA has read the token counts and the
     // call counter) advances both for the next call; a sequence whose append
     // was refused keeps its count
+    // (acquire-release: this CTA's reads above happen before the add, and
+    // the last CTA's writes below after every other CTA's add)
     int last = 0;
-    if (lane == 0) last = atomicAdd(&sp.ctl[kCtlStarted], 1) == (int)gridDim.x - 1;
+    if (lane == 0) last = atom_add_acq_rel(&sp.ctl[kCtlStarted], 1) == (int)gridDim.x - 1;
     if (__shfl_sync(0xffffffffu, last, 0)) {
       if (p.advance)
         for (int b = lane; b < B; b += 32) {

@@ -119,7 +119,7 @@ ENTRY_POINTS = ("mpc_static_evict_workspace_size", "mpc_build_clusters_workspace
                 "mpc_static_evict", "mpc_build_clusters", "mpc_select", "mpc_sparse_decode_attn",
                 "mpc_summary_rows", "mpc_last_error", "mpc_device_status", "mpc_abi_version",
                 "mpc_sparse_decode_attn_static_scratch", "mpc_commonality", "mpc_selftest_wait",
-                "mpc_decode_step_workspace_size", "mpc_decode_step")
+                "mpc_decode_step_workspace_size", "mpc_decode_step", "mpc_layer_refs", "mpc_choose_share_every")
 
 _LIB = None
 
@@ -159,6 +159,10 @@ def load(path: Optional[str] = None) -> C.CDLL:
     lib.mpc_commonality.argtypes = [C.c_void_p, C.c_void_p]
     lib.mpc_selftest_wait.restype = C.c_int
     lib.mpc_selftest_wait.argtypes = [C.c_int32, C.c_int32, C.c_void_p, C.c_void_p]
+    lib.mpc_layer_refs.restype = C.c_int
+    lib.mpc_layer_refs.argtypes = [C.c_int32, C.c_int32, C.c_void_p]
+    lib.mpc_choose_share_every.restype = C.c_int
+    lib.mpc_choose_share_every.argtypes = [C.c_int32, C.POINTER(C.c_float), C.c_float]
     if lib.mpc_abi_version() != ABI_VERSION:
         raise MPCError(MPC_ERR_INVALID_ARG,
                        f"libmpcache ABI {lib.mpc_abi_version()} does not match the binding's {ABI_VERSION}")
@@ -256,12 +260,22 @@ def window_rows_bound(t_max: int, window_ppm: int, long_ppm: int, threshold: int
     return max(a, b)
 
 
+def layer_refs(n_layers: int, share_every: int):
+    """mpc_layer_refs: [(layer, group, is_leader)] for layers 0 .. n_layers - 1
+    under cross-layer index sharing with groups of ``share_every``."""
+    arr = (LayerRef * n_layers)()
+    g = load().mpc_layer_refs(n_layers, max(1, share_every), arr)
+    _check(min(g, 0))
+    return [(r.layer, r.group, bool(r.leader)) for r in arr]
+
+
 def sharing_leader(layer: int, share_every: int) -> int:
-    """Leader layer of ``layer`` under cross-layer index sharing: layers 0 and 1
-    lead themselves, later layers form groups of ``share_every``."""
-    if share_every <= 1 or layer < 2:
-        return layer
-    return 2 + share_every * ((layer - 2) // share_every)
+    """Leader layer of ``layer`` under cross-layer index sharing (from
+    mpc_layer_refs: layers 0 and 1 lead themselves, later layers form groups
+    of ``share_every``)."""
+    refs = layer_refs(layer + 1, share_every)
+    group = refs[layer][1]
+    return next(l for l, g, leads in refs if leads and g == group)
 
 
 def commonality(sel: torch.Tensor, k: int, m: int, n_clusters: int):
@@ -286,15 +300,17 @@ def commonality(sel: torch.Tensor, k: int, m: int, n_clusters: int):
 
 
 def choose_share_every(scores: dict, threshold: float) -> int:
-    """Adaptive sharing-group size: the largest m whose commonality score of
-    m + 1 adjacent layers (``scores[m]``, e.g. the mean over sequences and kv
-    heads) reaches ``threshold`` -- groups of m + 1 layers then select nearly
-    the same clusters, so one leader can serve them -- else 1 (no sharing)."""
-    best = 1
-    for m in sorted(scores):
-        if scores[m] >= threshold:
-            best = max(best, m + 1)
-    return best
+    """mpc_choose_share_every: the adaptive sharing-group size, the largest
+    m + 1 whose commonality score of m + 1 adjacent layers (``scores[m]``, e.g.
+    the mean over sequences and kv heads, for m = 1 .. n) reaches
+    ``threshold``, else 1 (no sharing)."""
+    n = max(scores) if scores else 0
+    if n < 1:
+        return 1
+    arr = (C.c_float * n)(*[float(scores.get(m, -1.0)) for m in range(1, n + 1)])
+    r = load().mpc_choose_share_every(n, arr, float(threshold))
+    _check(min(r, 0))
+    return r
 
 
 def summary_rows(cap_tokens: int, s: int, fanouts: Sequence[int]) -> int:
@@ -346,7 +362,9 @@ class Engine:
         self.alpha, self.scale = alpha, scale
         self.window_ppm, self.long_window_ppm, self.long_threshold = window_ppm, long_window_ppm, long_prompt_threshold
         self.layers = list(range(n_layers)) if layers is None else list(layers)
-        lead = [sharing_leader(l, share_every) for l in range(n_layers)]
+        full = layer_refs(n_layers, share_every)  # (layer, group, leads) from mpc_layer_refs
+        lead_of_group = {g: l for l, g, leads in full if leads}
+        lead = [lead_of_group[g] for _, g, _ in full]
         self.leaders = sorted(set(lead[l] for l in self.layers))
         self.group_of = {l: self.leaders.index(lead[l]) for l in self.layers}
         self.refs_all = [(l, self.group_of[l], lead[l] == l) for l in self.layers]
@@ -378,6 +396,19 @@ class Engine:
         self.n_sel = torch.zeros((B,), **i32)
         self.out = torch.zeros((n_layers, B, n_q_heads, d), **f32)
         self._ws = {}
+
+    def check_status(self) -> int:
+        """Synchronizes, then reads and clears the device status word (see
+        ``device_status``).  A bounded wait that gave up (flag 1) can leave the
+        split-merge counters of a decode workspace nonzero, and the calls
+        require a zero-filled workspace again after that, so this engine's
+        workspaces are cleared before the flags are returned."""
+        st = device_status()
+        if st & 1:
+            for ws in self._ws.values():
+                ws.zero_()
+            torch.cuda.synchronize()
+        return st
 
     # --------------------------------------------------------- prefill ----
     @staticmethod

@@ -1,6 +1,9 @@
 """Shared helpers of the test-suite (no method arithmetic of their own)."""
 from __future__ import annotations
 
+import json
+import os
+
 import numpy as np
 import torch
 
@@ -104,3 +107,21 @@ def unswizzle(cache_rows: torch.Tensor) -> torch.Tensor:
     x = cache_rows.reshape(*cache_rows.shape[:-1], n_ch, E)
     idx = src.to(cache_rows.device).view(*([1] * (x.dim() - 3)), rows, n_ch, 1).expand_as(x)
     return torch.gather(x, -2, idx).reshape(cache_rows.shape)
+
+
+def log_parity(test: str, **fields):
+    """Reports one parity record (measured errors, the bands they are held to,
+    counts of tie swaps and skipped units): printed (shown with ``pytest -rP``
+    or ``-s``) and, when the environment variable MPC_PARITY_LOG names a file,
+    appended to it as a JSON line."""
+    rec = {"test": test}
+    for k, v in fields.items():
+        if isinstance(v, (np.floating, np.integer)):
+            v = v.item()
+        rec[k] = v
+    line = json.dumps(rec)
+    print("parity", line)
+    path = os.environ.get("MPC_PARITY_LOG")
+    if path:
+        with open(path, "a") as f:
+            f.write(line + "\n")

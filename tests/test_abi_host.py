@@ -10,6 +10,7 @@ import subprocess
 import pytest
 import torch
 
+from oracle import mpcache_oracle as O
 from paper_2501_06807_gb300 import build, mpcache
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
@@ -319,3 +320,45 @@ def test_decode_step_validation(lib):
     a.attn.rep = a.attn.r_max = a.attn.r_min = 16384
     assert lib.mpc_decode_step(C.byref(a), None, 0, None) == mpcache.MPC_ERR_WORKSPACE
     assert lib.mpc_decode_step(None, None, 0, None) == mpcache.MPC_ERR_INVALID_ARG
+
+
+def test_layer_refs_follow_the_sharing_rule(lib):
+    """mpc_layer_refs (Sec. 3.4): the first two layers lead themselves, later
+    layers reuse the first layer of their group of share_every; leaders are
+    the oracle's (leader_of, pinned by hand values), groups are numbered in
+    layer order."""
+    for L in (1, 2, 3, 6, 32, 33, 128):
+        for m in (1, 2, 3, 4, 7):
+            arr = (mpcache.LayerRef * L)()
+            g = lib.mpc_layer_refs(L, m, arr)
+            leaders = sorted({O.leader_of(l, m) for l in range(L)})
+            assert g == len(leaders)
+            for l in range(L):
+                lead = O.leader_of(l, m)
+                assert arr[l].layer == l
+                assert arr[l].group == leaders.index(lead)
+                assert arr[l].leader == (1 if lead == l else 0)
+    # the 32-layer workloads: groups of two (17 leaders) and of four (10 leaders)
+    assert lib.mpc_layer_refs(32, 2, (mpcache.LayerRef * 32)()) == 17
+    assert lib.mpc_layer_refs(32, 4, (mpcache.LayerRef * 32)()) == 10
+    bad = (mpcache.LayerRef * 4)()
+    assert lib.mpc_layer_refs(0, 2, bad) == mpcache.MPC_ERR_INVALID_ARG
+    assert lib.mpc_layer_refs(4, 0, bad) == mpcache.MPC_ERR_INVALID_ARG
+    assert lib.mpc_layer_refs(129, 2, (mpcache.LayerRef * 129)()) == mpcache.MPC_ERR_INVALID_ARG
+    assert lib.mpc_layer_refs(4, 2, None) == mpcache.MPC_ERR_INVALID_ARG
+
+
+def test_choose_share_every(lib):
+    """mpc_choose_share_every: the largest window (m + 1 layers) whose
+    commonality reaches the threshold, else no sharing."""
+    def choose(scores, thr):
+        arr = (C.c_float * len(scores))(*scores)
+        return lib.mpc_choose_share_every(len(scores), arr, thr)
+    assert choose([0.9, 0.7, 0.5], 0.6) == 3
+    assert choose([0.9, 0.7, 0.5], 0.5) == 4
+    assert choose([0.4, 0.3, 0.2], 0.5) == 1
+    assert choose([0.4, 0.8, 0.2], 0.5) == 3   # a later window may reach it alone
+    assert choose([1.0], 1.0) == 2
+    assert mpcache.choose_share_every({1: 0.9, 2: 0.7, 3: 0.5}, 0.6) == 3
+    assert choose([0.5], 1.5) == mpcache.MPC_ERR_INVALID_ARG
+    assert lib.mpc_choose_share_every(0, (C.c_float * 1)(0.5), 0.5) == mpcache.MPC_ERR_INVALID_ARG
