@@ -226,7 +226,7 @@ def test_commonality_validation(lib):
     assert lib.mpc_commonality(C.byref(a), None) == mpcache.MPC_ERR_INVALID_ARG
 
 
-def test_choose_share_every():
+def test_choose_share_every_binding():
     assert mpcache.choose_share_every({1: 0.95, 2: 0.9, 3: 0.6}, 0.85) == 3   # groups of 3 layers
     assert mpcache.choose_share_every({1: 0.5}, 0.85) == 1                     # no sharing
 
