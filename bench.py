@@ -51,6 +51,26 @@ def parse_args():
     p.add_argument("--workload", default=synth.C5.name, choices=sorted(synth.WORKLOADS))
     p.add_argument("--decode-steps", type=int, default=None)
     p.add_argument("--no-e2e", action="store_true")
+    # the paper's ablation axes, applied to --workload (the line's config
+    # reports them): alpha of Eq. 3, the window ratios of static eviction,
+    # the static budget, the cluster size, the hierarchy (fanouts and kept
+    # ratio per level, finest first), the sharing group size, and the
+    # cross-layer correlation of the synthetic inputs
+    p.add_argument("--alpha", type=float)
+    p.add_argument("--window-ppm", type=int)
+    p.add_argument("--long-window-ppm", type=int)
+    p.add_argument("--keep-ppm", type=int)
+    p.add_argument("--cluster-size", type=int)
+    p.add_argument("--fanouts", help="comma-separated children per coarser cluster ('' for one level)")
+    p.add_argument("--level-keep-ppm", help="comma-separated kept ppm per level, finest first")
+    p.add_argument("--share-every", type=int)
+    p.add_argument("--layer-rho-ppm", type=int)
+    # measured side reports instead of the bench line (one JSON line each):
+    # adaptive-sharing: commonality of unshared selections, the group size the
+    # adaptive rule picks, and the decode step with it; tokenwise: selection
+    # and decode step of the clustered path and of the token-wise comparator
+    p.add_argument("--report", choices=["adaptive-sharing", "tokenwise"])
+    p.add_argument("--share-threshold", type=float, default=0.25)
     # internal: print the oracle sample of --workload as JSON (the bench runs
     # it in a child process with one BLAS thread for the single-core figure)
     p.add_argument("--oracle-sample", action="store_true", help=argparse.SUPPRESS)
@@ -67,6 +87,47 @@ def peaks():
 
 
 # ------------------------------------------------------------ workload ----
+
+def _ints(text):
+    return tuple(int(v) for v in text.split(",") if v.strip())
+
+
+# (flag, Workload field, parser)
+OVERRIDES = (("--alpha", "alpha", float), ("--window-ppm", "window_ppm", int),
+             ("--long-window-ppm", "long_window_ppm", int), ("--keep-ppm", "keep_ppm", int),
+             ("--cluster-size", "cluster_size", int), ("--fanouts", "fanouts", _ints),
+             ("--level-keep-ppm", "level_keep_ppm", _ints), ("--share-every", "share_every", int),
+             ("--layer-rho-ppm", "layer_rho_ppm", int))
+
+
+def _attr(flag):
+    return flag[2:].replace("-", "_")
+
+
+def overrides_of(args):
+    """{field: value} of the ablation flags given on the command line."""
+    return {field: parse(getattr(args, _attr(flag))) if parse is _ints else getattr(args, _attr(flag))
+            for flag, field, parse in OVERRIDES if getattr(args, _attr(flag)) is not None}
+
+
+def override_argv(args):
+    """The ablation flags as given, to pass on to a child process."""
+    return [a for flag, _, _ in OVERRIDES if getattr(args, _attr(flag)) is not None
+            for a in (flag, str(getattr(args, _attr(flag))))]
+
+
+def workload_of(args):
+    """--workload with the ablation flags applied."""
+    w = synth.WORKLOADS[args.workload]
+    ov = overrides_of(args)
+    if not ov:
+        return w
+    w = w.replace(**ov)
+    if len(w.level_keep_ppm) != w.n_levels:
+        raise SystemExit(f"--level-keep-ppm needs {w.n_levels} ratios (one per level, finest first)")
+    if w.cluster_size < 1 or w.share_every < 1 or not 0 <= w.alpha <= 1:
+        raise SystemExit("cluster size and share_every must be >= 1 and alpha in [0, 1]")
+    return w
 
 def rules(w):
     from paper_2501_06807_gb300 import mpcache
@@ -179,25 +240,30 @@ class ClockSampler:
 
 # ------------------------------------------------------------ our arm ----
 
+def make_engine(w, E):
+    from paper_2501_06807_gb300 import mpcache
+    dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+    return mpcache.Engine(n_layers=w.n_layers, batch=w.batch, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads,
+                          head_dim=w.head_dim, dtype=dt, t_max=w.prompt_len, keep_ppm=w.keep_ppm,
+                          cluster_size=w.cluster_size, fanouts=w.fanouts, level_keep_ppm=w.level_keep_ppm,
+                          share_every=w.share_every, max_decode_steps=E, alpha=w.alpha,
+                          window_ppm=w.window_ppm, long_window_ppm=w.long_window_ppm,
+                          long_prompt_threshold=w.long_prompt_threshold)
+
+
 def run_ours(args, rank, world, dist):
     from paper_2501_06807_gb300 import build, mpcache
     build.build()
     mpcache.load()
     dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
     torch.cuda.set_device(dev)
-    w = replica_workload(synth.WORKLOADS[args.workload], rank)
+    w = replica_workload(workload_of(args), rank)
     E = args.decode_steps or w.decode_steps
     R, leaders = rules(w)
     x = synth.generate(w, R, device="cuda", decode_steps=E)
     lens = x.prompt_lens.cuda()
     pt = x.page_table.cuda() if x.page_table is not None else None
-    dt = torch.bfloat16 if w.dtype == "bf16" else torch.float32
-    eng = mpcache.Engine(n_layers=w.n_layers, batch=w.batch, n_q_heads=w.n_q_heads, n_kv_heads=w.n_kv_heads,
-                         head_dim=w.head_dim, dtype=dt, t_max=w.prompt_len, keep_ppm=w.keep_ppm,
-                         cluster_size=w.cluster_size, fanouts=w.fanouts, level_keep_ppm=w.level_keep_ppm,
-                         share_every=w.share_every, max_decode_steps=E, alpha=w.alpha,
-                         window_ppm=w.window_ppm, long_window_ppm=w.long_window_ppm,
-                         long_prompt_threshold=w.long_prompt_threshold)
+    eng = make_engine(w, E)
     out_all = torch.empty((E, w.n_layers, w.batch, w.n_q_heads, w.head_dim), dtype=torch.float32, device=dev)
 
     def prefill():
@@ -440,6 +506,121 @@ def run_ours(args, rank, world, dist):
     return line
 
 
+# ------------------------------------------------------------ reports ----
+
+def decode_timing(w, E, reps=5, calibrate=None):
+    """Graph-timed decode of ``w`` after its prefill: the median over ``reps``
+    replays of E whole decode steps (mpc_decode_step, every layer) and of E
+    standalone selections of the leaders (mpc_select at the prefill's cache).
+    ``calibrate(eng, x)`` runs on the prefilled engine before the timing."""
+    from paper_2501_06807_gb300 import mpcache
+    R, leaders = rules(w)
+    x = synth.generate(w, R, device="cuda", decode_steps=E)
+    lens = x.prompt_lens.cuda()
+    pt = x.page_table.cuda() if x.page_table is not None else None
+    eng = make_engine(w, E)
+
+    def prefill():
+        eng.prefill(x.k, x.v, x.q_win, lens, pt, w.page_size)
+
+    extra = {}
+    if calibrate is not None:
+        prefill()
+        extra = calibrate(eng, x)
+    # attended rows per step (selected clusters + tail), eager pass
+    prefill()
+    n_keep = eng.n_keep.cpu().tolist()
+    attended = 0
+    for e in range(E):
+        eng.decode_step(x.q[e], x.k_new[e], x.v_new[e])
+        n_sel = eng.n_sel.cpu().tolist()
+        attended += sum((n_sel[b] * w.cluster_size + (n_keep[b] + e) % w.cluster_size + 1)
+                        for b in range(w.batch)) * w.n_layers * w.n_kv_heads
+    if mpcache.device_status() != 0:
+        raise RuntimeError("device status set by the eager pass")
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    stream = torch.cuda.current_stream()
+
+    def timed(body):
+        prefill()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            body()
+        out = []
+        for i in range(reps + 2):
+            prefill()
+            a, b = ev(), ev()
+            a.record(stream)
+            g.replay()
+            b.record(stream)
+            torch.cuda.synchronize()
+            if i >= 2:
+                out.append(a.elapsed_time(b) * 1e3 / E)
+        return statistics.median(out)
+
+    step_us = timed(lambda: [eng.decode_step(x.q[e], x.k_new[e], x.v_new[e]) for e in range(E)])
+    sel_us = timed(lambda: [eng.select(x.q[e]) for e in range(E)])
+    res = {"decode_step_us": round(step_us, 2), "select_us": round(sel_us, 2), "leaders": len(leaders),
+           "attended_rows_per_step": attended / E,
+           "scored_rep_rows_per_step": sum(select_rows(w, n_keep[b]) for b in range(w.batch)) * len(leaders) *
+           w.n_kv_heads, **extra}
+    del eng, x
+    torch.cuda.empty_cache()
+    return res
+
+
+def run_report(args):
+    from paper_2501_06807_gb300 import build, mpcache
+    build.build()
+    mpcache.load()
+    torch.cuda.set_device(0)
+    if args.report == "tokenwise":
+        # the clustered method and the token-wise comparator (every prompt
+        # token kept, one token per cluster) on the same shapes and inputs
+        for clustered, tokenwise in ((synth.C3, synth.C3_TOKENWISE), (synth.C5, synth.C5_TOKENWISE)):
+            for w in (clustered, tokenwise):
+                E = args.decode_steps or w.decode_steps
+                r = decode_timing(w, E)
+                print(json.dumps({"report": "tokenwise", "workload": w.name, "decode_steps": E,
+                                  "cluster_size": w.cluster_size, "keep_ppm": w.keep_ppm,
+                                  "fanouts": list(w.fanouts), "level_keep_ppm": list(w.level_keep_ppm), **r}),
+                      flush=True)
+        return
+    # adaptive-sharing: each layer its own leader for a few calibration steps,
+    # the commonality of their selected tokens (windows of 2 .. 4 layers), the
+    # group size the adaptive rule picks at --share-threshold, then the
+    # decode step with no sharing, the picked group size and the workload's
+    ms = (1, 2, 3)
+    for base in (synth.C2, synth.C3, synth.C5):
+        for rho in (0, 950_000):
+            w1 = base.replace(share_every=1, layer_rho_ppm=rho)
+            E = args.decode_steps or base.decode_steps
+            n_cal = min(4, E)
+
+            def calibrate(eng, x):
+                acc = {m: [] for m in ms}
+                for e in range(n_cal):
+                    eng.decode_step(x.q[e], x.k_new[e], x.v_new[e])
+                    for m in ms:
+                        acc[m].append(float(eng.commonality(m)[1].mean()))
+                return {"commonality": {m + 1: round(statistics.mean(v), 4) for m, v in acc.items()}}
+
+            r1 = decode_timing(w1, E, calibrate=calibrate)
+            com = {m: r1["commonality"][m + 1] for m in ms}
+            chosen = mpcache.choose_share_every(com, args.share_threshold)
+            timings = {1: r1}
+            for se in sorted({chosen, base.share_every} - {1}):
+                timings[se] = decode_timing(base.replace(share_every=se, layer_rho_ppm=rho), E)
+            print(json.dumps({"report": "adaptive-sharing", "workload": base.name, "layer_rho_ppm": rho,
+                              "calibration_steps": n_cal, "commonality_by_layers": r1["commonality"],
+                              "threshold": args.share_threshold, "chosen_share_every": chosen,
+                              "fixed_share_every": base.share_every, "decode_steps": E,
+                              "decode_step_us": {se: r["decode_step_us"] for se, r in timings.items()},
+                              "select_us": {se: r["select_us"] for se, r in timings.items()},
+                              "leaders": {se: r["leaders"] for se, r in timings.items()}}), flush=True)
+
+
 # ------------------------------------------------------ oracle sample ----
 
 def oracle_sample(w, E_sample=4):
@@ -502,14 +683,15 @@ def oracle_sample(w, E_sample=4):
             "sample": sample, "seconds": t1 - t0 + t_build + t_dec, "whole_job_s_estimate": whole}
 
 
-def cpu_baseline(workload):
+def cpu_baseline(args):
     """The oracle sample on all host cores (numpy's BLAS threads), and again
     in a child process limited to one thread, each with its core count."""
-    allc = oracle_sample(synth.WORKLOADS[workload])
+    allc = oracle_sample(workload_of(args))
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                BLIS_NUM_THREADS="1", VECLIB_MAXIMUM_THREADS="1", NUMEXPR_NUM_THREADS="1")
     try:
-        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-sample", "--workload", workload],
+        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-sample", "--workload", args.workload,
+                            *override_argv(args)],
                            env=env, capture_output=True, text=True, timeout=600)
         one = json.loads(r.stdout.strip().splitlines()[-1])
         allc["single_thread"] = {"value": one["value"], "unit": one["unit"], "cores": 1,
@@ -526,14 +708,16 @@ def workload_config(w, E, parallelism):
             "kv_heads": w.n_kv_heads, "head_dim": w.head_dim, "prompt_len": w.prompt_len,
             "decode_steps": E, "cluster_size": w.cluster_size, "fanouts": list(w.fanouts),
             "level_keep_ppm": list(w.level_keep_ppm), "keep_ppm": w.keep_ppm,
-            "share_every": w.share_every, "paged": w.paged, "parallelism": parallelism,
+            "share_every": w.share_every, "alpha": w.alpha, "window_ppm": w.window_ppm,
+            "long_window_ppm": w.long_window_ppm, "layer_rho_ppm": w.layer_rho_ppm,
+            "paged": w.paged, "parallelism": parallelism,
             "l2": "inputs larger than L2 (prompt KV up to %.1f GB per step)" % kv_gb}
 
 
 def run_reference(args, rank, world):
     if rank != 0:
         return None
-    w = synth.WORKLOADS[args.workload]
+    w = workload_of(args)
     for _ in range(args.warmup):
         oracle_sample(w, E_sample=1)
     vals, secs, whole = [], [], []
@@ -569,14 +753,18 @@ def main():
         tdist.init_process_group(backend)
         dist = tdist
     if args.oracle_sample:
-        print(json.dumps(oracle_sample(synth.WORKLOADS[args.workload])), flush=True)
+        print(json.dumps(oracle_sample(workload_of(args))), flush=True)
+        return
+    if args.report:
+        if rank == 0 and world == 1:
+            run_report(args)
         return
     if args.impl == "reference":
         line = run_reference(args, rank, world)
     else:
         line = run_ours(args, rank, world, dist)
         if rank == 0 and world == 1:
-            line["cpu_baseline"] = cpu_baseline(args.workload)
+            line["cpu_baseline"] = cpu_baseline(args)
     if rank == 0 and line is not None:
         print(json.dumps(line), flush=True)
     if dist is not None:

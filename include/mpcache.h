@@ -70,7 +70,7 @@ extern "C" {
 
 #define MPC_API __attribute__((visibility("default")))
 
-#define MPC_ABI_VERSION 6
+#define MPC_ABI_VERSION 7
 #define MPC_MAX_LEVELS 4
 #define MPC_MAX_REFS 128
 
@@ -375,7 +375,17 @@ MPC_API int mpc_sparse_decode_attn_static_scratch(const mpc_attn_args* args, voi
  *   out_score[b][h] = out_total[b][h] / (k (n_layers - m))
  * 1 means the layers selected the same clusters.  sel entries are cluster ids
  * < n_clusters or -1 (padding, ignored); an id >= n_clusters sets status bit 4.
- * Read-only on sel; asynchronous on stream. */
+ *
+ * Token positions (kept != NULL).  Layers that lead their own groups also ran
+ * their own static eviction, so one cluster id names different tokens in
+ * different layers.  With kept set, every selected cluster c stands for the
+ * positions of its cluster_size cache rows r = c s .. c s + s - 1: kept[r]
+ * for a kept prompt row (r < n_keep[b]), prompt_len[b] + r - n_keep[b] for a
+ * row appended while decoding; the sets S_l are then these k s positions, the
+ * score divides by k s (n_layers - m), and n_clusters bounds the positions
+ * instead (every position < n_clusters; a larger one, or a kept row r >=
+ * kept_cap, sets status bit 4 and is skipped).
+ * Read-only on its inputs; asynchronous on stream. */
 typedef struct {
   uint32_t struct_size;        /* sizeof(mpc_commonality_args) */
   int32_t n_layers;            /* >= 2 */
@@ -388,6 +398,13 @@ typedef struct {
   int32_t m;                   /* windows of m + 1 layers, 1 .. n_layers - 1 */
   int32_t* out_total;          /* device [batch][n_kv_heads] */
   float* out_score;            /* device [batch][n_kv_heads] */
+  /* optional: compare token positions instead of cluster ids */
+  const int32_t* kept;         /* NULL, or device [n_layers][batch][n_kv_heads][kept_cap]: each layer's kept positions */
+  int64_t kept_layer_stride;   /* elements between layers of kept */
+  int32_t kept_cap;
+  int32_t cluster_size;        /* s (>= 1 when kept is set) */
+  const int32_t* n_keep;       /* device [batch], kept prompt rows (required with kept) */
+  const int32_t* prompt_len;   /* device [batch], prompt lengths (required with kept) */
 } mpc_commonality_args;
 
 MPC_API int mpc_commonality(const mpc_commonality_args* args, void* stream);

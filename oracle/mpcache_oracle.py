@@ -352,6 +352,20 @@ def commonality(indices: Sequence[Sequence[int]], k: int, m: int) -> float:
     return total / (k * (L - m))
 
 
+def selected_positions(kept: Sequence[int], prompt_len: int, selected: Sequence[int], s: int) -> List[int]:
+    """Token positions of the selected clusters (the idx sets of the
+    commonality score, Sec. 2 Observation 3, for a layer with its own static
+    eviction): cluster c holds cache rows c s .. c s + s - 1; a row r below
+    len(kept) is the kept prompt token kept[r], a later row is the token
+    appended at position prompt_len + r - len(kept) (App. A decode append)."""
+    n_keep = len(kept)
+    out = []
+    for c in selected:
+        for r in range(int(c) * s, int(c) * s + s):
+            out.append(int(kept[r]) if r < n_keep else prompt_len + r - n_keep)
+    return sorted(out)
+
+
 # ------------------------------------------------------- full pipeline ----
 
 @dataclass

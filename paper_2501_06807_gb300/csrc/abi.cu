@@ -6,9 +6,17 @@
 #include <cstring>
 #include <string>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "kernels.cuh"
 
 namespace mpc {
+
+// NVTX range over one ABI call (a host-side marker for profilers and
+// tracers; without an attached tool the push and pop return at once)
+NvtxRange::NvtxRange(const char* name) { nvtxRangePushA(name); }
+NvtxRange::~NvtxRange() { nvtxRangePop(); }
+
 namespace {
 
 thread_local std::string g_err;
@@ -670,6 +678,7 @@ MPC_API int mpc_static_evict_workspace_size(const mpc_static_args* args, size_t*
 }
 
 MPC_API int mpc_static_evict(const mpc_static_args* args, void* workspace, size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx("mpc_static_evict");
   StaticParams p;
   MPC_TRY(validate_static(args, &p));
   if (!args->q_win || !args->k.data || !args->prompt_lens || !args->out_scores || !args->out_kept || !args->out_n_keep)
@@ -703,6 +712,7 @@ MPC_API int mpc_build_clusters_workspace_size(const mpc_cluster_args* args, size
 }
 
 MPC_API int mpc_build_clusters(const mpc_cluster_args* args, void* workspace, size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx("mpc_build_clusters");
   (void)workspace;
   (void)workspace_bytes;
   ClusterParams p;
@@ -731,6 +741,7 @@ MPC_API int mpc_select_workspace_size(const mpc_select_args* args, size_t* bytes
 }
 
 MPC_API int mpc_select(const mpc_select_args* args, void* workspace, size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx("mpc_select");
   (void)workspace;
   (void)workspace_bytes;
   SelectParams p;
@@ -756,6 +767,7 @@ MPC_API int mpc_sparse_decode_attn_workspace_size(const mpc_attn_args* args, siz
 }
 
 MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace, size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx("mpc_sparse_decode_attn");
   AttnParams p;
   AttnPlan plan;
   MPC_TRY(validate_attn(args, &p, &plan));
@@ -797,6 +809,7 @@ MPC_API int mpc_decode_step_workspace_size(const mpc_decode_args* args, size_t* 
 }
 
 MPC_API int mpc_decode_step(const mpc_decode_args* args, void* workspace, size_t workspace_bytes, void* stream) {
+  NvtxRange nvtx("mpc_decode_step");
   StepParams sp;
   SelectParams sel;
   StepPlan plan;

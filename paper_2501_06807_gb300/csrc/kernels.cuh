@@ -7,6 +7,14 @@
 
 namespace mpc {
 
+// RAII NVTX range: one named range over each ABI call
+struct NvtxRange {
+  explicit NvtxRange(const char* name);
+  ~NvtxRange();
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
 struct AttnParams {
   RefTable refs;
   int n_refs, B, Hq, Hkv, G;

@@ -36,6 +36,7 @@ int scratch_address(void** out) {
 }  // namespace mpc
 
 extern "C" MPC_API int mpc_sparse_decode_attn_static_scratch(const mpc_attn_args* args, void* stream) {
+  mpc::NvtxRange nvtx("mpc_sparse_decode_attn_static_scratch");
   using namespace mpc;
   size_t need = 0;
   int rc = mpc_sparse_decode_attn_workspace_size(args, &need);

@@ -28,7 +28,7 @@ MPC_F32, MPC_BF16 = 0, 1
 MPC_SIM_EQ3, MPC_SIM_BOUND, MPC_SIM_MEAN, MPC_SIM_FXP = 0, 1, 2, 3
 FXP_FRAC_BITS = 18
 MAX_LEVELS = 4
-ABI_VERSION = 6
+ABI_VERSION = 7
 MAX_REFS = 128
 PPM = 1_000_000
 
@@ -88,7 +88,9 @@ class CommonalityArgs(C.Structure):
     _fields_ = [("struct_size", C.c_uint32), ("n_layers", C.c_int32), ("batch", C.c_int32),
                 ("n_kv_heads", C.c_int32), ("sel", C.c_void_p), ("sel_layer_stride", C.c_int64),
                 ("sel_cap", C.c_int32), ("n_clusters", C.c_int32), ("k", C.c_int32), ("m", C.c_int32),
-                ("out_total", C.c_void_p), ("out_score", C.c_void_p)]
+                ("out_total", C.c_void_p), ("out_score", C.c_void_p), ("kept", C.c_void_p),
+                ("kept_layer_stride", C.c_int64), ("kept_cap", C.c_int32), ("cluster_size", C.c_int32),
+                ("n_keep", C.c_void_p), ("prompt_len", C.c_void_p)]
 
 
 class AttnArgs(C.Structure):
@@ -278,13 +280,19 @@ def sharing_leader(layer: int, share_every: int) -> int:
     return next(l for l, g, leads in refs if leads and g == group)
 
 
-def commonality(sel: torch.Tensor, k: int, m: int, n_clusters: int):
+def commonality(sel: torch.Tensor, k: int, m: int, n_clusters: int, kept: Optional[torch.Tensor] = None,
+                cluster_size: int = 1, n_keep: Optional[torch.Tensor] = None,
+                prompt_len: Optional[torch.Tensor] = None):
     """Commonality of per-layer selections (Sec. 2, Observation 3; mpc_commonality).
 
     sel: int32 [L][B][Hkv][sel_cap] selections of consecutive layers, each its
     own leader (ids ascending, -1 padded).  Returns (total, score), each
     [B][Hkv]: total = sum over l < L - m of |S_l n ... n S_{l+m}| over the
-    first k ids of each list, score = total / (k (L - m)).
+    first k ids of each list, score = total / (k (L - m)).  With ``kept``
+    (int32 [L][B][Hkv][kept_cap], each layer's kept positions) the sets are
+    the token positions of the selected clusters' rows (``n_keep`` and
+    ``prompt_len``, int32 [B], place the rows appended while decoding), the
+    score divides by k s (L - m), and ``n_clusters`` bounds the positions.
     """
     L, B, Hkv, cap = sel.shape
     total = torch.zeros((B, Hkv), dtype=torch.int32, device=sel.device)
@@ -295,6 +303,12 @@ def commonality(sel: torch.Tensor, k: int, m: int, n_clusters: int):
     a.sel, a.sel_layer_stride, a.sel_cap = _ptr(sel), sel.stride(0), cap
     a.n_clusters, a.k, a.m = n_clusters, k, m
     a.out_total, a.out_score = _ptr(total), _ptr(score)
+    if kept is not None:
+        _check_input(kept, "kept", torch.int32, (L, B, Hkv, None))
+        _check_input(n_keep, "n_keep", torch.int32, (B,))
+        _check_input(prompt_len, "prompt_len", torch.int32, (B,))
+        a.kept, a.kept_layer_stride, a.kept_cap = _ptr(kept), kept.stride(0), kept.shape[3]
+        a.cluster_size, a.n_keep, a.prompt_len = cluster_size, _ptr(n_keep), _ptr(prompt_len)
     _check(load().mpc_commonality(C.byref(a), C.c_void_p(_stream())))
     return total, score
 
@@ -395,6 +409,7 @@ class Engine:
         self.sel = torch.full((G, B, Hkv, self.sel_cap), -1, **i32)
         self.n_sel = torch.zeros((B,), **i32)
         self.out = torch.zeros((n_layers, B, n_q_heads, d), **f32)
+        self.prompt_lens = None  # the lens of the last static eviction (device int32 [B])
         self._ws = {}
 
     def check_status(self) -> int:
@@ -483,6 +498,7 @@ class Engine:
         _check(lib.mpc_static_evict_workspace_size(C.byref(a), C.byref(n)))
         ws = _ws_zero(n.value, self._ws, "static")
         _check(lib.mpc_static_evict(C.byref(a), C.c_void_p(_ptr(ws)), n.value, C.c_void_p(_stream())))
+        self.prompt_lens = lens
 
     def build_clusters(self, k, v, page_table=None, page_size=16, layers=None):
         """Gathering and clustering of every layer (of ``layers`` only, if
@@ -606,6 +622,25 @@ class Engine:
         _check(lib.mpc_decode_step_workspace_size(C.byref(a), C.byref(n)))
         ws = _ws_zero(n.value, self._ws, "step")
         _check(lib.mpc_decode_step(C.byref(a), C.c_void_p(_ptr(ws)), n.value, C.c_void_p(_stream())))
+
+    def commonality(self, m: int):
+        """Commonality score of windows of m + 1 adjacent layers over this
+        step's selections (the last select or decode step), compared as the
+        token positions of the selected clusters.  Every processed layer
+        must lead its own group (share_every = 1, consecutive layers).  The
+        sets hold the first k clusters of each list, k the fewest selected by
+        a sequence of the batch; returns (total, score), each [B][Hkv] on the
+        device."""
+        if self.n_groups != len(self.layers) or self.layers != list(range(self.layers[0], self.layers[-1] + 1)):
+            raise ValueError("commonality needs consecutive layers, each its own leader (share_every = 1)")
+        if self.prompt_lens is None:
+            raise ValueError("commonality needs the prefill's prompt lengths (run static_evict first)")
+        bound = self.t_max + self.cap_tokens  # every position: prompt rows and appended rows
+        k = int(self.n_sel.min())
+        if k < 1:
+            raise ValueError("commonality needs a selection of at least one cluster per sequence")
+        return commonality(self.sel, k, m, bound, kept=self.kept, cluster_size=self.s,
+                           n_keep=self.n_keep, prompt_len=self.prompt_lens)
 
     def decode_step_two_calls(self, q, k_new, v_new, out=None):
         """The same decode step as two calls: ``select`` (leaders), then

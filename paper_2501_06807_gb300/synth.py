@@ -20,6 +20,14 @@ seeded distributions described in ``Workload.rule``:
                q = 0.35 * k_j + 0.7 * u + 0.622 * n (the needle direction
                dominates, as a question about the planted passage would).
 
+``layer_rho_ppm`` = rho > 0 (``outlier`` and ``needle``) chains the layers of
+a sequence the way a residual stream would (Sec. 2, Observation 3): layer l's
+keys are rho K_{l-1} + sqrt(1 - rho^2) K_fresh (after the outlier scaling),
+slot i of its subset S keeps layer l-1's position with probability rho (else
+a fresh position), and the slot each window/decode query targets is drawn
+from one stream per sequence, shared by all layers.  rho = 0 (the default)
+draws every layer independently.
+
 Layouts (all row-major, head_dim innermost):
 
 * dense prompt K/V: ``[L][B][Hkv][T_max][d]``; positions >= T_b are zero.
@@ -75,6 +83,7 @@ class Workload:
     long_prompt_threshold: int = 24_576
     alpha: float = 0.6
     needle_len: int = 64
+    layer_rho_ppm: int = 0          # cross-layer correlation (0: independent layers)
 
     @property
     def group(self) -> int:
@@ -106,7 +115,16 @@ C5 = Workload("c5_llama3_8b_gqa_t32768_needles", 32, 1, 32, 8, 128, "bf16",
 C4_BATCHES = (1, 4, 16, 32)
 # the batched paged workload at its other batch sizes (same seed and rule)
 C4_VARIANTS = tuple(C4.replace(name=f"c4_llama2_7b_paged_b{b}", batch=b) for b in C4_BATCHES if b != C4.batch)
-WORKLOADS = {w.name: w for w in (C1, C2, C3, C4, C5) + C4_VARIANTS}
+# The token-wise comparator (LongCache-style dynamic selection of single
+# tokens, no static eviction) on the 8k and 32k shapes: every prompt token
+# kept, clusters of one token under groups of 16, and as many selected tokens
+# as the clustered workload attends in selected clusters (13 and 26 clusters
+# of 16); the groups' level keeps 10% (8k) or 5% (32k) of them.
+C3_TOKENWISE = C3.replace(name="c3_tokenwise_t8192", keep_ppm=1_000_000, cluster_size=1, fanouts=(16,),
+                          level_keep_ppm=(25_391, 100_000))
+C5_TOKENWISE = C5.replace(name="c5_tokenwise_t32768_needles", keep_ppm=1_000_000, cluster_size=1, fanouts=(16,),
+                          level_keep_ppm=(12_695, 50_000))
+WORKLOADS = {w.name: w for w in (C1, C2, C3, C4, C5) + C4_VARIANTS + (C3_TOKENWISE, C5_TOKENWISE)}
 
 
 @dataclass
@@ -192,6 +210,8 @@ def generate(work: Workload, window_rows: int, device="cpu",
     if work.rule == "needle":
         needle_pos = torch.zeros((L, B, Hkv), dtype=torch.int32)
 
+    rho = work.layer_rho_ppm / PPM
+    prev = {}  # b -> (scaled keys, S) of the previous layer (rho > 0)
     for l in range(L):
         for b in range(B):
             T = int(lens[b])
@@ -217,6 +237,8 @@ def generate(work: Workload, window_rows: int, device="cpu",
             scale = torch.ones((Hkv, d), **f32)
             scale.scatter_(1, ch, 8.0)
             K = K * scale[:, None, :]
+            if rho > 0 and b in prev:
+                K = rho * prev[b][0] + (1.0 - rho * rho) ** 0.5 * K
             u = None
             if work.rule == "needle":
                 u = torch.randn((Hkv, d), generator=gs, **f32)
@@ -235,11 +257,19 @@ def generate(work: Workload, window_rows: int, device="cpu",
             # 5% seeded position subset per kv head; queries follow its keys
             n_s = max(1, (T * 5 + 99) // 100)
             S = torch.stack([torch.randperm(T, generator=gs, device=device)[:n_s] for _ in range(Hkv)])
+            if rho > 0:
+                if b in prev:
+                    stay = torch.rand((Hkv, n_s), generator=gs, device=device) < rho
+                    S = torch.where(stay, prev[b][1], S)
+                prev[b] = (K, S)
             Kf = Kq.float()
+            # rho > 0: the targeted slots come from one stream per sequence
+            gp = {"q": st.gen(0, 6 + 16 * b), "d": st.gen(0, 7 + 16 * b)} if rho > 0 else None
 
-            def draw_q(count: int, gen: torch.Generator) -> torch.Tensor:
+            def draw_q(count: int, gen: torch.Generator, which: str) -> torch.Tensor:
                 # [Hq][count][d]: q = 0.7 k_j (+ 0.35 u) + noise
-                pick = torch.randint(0, n_s, (Hq, count), generator=gen, device=device)
+                pick = torch.randint(0, n_s, (Hq, count), generator=gen if gp is None else gp[which],
+                                     device=device)
                 kvh = torch.arange(Hq, device=device) // G
                 j = S[kvh[:, None], pick]
                 kj = Kf[kvh[:, None], j]
@@ -249,8 +279,8 @@ def generate(work: Workload, window_rows: int, device="cpu",
                 return 0.35 * kj + 0.7 * u[kvh][:, None, :] + 0.622 * noise
 
             rows = min(R, T)
-            q_win[l, b, :, R - rows:] = draw_q(rows, gq).to(dt)
-            q_dec[:, l, b] = draw_q(E, gd).permute(1, 0, 2).to(dt)
+            q_win[l, b, :, R - rows:] = draw_q(rows, gq, "q").to(dt)
+            q_dec[:, l, b] = draw_q(E, gd, "d").permute(1, 0, 2).to(dt)
             kn = torch.randn((E, Hkv, d), generator=gd, **f32) * scale[None]
             k_new[:, l, b] = kn.to(dt)
             v_new[:, l, b] = torch.randn((E, Hkv, d), generator=gd, **f32).to(dt)

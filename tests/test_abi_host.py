@@ -34,7 +34,7 @@ def test_exports_every_declared_symbol(lib):
                          capture_output=True, text=True).stdout
     exported = set(re.findall(r"\b(mpc_\w+)\b", out))
     assert set(names) <= exported
-    assert lib.mpc_abi_version() == mpcache.ABI_VERSION == 6
+    assert lib.mpc_abi_version() == mpcache.ABI_VERSION == 7
 
 
 def test_struct_layout_matches_c(tmp_path):
@@ -219,6 +219,15 @@ def test_commonality_validation(lib):
     a.sel = a.out_total = a.out_score = None
     assert lib.mpc_commonality(C.byref(a), None) == mpcache.MPC_ERR_INVALID_ARG  # NULL pointers
     for field, bad in (("m", 0), ("m", 4), ("k", 9), ("n_layers", 1), ("sel_layer_stride", 47)):
+        b = mpcache.CommonalityArgs.from_buffer_copy(a)
+        setattr(b, field, bad)
+        assert lib.mpc_commonality(C.byref(b), None) == mpcache.MPC_ERR_BAD_SHAPE, field
+    # the position map: checked before any launch (the fake pointers are never read)
+    a.sel, a.out_total, a.out_score = 16, 32, 48
+    a.kept, a.kept_layer_stride, a.kept_cap, a.cluster_size = 64, 2 * 3 * 40, 40, 16
+    assert lib.mpc_commonality(C.byref(a), None) == mpcache.MPC_ERR_INVALID_ARG  # no n_keep / prompt_len
+    a.n_keep, a.prompt_len = 80, 96
+    for field, bad in (("cluster_size", 0), ("kept_cap", 0), ("kept_layer_stride", 2 * 3 * 40 - 1)):
         b = mpcache.CommonalityArgs.from_buffer_copy(a)
         setattr(b, field, bad)
         assert lib.mpc_commonality(C.byref(b), None) == mpcache.MPC_ERR_BAD_SHAPE, field

@@ -696,6 +696,72 @@ def test_commonality_of_unshared_selections():
                 assert int(total[b, h]) == round(ref * n_sel * (w.n_layers - m))
 
 
+def test_adaptive_sharing_loop():
+    """Adaptive cross-layer index sharing end to end (Sec. 2 Obs. 3, Sec. 3.4):
+    every layer its own leader, the commonality of the selected tokens on the
+    GPU for windows of 2 .. 4 layers at every decode step (exact totals
+    against the oracle's commonality of the same selections as positions, and
+    against the oracle's own pipeline where its kept sets and selections are
+    the GPU's), the group size from mpc_choose_share_every against the rule
+    worked by hand, then the method run with that group size against the
+    oracle.  Adjacent layers are correlated (rho = 0.95) as a residual stream
+    would make them; on these inputs the oracle's commonality is about 0.37,
+    0.15 and 0.09 for windows of 2, 3 and 4 layers, so a threshold of 0.25
+    shares between pairs of layers."""
+    from paper_2501_06807_gb300 import mpcache
+    w = synth.C3.replace(n_layers=6, prompt_len=2048, prompt_len_min=2048, n_q_heads=8, n_kv_heads=2,
+                         keep_ppm=500_000, share_every=1, layer_rho_ppm=950_000)
+    E, L, s, Hkv = 3, w.n_layers, w.cluster_size, w.n_kv_heads
+    R = H.window_rows_for(w)
+    x = synth.generate(w, R, device="cpu", decode_steps=E)
+    xc = H.to_cuda(x)
+    eng = H.make_engine(w, E)
+    eng.prefill(xc.k, xc.v, xc.q_win, x.prompt_lens.cuda())
+    res = H.oracle_run(x, E, list(range(L)))
+    T = int(x.prompt_lens[0])
+    ms = (1, 2, 3)
+    scores = {m: [] for m in ms}
+    units = same = 0
+    for e in range(E):
+        eng.decode_step(xc.q[e], xc.k_new[e], xc.v_new[e])
+        torch.cuda.synchronize()
+        sel, kept = eng.sel.cpu().numpy(), eng.kept.cpu().numpy()
+        n_sel, nk = int(eng.n_sel[0]), int(eng.n_keep[0])
+        assert n_sel >= 1
+        prev_total = None
+        for m in ms:
+            total, score = eng.commonality(m)
+            total, score = total.cpu().numpy(), score.cpu().numpy()
+            for h in range(Hkv):
+                pos = [O.selected_positions(kept[l, 0, h, :nk], T, sel[l, 0, h, :n_sel], s) for l in range(L)]
+                ref = O.commonality(pos, n_sel * s, m)
+                assert total[0, h] == round(ref * n_sel * s * (L - m)), (e, m, h)
+                assert abs(score[0, h] - ref) <= 1e-6
+                agree = all(np.array_equal(kept[l, 0, h, :nk], res.kept[(l, 0, h)]) and
+                            np.array_equal(sel[l, 0, h, :n_sel], res.selected[(e, l, 0, h)]) for l in range(L))
+                units += 1
+                if agree:
+                    same += 1
+                    pos_o = [O.selected_positions(res.kept[(l, 0, h)], T, res.selected[(e, l, 0, h)], s)
+                             for l in range(L)]
+                    assert O.commonality(pos_o, n_sel * s, m) == ref
+                scores[m].append(float(score[0, h]))
+            # a window of m + 1 layers shares no more than its first m
+            if prev_total is not None:
+                assert (total <= prev_total).all()
+            prev_total = total
+    assert same >= 0.9 * units, (same, units)
+    mean = {m: float(np.mean(v)) for m, v in scores.items()}
+    for thr in (0.0, 0.25, 0.5, 0.75, 1.0):
+        want = max([1] + [m + 1 for m in ms if mean[m] >= thr])
+        assert mpcache.choose_share_every(mean, thr) == want, (thr, mean)
+    chosen = mpcache.choose_share_every(mean, 0.25)
+    H.log_parity("adaptive_sharing", case=w.name, rho_ppm=w.layer_rho_ppm, commonality=mean, threshold=0.25,
+                 chosen_share_every=chosen, units_matching_oracle=same, units=units)
+    assert chosen >= 2, mean
+    _pipeline(w.replace(share_every=chosen), E, list(range(L)))
+
+
 # ------------------------------------------ full size, sampled outputs ----
 
 def _full_size_sampled(w, E, pick):

@@ -617,6 +617,32 @@ def test_p11_commonality():
     assert O.commonality([sel[0], sel[1]], k, 1) == 1.0      # layers 2, 3 share
 
 
+def test_p11_selected_positions_name_the_cached_tokens():
+    """The positions of a selected cluster are the tokens its cache rows hold:
+    a kept row holds the prompt key at its position, a row appended at
+    decode step e holds that step's key, at position prompt_len + e."""
+    assert O.selected_positions([3, 7, 9, 12], 14, [1, 2], 2) == [9, 12, 14, 15]
+    assert O.selected_positions([0, 5], 6, [], 2) == []
+    rng = np.random.default_rng(5)
+    L, Hkv, T, d, s, E = 2, 2, 40, 8, 4, 10
+    K = rng.standard_normal((L, Hkv, T, d)); V = rng.standard_normal((L, Hkv, T, d))
+    Qw = rng.standard_normal((L, Hkv, T, d))
+    q = rng.standard_normal((E, L, Hkv, d)); kn = rng.standard_normal((E, L, Hkv, d))
+    p = O.Params(keep_ppm=500_000, cluster_size=s, fanouts=(2,), level_keep_ppm=(250_000, 500_000), share_every=1)
+    res = O.run(lambda l, b: K[l], lambda l, b: V[l], lambda l, b: Qw[l], lambda e, l, b: q[e, l],
+                lambda e, l, b: kn[e, l], lambda e, l, b: V[l][:, 0] * 0, [T], p, steps=E, layers=[0, 1])
+    for l in range(L):
+        for h in range(Hkv):
+            kept = res.kept[(l, 0, h)]
+            cache = np.vstack([res.cache_k[(l, 0, h)], kn[:, l, h]])   # every row after E appends
+            n_clusters = cache.shape[0] // s
+            for c in range(n_clusters):
+                pos = O.selected_positions(kept, T, [c], s)
+                want = [K[l, h, x] if x < T else kn[x - T, l, h] for x in pos]
+                assert np.array_equal(np.array(want), cache[c * s:(c + 1) * s]), (l, h, c)
+            assert len(set(O.selected_positions(kept, T, range(n_clusters), s))) == n_clusters * s
+
+
 def test_mean_summary_composes_by_member_counts():
     """A coarse cluster's mean key is its children's means weighted by their
     token counts (the last cluster of a level may hold fewer children)."""
