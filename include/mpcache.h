@@ -316,19 +316,25 @@ MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace,
  *   attn.alpha).
  * - speculate: -1 automatic, 0 or 1: whether the selection's first round
  *   also scores every cluster of the level below the coarsest (one
- *   dependent round fewer, more rows read).
+ *   dependent round fewer, more rows read); both forms of the step.
  * - static_ppm, slice_tiles: the attention's tile list is cut into one
  *   contiguous range per warp for its first static_ppm parts per million,
  *   the rest into slices of slice_tiles tiles that warps claim once their
  *   range is done (a balance for SMs that stream slower); 1e6 keeps every
- *   tile static; 0 picks either.
- * With bf16 caches and the EQ3 / BOUND / MEAN metrics the step is one
- * persistent kernel: selection teams publish each unit's ids in the
+ *   tile static; 0 picks either.  (Fused kernel only.)
+ * - fuse: 0 or -1 (automatic): two launches, mpc_select's kernel followed by
+ *   mpc_sparse_decode_attn's (with programmatic stream serialization, so the
+ *   attention kernel becomes resident while the selection runs); 1: one
+ *   persistent kernel for the whole step where it applies (bf16 caches, the
+ *   EQ3 / BOUND / MEAN metrics, at most 1024 candidates at a level), else
+ *   the two launches.  Measured on GB300, the two launches are the faster
+ *   form on the 8k and 32k GQA workloads (22.8 and 32.0 us per step against
+ *   25.2 and 35.6) and within 1.5% of the fused kernel on the 2k MHA one,
+ *   so automatic takes them.
+ * In the fused kernel, selection teams publish each unit's ids in the
  * workspace (each word tagged with the call) and the attention warps wait
  * for them (bounded, 1 s; a wait that gives up sets flag 1 of
- * mpc_device_status and the call's outputs are undefined).  Otherwise (fp32 caches, MPC_SIM_FXP,
- * more than 1024 candidates at a level) it is mpc_select's kernel followed
- * by mpc_sparse_decode_attn's.
+ * mpc_device_status and the call's outputs are undefined).
  * Workspace: mpc_decode_step_workspace_size bytes, zero-filled once; the
  * call leaves it ready for the next call, except after a wait that gave up
  * (flag 1 of mpc_device_status): zero-fill it again before the next call. */
@@ -341,6 +347,7 @@ typedef struct {
   int32_t speculate;           /* -1 = automatic */
   int32_t static_ppm;          /* share of the attention tiles in static warp ranges; 0 = automatic */
   int32_t slice_tiles;         /* tiles per dynamically claimed slice of the rest; 0 = automatic */
+  int32_t fuse;                /* 1 = one fused kernel; 0 / -1 (automatic) = selection + attention launches */
 } mpc_decode_args;
 
 MPC_API int mpc_decode_step_workspace_size(const mpc_decode_args* args, size_t* bytes);

@@ -328,8 +328,7 @@ int validate_select(const mpc_select_args* a, SelectParams* p) {
 // ---------------------------------------------------------- attention ----
 struct AttnPlan {
   int units, n_split, tps;
-  int rec_slots, static_ppm, slice_tiles;  // bf16: the step kernel's split
-  size_t part_off, ucnt_off, gcnt_off, ctl_off, bytes;
+  size_t part_off, ucnt_off, gcnt_off, bytes;
 };
 
 int validate_attn(const mpc_attn_args* a, AttnParams* p, AttnPlan* plan) {
@@ -383,24 +382,16 @@ int validate_attn(const mpc_attn_args* a, AttnParams* p, AttnPlan* plan) {
   };
   if (a->dtype == MPC_BF16) {
     // persistent kernel: two partial records per warp of the grid
-    if (a->batch > kStepBatchMax)
-      return fail(MPC_ERR_BAD_SHAPE, "batch %d > %d sequences per call", a->batch, kStepBatchMax);
-    // the step kernel with no selection units: two partial records per range slot
-    int wpc = 0, nst = 0;
-    step_shape(a->head_dim, G, a->batch, &wpc, &nst);
-    StepParams bal;
-    const long long ntm = (a->cluster_size + 15) / 16 + ((long long)a->sel_cap * a->cluster_size + 15) / 16;
-    step_balance(units, ntm, wpc, 0, 0, &bal);
-    plan->rec_slots = bal.rec_slots;
-    plan->static_ppm = bal.static_ppm;
-    plan->slice_tiles = bal.slice_tiles;
-    plan->part_off = take((size_t)2 * bal.rec_slots * G * (a->head_dim + 4) * sizeof(float));
+    // persistent kernel: one partial record per warp slot (at most eight
+    // warps per CTA, so 2 x 4 x G records cover a CTA's slots)
+    if (a->batch > attn_persist_batch_max())
+      return fail(MPC_ERR_BAD_SHAPE, "batch %d > %d sequences per call", a->batch, attn_persist_batch_max());
+    plan->part_off = take((size_t)2 * attn_persist_ctas_max() * 4 * G * (a->head_dim + 4) * sizeof(float));
   } else {
     plan->part_off = take(n_split > 1 ? (size_t)units * n_split * G * (a->head_dim + 4) * sizeof(float) : 0);
   }
   plan->ucnt_off = take((size_t)units * sizeof(int));
   plan->gcnt_off = take(sizeof(int));
-  plan->ctl_off = take(8 * sizeof(int));
   plan->bytes = off;
 
   p->n_refs = a->n_refs;
@@ -507,6 +498,11 @@ int validate_step(const mpc_decode_args* a, StepParams* sp, SelectParams* sel, S
   sa.frac_bits = a->frac_bits;
   MPC_TRY(validate_select(&sa, sel));
   if (a->speculate < -1 || a->speculate > 1) return fail(MPC_ERR_BAD_SHAPE, "speculate %d not in {-1, 0, 1}", a->speculate);
+  if (a->fuse < -1 || a->fuse > 1) return fail(MPC_ERR_BAD_SHAPE, "fuse %d not in {-1, 0, 1}", a->fuse);
+  // an explicit speculate applies to the selection kernel of the two-launch
+  // path too (its first round then stages the level below only if it fits
+  // the row buffer sized above)
+  if (a->speculate >= 0) sel->spec_first = a->speculate;
 
   const int D = t.head_dim, G = sp->a.G, B = t.batch, s = t.cluster_size;
   const int units = plan->attn.units;
@@ -514,8 +510,9 @@ int validate_step(const mpc_decode_args* a, StepParams* sp, SelectParams* sel, S
   const int n_src = select_n_src(a->metric);
   int wpc = 0, nst = 0;
   step_shape(D, G, B, &wpc, &nst);
-  // published ids and counts are 16-bit values
-  plan->fused = t.dtype == MPC_BF16 && a->metric != MPC_SIM_FXP && sel->max_cand <= 1024 &&
+  // published ids and counts are 16-bit values; two launches unless the
+  // fused kernel is asked for (they measured faster, see the header)
+  plan->fused = a->fuse == 1 && t.dtype == MPC_BF16 && a->metric != MPC_SIM_FXP && sel->max_cand <= 1024 &&
                 step_smem_bytes(D, G, B) <= kSmemOptin && t.cap_tokens / s < 65535 && t.sel_cap < 65535;
   int tw = 1, rb = 0;
   if (plan->fused) {
@@ -780,20 +777,7 @@ MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace, s
   p.part = reinterpret_cast<float*>(ws + plan.part_off);
   p.unit_counter = reinterpret_cast<int*>(ws + plan.ucnt_off);
   p.grid_counter = reinterpret_cast<int*>(ws + plan.gcnt_off);
-  cudaError_t e;
-  if (args->dtype == MPC_BF16) {
-    // the decode step kernel with every selection an input (no selection units)
-    StepParams sp;
-    memset(&sp, 0, sizeof(sp));
-    sp.a = p;
-    sp.ctl = reinterpret_cast<int*>(ws + plan.ctl_off);
-    sp.rec_slots = plan.rec_slots;
-    sp.static_ppm = plan.static_ppm;
-    sp.slice_tiles = plan.slice_tiles;
-    e = launch_step(sp, args->head_dim, static_cast<cudaStream_t>(stream));
-  } else {
-    e = launch_attn(p, args->dtype, args->head_dim, plan.units, static_cast<cudaStream_t>(stream));
-  }
+  const cudaError_t e = launch_attn(p, args->dtype, args->head_dim, plan.units, static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_fail(e, "mpc_sparse_decode_attn launch");
   return ok();
 }
@@ -839,18 +823,7 @@ MPC_API int mpc_decode_step(const mpc_decode_args* args, void* workspace, size_t
   sp.a.part = reinterpret_cast<float*>(ws + plan.attn.part_off);
   sp.a.unit_counter = reinterpret_cast<int*>(ws + plan.attn.ucnt_off);
   sp.a.grid_counter = reinterpret_cast<int*>(ws + plan.attn.gcnt_off);
-  if (t.dtype == MPC_BF16) {  // the step kernel with the selections as inputs
-    StepParams ap;
-    memset(&ap, 0, sizeof(ap));
-    ap.a = sp.a;
-    ap.ctl = reinterpret_cast<int*>(ws + plan.attn.ctl_off);
-    ap.rec_slots = plan.attn.rec_slots;
-    ap.static_ppm = plan.attn.static_ppm;
-    ap.slice_tiles = plan.attn.slice_tiles;
-    e = launch_step(ap, t.head_dim, st);
-  } else {
-    e = launch_attn(sp.a, t.dtype, t.head_dim, plan.attn.units, st);
-  }
+  e = launch_attn(sp.a, t.dtype, t.head_dim, plan.attn.units, st);
   if (e != cudaSuccess) return cuda_fail(e, "mpc_decode_step attention launch");
   return ok();
 }

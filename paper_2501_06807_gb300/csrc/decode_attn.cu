@@ -1,20 +1,24 @@
 // Sparse decode attention over the selected clusters and the tail, with the
-// decode-step append and the tail seal (Alg. 1; Alg. 2 Step 2; App. A), for
-// fp32 caches.  (bf16 caches take the decode step kernel, decode_step.cu,
-// with the selections as inputs.)
+// decode-step append and the tail seal (Alg. 1; Alg. 2 Step 2; App. A).
+// One unit = (ref, sequence b, kv head h); the rows a unit attends are the s
+// rows of every selected cluster, then the tail rows already in the cache,
+// then the row appended now, cut into 16-row tiles.
 //
-// Work decomposition: one unit = (ref, sequence b, kv head h).  The rows a
-// unit attends are listed in order: the s rows of every selected cluster,
-// then the tail rows already in the cache, then the row appended now.  The
-// list is cut into 16-row tiles and the tiles into `tiles_per_split` chunks,
-// one CTA per (chunk, unit).  Each of the CTA's four warps streams its tiles
-// (key rows and value rows) from HBM into its own shared-memory ring with 1-D
-// bulk copies (TMA engine, completion on an mbarrier), then computes the
-// tile's scores for all query heads of the GQA group at once and updates an
-// online softmax.  The four warps' partial results are merged in shared
-// memory; with several chunks per unit the CTA writes (max, sum, o) to the
-// workspace and the last CTA of the unit (atomic ticket, no waiting) merges
-// them by log-sum-exp and writes o.
+// bf16 caches: attn_bf16_persist_kernel, one persistent CTA per SM whose
+// warps stream equal contiguous ranges of the list of all units' tiles
+// (below, "bf16 path").
+//
+// fp32 caches: attn_f32_kernel, one CTA per (chunk of `tiles_per_split`
+// tiles, unit).  Each of the CTA's four warps streams its tiles (key rows and
+// value rows) from HBM into its own shared-memory ring with 1-D bulk copies
+// (TMA engine, completion on an mbarrier), then computes the tile's scores
+// for all query heads of the GQA group at once and updates an online
+// softmax.  The four warps' partial results are merged in shared memory;
+// with several chunks per unit the CTA writes (max, sum, o) to the workspace
+// and the last CTA of the unit (atomic ticket, no waiting) merges them by
+// log-sum-exp and writes o.
+#include <mutex>
+
 #include "kernels.cuh"
 #include "seal.cuh"
 
@@ -234,6 +238,560 @@ __device__ __forceinline__ void finish_grid(const AttnParams& p) {
   }
 }
 
+// ------------------------------------------------ bf16 path (persistent) ----
+//
+// One CTA per SM, four to eight warps.  The tiles of all units (every selected
+// cluster row tile, tail and appended row of every (layer, sequence, kv
+// head)) form one list, cut into contiguous, equal ranges, one per warp slot
+// (slots interleaved over the CTAs, at most one slot per tile).  Every warp
+// streams its range through its own ring of shared-memory stages (K and V
+// tile rows), so every SM moves the same amount of KV.
+//
+// Tiles are staged with cp.async (16 bytes per lane, committed as one group
+// per tile, so a warp keeps NST tiles in flight at the cost of a few
+// instructions each).  With s a multiple of 16 every tile is one run of
+// consecutive cache rows; other cluster sizes gather the rows one by one.
+//
+// Per tile the group's heads are the N dimension of the tensor-core products
+// (S^T = K Q^T, O^T = V^T P^T with m16n8k16 bf16 mma, P split into bf16 hi +
+// lo), so one 8-head n-tile covers a GQA group of up to 8 query heads.  P
+// moves from the accumulator layout of S^T to the operand layout of P^T with
+// movmatrix (an in-register 8x8 transpose).
+//
+// A unit finished inside one warp is written directly.  A unit split across
+// warps is merged by its owner, the warp holding its first piece: that piece
+// ends its warp's range, so it finishes last in time.  Every later piece is
+// the first piece of its warp, finished early; it writes a partial (max,
+// sum, o) record (one slot per warp) and signals the owner with a release
+// reduction on the unit's counter, without waiting.  The owner waits (bounded)
+// for the count, then folds the records into its registers by log-sum-exp.
+
+constexpr int kMaxPersistCtas = 152;
+
+constexpr int kMaxBatchPersist = 512;
+constexpr int kSelSmem = 256;  // selected ids staged per warp (longer lists are read from global)
+
+template <int D>
+struct PSmem {
+  static constexpr int ROWB = D * 2;
+  static constexpr int TILEB = 16 * ROWB;
+  static __host__ __device__ constexpr int qbytes(int G) { return ((G * D * 2 + 127) / 128) * 128; }
+  static __host__ __device__ constexpr int stage(int G) { return 2 * TILEB + qbytes(G); }
+  // wpc warps per CTA, each with an nst-stage ring
+  static __host__ __device__ constexpr int key_off(int G, int nst, int wpc) { return wpc * nst * stage(G); }
+  static __host__ __device__ constexpr int sel_off(int G, int nst, int wpc) { return key_off(G, nst, wpc) + wpc * nst * 16; }
+  static __host__ __device__ constexpr int tab_off(int G, int nst, int wpc) { return sel_off(G, nst, wpc) + wpc * kSelSmem * 4; }
+  static __host__ __device__ constexpr int total(int G, int nst, int wpc, int B) { return tab_off(G, nst, wpc) + (4 * B + 2) * 4; }
+};
+
+// Warps per CTA and ring depth per warp (compile-time for
+// cp.async.wait_group).  More warps hide the per-tile compute better than
+// deeper rings at the same bytes in flight (measured: 2 x 12 and 4 x 6 are
+// slower than 6 x 4; 8 x 3 is best with one query head per group, whose
+// tiles carry the same mma work for a quarter of the heads).  d 64: 4 x 8.
+// d 128, up to 8 heads per group: 8 x 3 (one head) or 6 x 4 when that fits
+// shared memory with the batch's tables, else 4 x 5; up to 16 heads: 4 x 4.
+struct PersistCfg {
+  int wpc, nst;
+};
+inline PersistCfg persist_cfg(int D, int G, int B) {
+  if (D == 64) return {4, 8};
+  if (G == 1 && PSmem<128>::total(G, 3, 8, B) <= kSmemOptin) return {8, 3};
+  if (G <= 8 && PSmem<128>::total(G, 4, 6, B) <= kSmemOptin) return {6, 4};
+  return {4, G <= 8 ? 5 : 4};
+}
+
+struct Cursor {
+  int ri, b, h, lt;
+};
+
+// In-register transpose of an 8x8 b16 matrix held in mma fragment layout.
+__device__ __forceinline__ uint32_t movmatrix_t(uint32_t a) {
+  uint32_t d;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
+  return d;
+}
+
+template <int D, int HN, int NST, int WPC>
+__global__ void __launch_bounds__(WPC * 32, 1) attn_bf16_persist_kernel(const __grid_constant__ AttnParams p) {
+  using S = PSmem<D>;
+  constexpr int ROWB = S::ROWB;
+  constexpr int TILEB = S::TILEB;
+  constexpr int KS = D / 16;  // k-steps of S^T and m-tiles of O^T
+  extern __shared__ __align__(128) uint8_t smem[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int G = p.G, B = p.B, Hkv = p.Hkv, s = p.pyr.s;
+  const int STAGE = S::stage(G);
+  constexpr int CH = ROWB / 16;  // 16-byte chunks per row
+  uint8_t* ring = smem + warp * NST * STAGE;
+  int8_t* keys = reinterpret_cast<int8_t*>(smem + S::key_off(G, NST, WPC)) + warp * NST * 16;
+  int* sel_s = reinterpret_cast<int*>(smem + S::sel_off(G, NST, WPC)) + warp * kSelSmem;
+  int* s_nt = reinterpret_cast<int*>(smem + S::tab_off(G, NST, WPC));  // tiles per unit of sequence b
+  int* s_pre = s_nt + B;                                           // exclusive prefix of s_nt (B + 1)
+  int* s_n = s_pre + B + 1;                                        // cache rows before the append
+  int* s_k1 = s_n + B;                                             // selected clusters
+  grid_dep_launch();
+  grid_dep_wait();
+
+  // ---- per-sequence table
+  if (warp == 0) {
+    int carry = 0;
+    for (int b0 = 0; b0 < B; b0 += 32) {
+      const int b = b0 + lane;
+      int nt = 0, n = 0, k1 = 0;
+      if (b < B) {
+        // both counts are requested at once (one round trip, not two)
+        n = p.n_tok[b];
+        const int ns = p.sel_cap > 0 ? p.n_sel[b] : 0;
+        if (n < 0 || n + 1 > p.cap_tokens) {
+          atomicOr(&g_mpc_status, 2);  // no room for the append: skip the sequence
+        } else {
+          const int C1 = n / s;
+          k1 = min(ns, min(C1, p.sel_cap));
+          nt = (k1 * s + (n - C1 * s) + 1 + 15) / 16;
+        }
+      }
+      int incl = nt;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      if (b < B) {
+        s_nt[b] = nt;
+        s_pre[b] = carry + incl - nt;
+        s_n[b] = n;
+        s_k1[b] = k1;
+      }
+      carry += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) s_pre[B] = carry;
+  }
+  __syncthreads();
+  const bool fast = (s & 15) == 0;  // every tile is one run of consecutive rows
+  const int s16 = s >> 4;
+
+  const int64_t TPR = (int64_t)Hkv * s_pre[B];
+  const int64_t NT = TPR * p.n_refs;
+  const int64_t NW_all = (int64_t)gridDim.x * WPC;
+  const int NW = (int)(NW_all < NT ? NW_all : NT);
+  const int gw = warp * gridDim.x + blockIdx.x;
+  const int64_t x0 = gw < NW ? NT * gw / NW : 0, x1 = gw < NW ? NT * (gw + 1) / NW : 0;
+  auto warp_of = [&](int64_t x) { return (int)((x * NW + NW - 1) / NT); };
+  auto locate = [&](int64_t x) {
+    Cursor c;
+    c.ri = (int)(x / TPR);
+    const int64_t rem = x - c.ri * TPR;
+    int lo = 0, hi = B - 1;  // largest b with Hkv * pre[b] <= rem
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if ((int64_t)Hkv * s_pre[mid] <= rem) lo = mid;
+      else hi = mid - 1;
+    }
+    c.b = lo;
+    const int64_t rem2 = rem - (int64_t)Hkv * s_pre[lo];
+    c.h = (int)(rem2 / s_nt[lo]);
+    c.lt = (int)(rem2 % s_nt[lo]);
+    return c;
+  };
+  auto advance = [&](Cursor& c) {
+    if (++c.lt < s_nt[c.b]) return;
+    c.lt = 0;
+    if (++c.h < Hkv) return;
+    c.h = 0;
+    do {
+      if (++c.b == B) {
+        c.b = 0;
+        ++c.ri;
+      }
+    } while (s_nt[c.b] == 0);
+  };
+  auto unit_at = [&](const Cursor& c) {
+    Unit u;
+    u.h = c.h;
+    u.b = c.b;
+    u.layer = p.refs.layer[c.ri];
+    u.group = p.refs.group[c.ri];
+    u.leader = p.refs.leader[c.ri];
+    u.n = s_n[c.b];
+    u.C1 = u.n / s;
+    u.tail = u.n - u.C1 * s;
+    u.k1 = s_k1[c.b];
+    u.n_sel_rows = u.k1 * s;
+    u.n_att = u.n_sel_rows + u.tail + 1;
+    u.n_tiles = s_nt[c.b];
+    u.t_begin = 0;
+    u.t_end = u.n_tiles;
+    u.sel = p.sel + ((int64_t)(u.group * B + c.b) * Hkv + c.h) * p.sel_cap;
+    return u;
+  };
+  auto kv_base = [&](const Unit& u, int which) {
+    const bf16* base = (const bf16*)(which ? p.vc : p.kc) + u.layer * p.cache_ls +
+                       (int64_t)(u.b * Hkv + u.h) * p.cap_tokens * D;
+    return reinterpret_cast<const uint8_t*>(base);
+  };
+  const int nj = (int)(x1 - x0);
+
+  // ---- issue side: runs NST tiles ahead of the compute side
+  Unit iu;
+  const uint8_t* ikb = nullptr;
+  const uint8_t* ivb = nullptr;
+  auto issue = [&](const Cursor& c, int j) {
+    const bool first = (j == 0) || (c.lt == 0);
+    if (first) {
+      iu = unit_at(c);
+      ikb = kv_base(iu, 0);
+      ivb = kv_base(iu, 1);
+      if (iu.k1 <= kSelSmem) {  // stage the unit's selected ids once
+        __syncwarp();
+        for (int i = lane; i < iu.k1; i += 32) sel_s[i] = iu.sel[i];
+        __syncwarp();
+        iu.sel = sel_s;
+      }
+    }
+    uint8_t* sK = ring + (j % NST) * STAGE;
+    uint8_t* sV = sK + TILEB;
+    const int t = c.lt;
+    const int a0 = t * 16;
+    const int ncache = max(0, min(16, iu.n_att - 1 - a0));  // cache rows of the tile
+    if (fast) {
+      int src0;
+      if (a0 < iu.n_sel_rows) {
+        const int ci = t / s16;
+        int id = iu.sel[ci];
+        if (id < 0 || id >= iu.C1) {
+          if (lane == 0) atomicOr(&g_mpc_status, 4);
+          id = 0;
+        }
+        src0 = id * s + (a0 - ci * s);
+      } else {
+        src0 = iu.C1 * s + (a0 - iu.n_sel_rows);
+      }
+      const uint8_t* gk = ikb + (int64_t)src0 * ROWB;
+      const uint8_t* gv = ivb + (int64_t)src0 * ROWB;
+      for (int i = lane; i < ncache * CH; i += 32) {
+        cp_async16(sK + i * 16, gk + i * 16);
+        cp_async16(sV + i * 16, gv + i * 16);
+      }
+    } else {
+      const int r = lane & 15;
+      const int arow = a0 + r;
+      int src = 0;
+      if (r < ncache) src = src_row(iu, s, arow);
+      else if (arow == iu.n_att - 1) src = iu.n;
+      if (lane < 16) keys[(j % NST) * 16 + r] = (int8_t)((arow < iu.n_att) ? (src & 7) : (r & 7));
+#pragma unroll 4
+      for (int i = lane; i < 16 * CH; i += 32) {
+        const int row = i / CH, ch = i % CH;
+        const int srow = __shfl_sync(0xffffffffu, src, row);
+        if (row < ncache) {
+          cp_async16(sK + i * 16, ikb + (int64_t)srow * ROWB + ch * 16);
+          cp_async16(sV + i * 16, ivb + (int64_t)srow * ROWB + ch * 16);
+        }
+      }
+    }
+    if (first) {
+      const uint8_t* q = reinterpret_cast<const uint8_t*>((const bf16*)p.q + iu.layer * p.q_ls +
+                                                          ((int64_t)iu.b * p.Hq + iu.h * G) * D);
+      for (int i = lane; i < G * D * 2 / 16; i += 32) cp_async16(sK + 2 * TILEB + i * 16, q + i * 16);
+    }
+  };
+
+  Cursor cc, ic;
+  if (nj > 0) {
+    cc = locate(x0);
+    ic = cc;
+    for (int j = 0; j < NST; ++j) {
+      if (j < nj) {
+        issue(ic, j);
+        advance(ic);
+      }
+      cp_async_commit();
+    }
+  }
+
+  // ---- compute side
+  uint32_t qb[HN][KS][2];  // Q^T operand: k = channels, n = heads
+  float o[KS][HN][4];      // O^T accumulators: m = channels, n = heads
+  float m_run[HN][2], l_run[HN][2];
+  Unit u;
+  int u_ri = 0;
+  bool have = false;
+  const int r_tok = lane >> 2;      // token row of S^T (and +8)
+  const int h_off = 2 * (lane & 3);  // first of this thread's two heads in an n-tile
+
+  auto flush = [&]() {
+    float lq[HN][2];
+#pragma unroll
+    for (int hn = 0; hn < HN; ++hn)
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        float v = l_run[hn][e];
+        v += __shfl_xor_sync(0xffffffffu, v, 4);
+        v += __shfl_xor_sync(0xffffffffu, v, 8);
+        v += __shfl_xor_sync(0xffffffffu, v, 16);
+        lq[hn][e] = v;
+      }
+    const int64_t ustart = (int64_t)u_ri * TPR + (int64_t)Hkv * s_pre[u.b] + (int64_t)u.h * s_nt[u.b];
+    const int64_t uend = ustart + s_nt[u.b];
+    const bool before = ustart < x0, after = uend > x1;
+    float* outp = p.out + u.layer * p.out_ls + ((int64_t)u.b * p.Hq + u.h * G) * D;
+    const int64_t unit_id = ((int64_t)u_ri * B + u.b) * Hkv + u.h;
+    if (before) {
+      // a later piece of a unit that began in an earlier warp: publish the
+      // (max, sum, o) record and signal the unit's owner, without waiting
+      float* dst = p.part + (int64_t)gw * G * (D + 4);
+#pragma unroll
+      for (int hn = 0; hn < HN; ++hn)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int g = hn * 8 + h_off + e;
+          if (g < G) {
+            if (r_tok == 0) {
+              dst[g * (D + 4)] = m_run[hn][e];
+              dst[g * (D + 4) + 1] = lq[hn][e];
+            }
+#pragma unroll
+            for (int mt = 0; mt < KS; ++mt) {
+              dst[g * (D + 4) + 4 + mt * 16 + r_tok] = o[mt][hn][e];
+              dst[g * (D + 4) + 4 + mt * 16 + r_tok + 8] = o[mt][hn][2 + e];
+            }
+          }
+        }
+      __syncwarp();
+      if (lane == 0) red_release_add(&p.unit_counter[unit_id], 1);
+    } else {
+      if (after) {
+        // this warp holds the unit's first piece, which ends last in time:
+        // wait for the later pieces' records and merge them into registers
+        const int nother = warp_of(uend - 1) - gw;
+        if (lane == 0) {
+          if (ld_acquire(&p.unit_counter[unit_id]) < nother) {
+            const uint64_t t0 = global_timer_ns();
+            while (ld_acquire(&p.unit_counter[unit_id]) < nother) {
+              if (global_timer_ns() - t0 > 1000000000ull) {
+                atomicOr(&g_mpc_status, kStatusWaitTimeout);
+                break;
+              }
+              __nanosleep(64);
+            }
+          }
+          p.unit_counter[unit_id] = 0;
+        }
+        __syncwarp();
+        // the records of warps gw + 1 .. gw + nother are contiguous: copy
+        // them into this warp's ring (idle: the owner piece ends the warp's
+        // range, after its last tile) with one batch of copies in flight,
+        // instead of one dependent round trip per record
+        const int rec = G * (D + 4);
+        const float* recs = p.part + (int64_t)(gw + 1) * rec;
+        const bool staged = nother * rec * 4 <= NST * STAGE;
+        auto ld_rec = [&](const float* a) { return staged ? *a : __ldcg(a); };
+        if (staged) {
+          const uint8_t* src = reinterpret_cast<const uint8_t*>(recs);
+          for (int i = lane; i < nother * rec / 4; i += 32) cp_async16(ring + i * 16, src + i * 16);
+          cp_async_commit();
+          cp_async_wait<0>();
+          __syncwarp();
+          recs = reinterpret_cast<const float*>(ring);
+        }
+        for (int k = 1; k <= nother; ++k) {
+          const float* rec_k = recs + (int64_t)(k - 1) * rec;
+#pragma unroll
+          for (int hn = 0; hn < HN; ++hn)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+              const int g = hn * 8 + h_off + e;
+              if (g < G) {
+                const float* rg = rec_k + g * (D + 4);
+                const float mk = ld_rec(rg), lk = ld_rec(rg + 1);
+                const float M = fmaxf(m_run[hn][e], mk);
+                const float wa = (m_run[hn][e] == kNegInf) ? 0.f : fast_exp2(m_run[hn][e] - M);
+                const float wb = (mk == kNegInf) ? 0.f : fast_exp2(mk - M);
+                m_run[hn][e] = M;
+                lq[hn][e] = lq[hn][e] * wa + lk * wb;
+#pragma unroll
+                for (int mt = 0; mt < KS; ++mt) {
+                  o[mt][hn][e] = o[mt][hn][e] * wa + wb * ld_rec(rg + 4 + mt * 16 + r_tok);
+                  o[mt][hn][2 + e] = o[mt][hn][2 + e] * wa + wb * ld_rec(rg + 4 + mt * 16 + r_tok + 8);
+                }
+              }
+            }
+        }
+      }
+#pragma unroll
+      for (int hn = 0; hn < HN; ++hn)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int g = hn * 8 + h_off + e;
+          if (g < G) {
+            const float inv = 1.f / lq[hn][e];
+#pragma unroll
+            for (int mt = 0; mt < KS; ++mt) {
+              outp[g * D + mt * 16 + r_tok] = o[mt][hn][e] * inv;
+              outp[g * D + mt * 16 + r_tok + 8] = o[mt][hn][2 + e] * inv;
+            }
+          }
+        }
+    }
+    // the piece that holds the appended row seals a full tail
+    if (uend <= x1) seal_tail<bf16, D>(p, u, reinterpret_cast<const bf16*>(kv_base(u, 0)));
+  };
+
+  for (int j = 0; j < nj; ++j) {
+    const int st = j % NST;
+    uint8_t* sK = ring + st * STAGE;
+    uint8_t* sV = sK + TILEB;
+    int8_t* kk = keys + st * 16;
+    const bool new_unit = (j == 0) || (cc.lt == 0);
+    if (new_unit) {
+      if (have) flush();
+      u = unit_at(cc);
+      u_ri = cc.ri;
+      have = true;
+#pragma unroll
+      for (int hn = 0; hn < HN; ++hn) {
+        m_run[hn][0] = m_run[hn][1] = kNegInf;
+        l_run[hn][0] = l_run[hn][1] = 0.f;
+#pragma unroll
+        for (int mt = 0; mt < KS; ++mt) o[mt][hn][0] = o[mt][hn][1] = o[mt][hn][2] = o[mt][hn][3] = 0.f;
+      }
+    }
+    cp_async_wait<NST - 1>();  // this lane's copies of tile j have landed
+    __syncwarp();
+    if (new_unit) {
+      // Q^T operand from the stage's q slot: b0 = q[head][2c, 2c+1], b1 = +8
+      const bf16* qs = reinterpret_cast<const bf16*>(sK + 2 * TILEB);
+#pragma unroll
+      for (int hn = 0; hn < HN; ++hn) {
+        const int hq = hn * 8 + r_tok;
+#pragma unroll
+        for (int ks = 0; ks < KS; ++ks) {
+          const int c = ks * 16 + h_off;
+          qb[hn][ks][0] = (hq < G) ? *reinterpret_cast<const uint32_t*>(qs + hq * D + c) : 0u;
+          qb[hn][ks][1] = (hq < G) ? *reinterpret_cast<const uint32_t*>(qs + hq * D + c + 8) : 0u;
+        }
+      }
+    }
+    const int t = cc.lt;
+    const int n_valid = min(16, u.n_att - t * 16);
+    const int cur_r = (u.n_att - 1) - t * 16;
+    if (cur_r < 16 || n_valid < 16) {
+      constexpr int CH = ROWB / 16;
+      if (cur_r >= 0 && cur_r < 16) {
+        // the appended row goes from the inputs to the cache and to this tile
+        const int64_t nb = u.layer * p.kvn_ls + (int64_t)(u.b * Hkv + u.h) * D;
+        const uint4* kn = reinterpret_cast<const uint4*>((const bf16*)p.k_new + nb);
+        const uint4* vn = reinterpret_cast<const uint4*>((const bf16*)p.v_new + nb);
+        bf16* kcw = (bf16*)p.kc + u.layer * p.cache_ls + (int64_t)(u.b * Hkv + u.h) * p.cap_tokens * D;
+        bf16* vcw = (bf16*)p.vc + u.layer * p.cache_ls + (int64_t)(u.b * Hkv + u.h) * p.cap_tokens * D;
+        for (int i = lane; i < 2 * CH; i += 32) {
+          const int ch = i % CH;
+          const bool isv = i >= CH;
+          const uint4 val = isv ? vn[ch] : kn[ch];
+          const int pch = ch ^ (u.n & 7);
+          *reinterpret_cast<uint4*>((isv ? sV : sK) + cur_r * ROWB + pch * 16) = val;
+          reinterpret_cast<uint4*>((isv ? vcw : kcw) + (int64_t)u.n * D)[pch] = val;
+        }
+      }
+      // rows past the end of the list are zeroed so that P V sees finite values
+      for (int i = lane; i < (16 - n_valid) * CH; i += 32)
+        reinterpret_cast<uint4*>(sV + n_valid * ROWB)[i] = make_uint4(0, 0, 0, 0);
+      __syncwarp();
+    }
+    // S^T = K Q^T: 16 tokens x 8 heads per n-tile, two accumulators per
+    // n-tile (even / odd k-steps) to halve the dependency chain
+    float sc[HN][2][4];
+#pragma unroll
+    for (int hn = 0; hn < HN; ++hn)
+#pragma unroll
+      for (int a2 = 0; a2 < 2; ++a2) sc[hn][a2][0] = sc[hn][a2][1] = sc[hn][a2][2] = sc[hn][a2][3] = 0.f;
+    {
+      // A = K tile: matrices (tok 0-7, ch 2ks), (tok 8-15, 2ks), (tok 0-7, 2ks+1), (tok 8-15, 2ks+1)
+      const int tok = ((lane >> 3) & 1) * 8 + (lane & 7);
+      const int key = fast ? (tok & 7) : kk[tok];
+      const uint32_t base = smem_u32(sK + tok * ROWB);
+      const int chb = lane >> 4;
+#pragma unroll
+      for (int ks = 0; ks < KS; ++ks) {
+        uint32_t a[4];
+        ldsm_x4(base + ((((2 * ks + chb) ^ key)) << 4), a[0], a[1], a[2], a[3]);
+#pragma unroll
+        for (int hn = 0; hn < HN; ++hn) mma_bf16(sc[hn][ks & 1], a, qb[hn][ks][0], qb[hn][ks][1]);
+      }
+    }
+    uint32_t pbh[HN][2], pbl[HN][2];
+    float corr[HN][2];
+#pragma unroll
+    for (int hn = 0; hn < HN; ++hn) {
+      float x[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int tk = r_tok + (e >> 1) * 8;
+        x[e] = (t * 16 + tk < u.n_att) ? (sc[hn][0][e] + sc[hn][1][e]) * p.scale_log2 : kNegInf;
+      }
+      float pr[4];
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {  // this thread's two heads
+        float mx = fmaxf(x[e], x[e + 2]);
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+        const float mnew = fmaxf(m_run[hn][e], mx);
+        corr[hn][e] = (m_run[hn][e] == kNegInf) ? 0.f : fast_exp2(m_run[hn][e] - mnew);
+        m_run[hn][e] = mnew;
+        pr[e] = fast_exp2(x[e] - mnew);
+        pr[e + 2] = fast_exp2(x[e + 2] - mnew);
+        l_run[hn][e] = l_run[hn][e] * corr[hn][e] + pr[e] + pr[e + 2];
+      }
+      // P^T operand (k = tokens, n = heads): transpose the 8x8 blocks of P
+      const __nv_bfloat162 h01 = __floats2bfloat162_rn(pr[0], pr[1]);
+      const __nv_bfloat162 h23 = __floats2bfloat162_rn(pr[2], pr[3]);
+      const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+      pbh[hn][0] = movmatrix_t(*reinterpret_cast<const uint32_t*>(&h01));
+      pbh[hn][1] = movmatrix_t(*reinterpret_cast<const uint32_t*>(&h23));
+      pbl[hn][0] = movmatrix_t(pack_bf16(pr[0] - f01.x, pr[1] - f01.y));
+      pbl[hn][1] = movmatrix_t(pack_bf16(pr[2] - f23.x, pr[3] - f23.y));
+    }
+#pragma unroll
+    for (int mt = 0; mt < KS; ++mt)
+#pragma unroll
+      for (int hn = 0; hn < HN; ++hn) {
+        o[mt][hn][0] *= corr[hn][0];
+        o[mt][hn][1] *= corr[hn][1];
+        o[mt][hn][2] *= corr[hn][0];
+        o[mt][hn][3] *= corr[hn][1];
+      }
+    {
+      // A = V^T tile: transposed matrices (tok 0-7, ch 2mt), (tok 0-7, 2mt+1), (tok 8-15, 2mt), (tok 8-15, 2mt+1)
+      const int tok = (lane >> 4) * 8 + (lane & 7);
+      const int key = fast ? (tok & 7) : kk[tok];
+      const uint32_t base = smem_u32(sV + tok * ROWB);
+      const int chb = (lane >> 3) & 1;
+#pragma unroll
+      for (int mt = 0; mt < KS; ++mt) {
+        uint32_t a[4];
+        ldsm_x4_t(base + ((((2 * mt + chb) ^ key)) << 4), a[0], a[1], a[2], a[3]);
+#pragma unroll
+        for (int hn = 0; hn < HN; ++hn) {
+          mma_bf16(o[mt][hn], a, pbh[hn][0], pbh[hn][1]);
+          mma_bf16(o[mt][hn], a, pbl[hn][0], pbl[hn][1]);
+        }
+      }
+    }
+    __syncwarp();
+    if (j + NST < nj) {
+      issue(ic, j + NST);
+      advance(ic);
+    }
+    cp_async_commit();  // one group per tile, empty near the end
+    advance(cc);
+  }
+  cp_async_wait<0>();
+  if (have) flush();
+  finish_grid(p);
+}
+
 // ------------------------------------------------------------- f32 path ----
 template <int D, int GM>
 __global__ void __launch_bounds__(128) attn_f32_kernel(const __grid_constant__ AttnParams p) {
@@ -417,6 +975,17 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const __grid_constant__ A
 
 // ------------------------------------------------------------- launch ----
 
+int attn_smem_bytes(int dtype, int D, int G, int B) {
+  if (dtype == MPC_BF16) {
+    const PersistCfg c = persist_cfg(D, G, B);
+    return D == 64 ? PSmem<64>::total(G, c.nst, c.wpc, B) : PSmem<128>::total(G, c.nst, c.wpc, B);
+  }
+  return D == 64 ? Smem<64, 4>::total(G) : Smem<128, 4>::total(G);
+}
+
+int attn_persist_ctas_max() { return kMaxPersistCtas; }
+int attn_persist_batch_max() { return kMaxBatchPersist; }
+
 template <typename K>
 static cudaError_t launch_k(K kernel, dim3 grid, int smem, cudaStream_t st, const AttnParams& p, int threads = 128) {
   cudaError_t e = ensure_dyn_smem((const void*)kernel, smem);
@@ -424,11 +993,44 @@ static cudaError_t launch_k(K kernel, dim3 grid, int smem, cudaStream_t st, cons
   return launch_pdl(kernel, grid, dim3(threads), smem, st, p);
 }
 
+// CTAs of the persistent grid: one per SM, at most kMaxPersistCtas.
+static int persist_ctas() {
+  static std::mutex mu;
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return kMaxPersistCtas;
+  std::lock_guard<std::mutex> lk(mu);
+  if (cached[dev] == 0) {
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
+      sms = kMaxPersistCtas;
+    cached[dev] = sms < kMaxPersistCtas ? sms : kMaxPersistCtas;
+  }
+  return cached[dev];
+}
+
 cudaError_t launch_attn(const AttnParams& p0, int dtype, int D, int n_units, cudaStream_t st) {
-  const AttnParams& p = p0;
-  if (dtype != MPC_F32) return cudaErrorInvalidValue;
+  AttnParams p = p0;
+  if (dtype == MPC_BF16) {
+    const PersistCfg c = persist_cfg(D, p.G, p.B);
+    p.n_stages = c.nst;
+    const int smem = attn_smem_bytes(dtype, D, p.G, p.B);
+    const dim3 grid(persist_ctas());
+    const int th = 32 * c.wpc;
+#define MPC_PERSIST(DD, HH, NN, WW)                                                                 \
+  if (D == DD && (p.G <= 8 ? 1 : 2) == HH && c.nst == NN && c.wpc == WW)                           \
+    return launch_k(attn_bf16_persist_kernel<DD, HH, NN, WW>, grid, smem, st, p, th);
+    MPC_PERSIST(64, 1, 8, 4)
+    MPC_PERSIST(128, 1, 3, 8)
+    MPC_PERSIST(128, 1, 4, 6)
+    MPC_PERSIST(128, 1, 5, 4)
+    MPC_PERSIST(64, 2, 8, 4)
+    MPC_PERSIST(128, 2, 4, 4)
+#undef MPC_PERSIST
+    return cudaErrorInvalidValue;
+  }
   const dim3 grid(p.n_split, n_units);
-  const int smem = D == 64 ? Smem<64, 4>::total(p.G) : Smem<128, 4>::total(p.G);
+  const int smem = attn_smem_bytes(dtype, D, p.G, p.B);
   const int G = p.G;
 #define MPC_F32_CASE(DD, GG) \
   if (D == DD && G <= GG) return launch_k(attn_f32_kernel<DD, GG>, grid, smem, st, p);

@@ -173,8 +173,12 @@ __host__ __device__ inline int select_n_src(int metric) {
   return metric == MPC_SIM_BOUND || metric == MPC_SIM_FXP ? 2 : 1;
 }
 
-// fp32 attention (split grid, last-CTA merge)
+// Sparse decode attention: bf16 caches on the persistent kernel (one CTA
+// per SM, owner merges), fp32 caches on the split grid (last-CTA merge).
 cudaError_t launch_attn(const AttnParams& p, int dtype, int D, int n_units, cudaStream_t st);
+int attn_smem_bytes(int dtype, int D, int G, int B);
+int attn_persist_ctas_max();
+int attn_persist_batch_max();
 cudaError_t launch_step(const StepParams& p, int D, cudaStream_t st);
 int step_smem_bytes(int D, int G, int B);
 // CTA shape of the fused step kernel: warps per CTA and ring stages per warp

@@ -113,7 +113,7 @@ class DecodeArgs(C.Structure):
     """mpc_decode_args: the arguments of mpc_decode_step (attention arguments plus selection settings)."""
     _fields_ = [("struct_size", C.c_uint32), ("attn", AttnArgs), ("level_keep_ppm", C.c_int32 * MAX_LEVELS),
                 ("metric", C.c_int32), ("frac_bits", C.c_int32), ("speculate", C.c_int32),
-                ("static_ppm", C.c_int32), ("slice_tiles", C.c_int32)]
+                ("static_ppm", C.c_int32), ("slice_tiles", C.c_int32), ("fuse", C.c_int32)]
 
 
 ENTRY_POINTS = ("mpc_static_evict_workspace_size", "mpc_build_clusters_workspace_size",
@@ -596,7 +596,7 @@ class Engine:
 
     def step_args(self, q, k_new, v_new, advance=True, out=None, metric: int = MPC_SIM_EQ3,
                   frac_bits: int = FXP_FRAC_BITS, speculate: int = -1, static_ppm: int = 0,
-                  slice_tiles: int = 0) -> DecodeArgs:
+                  slice_tiles: int = 0, fuse: int = -1) -> DecodeArgs:
         """The checked mpc_decode_args of one whole decode step of every
         processed layer (selection of the leaders, then attention)."""
         a = DecodeArgs()
@@ -606,18 +606,19 @@ class Engine:
         a._refs = att._refs  # which stays alive as long as the args
         a.level_keep_ppm = _fan(self.level_keep_ppm)
         a.metric, a.frac_bits, a.speculate = metric, frac_bits, speculate
-        a.static_ppm, a.slice_tiles = static_ppm, slice_tiles
+        a.static_ppm, a.slice_tiles, a.fuse = static_ppm, slice_tiles, fuse
         return a
 
     def decode_step(self, q, k_new, v_new, out=None, metric: int = MPC_SIM_EQ3, speculate: int = -1,
-                    static_ppm: int = 0, slice_tiles: int = 0):
+                    static_ppm: int = 0, slice_tiles: int = 0, fuse: int = -1):
         """One decode step of every layer in one call (mpc_decode_step):
         q [L][B][Hq][d], k_new / v_new [L][B][Hkv][d] (layer index = position
         along dim 0).  Same selections and outputs as ``select`` followed by
-        ``attend``."""
+        ``attend``; ``fuse`` = 1 runs the step as one fused kernel, -1 / 0 as
+        the selection and attention launches."""
         lib = load()
         a = self.step_args(q, k_new, v_new, True, out, metric, speculate=speculate, static_ppm=static_ppm,
-                           slice_tiles=slice_tiles)
+                           slice_tiles=slice_tiles, fuse=fuse)
         n = C.c_size_t(0)
         _check(lib.mpc_decode_step_workspace_size(C.byref(a), C.byref(n)))
         ws = _ws_zero(n.value, self._ws, "step")

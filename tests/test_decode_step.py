@@ -1,7 +1,8 @@
 """mpc_decode_step (one call per decode step) against the two calls it fuses.
 
-The fused step runs the leaders' selection and every layer's attention in one
-persistent kernel.  It is specified to give the selections of mpc_select
+With ``fuse`` = 1 the step runs the leaders' selection and every layer's
+attention in one persistent kernel (the automatic setting launches the two
+kernels of mpc_select and mpc_sparse_decode_attn, also checked here).  It is specified to give the selections of mpc_select
 followed by mpc_sparse_decode_attn: the same fp32 similarity arithmetic and
 ranking (so the selected ids are identical, no tie band), the same appended
 rows and seals (so caches and pyramids are bit-identical), and the same
@@ -45,6 +46,7 @@ def _twin(w, E, **step_kw):
     assert torch.equal(fused.rep, ref.rep) and torch.equal(fused.kc, ref.kc)
     worst = 0.0
     metric = step_kw.pop("metric", mpcache.MPC_SIM_EQ3)
+    step_kw.setdefault("fuse", 1)
     for e in range(E):
         fused.decode_step(x.q[e], x.k_new[e], x.v_new[e], metric=metric, **step_kw)
         ref.select(x.q[e], metric=metric)
@@ -101,6 +103,9 @@ CASES = [
     ("prompt_shorter_than_a_cluster", synth.C3.replace(n_layers=2, prompt_len=12, prompt_len_min=12,
                                                        n_q_heads=4, n_kv_heads=2, keep_ppm=1_000_000,
                                                        fanouts=(2,), share_every=1), 24, {}),
+    ("automatic_two_launches", synth.C5.replace(n_layers=6, prompt_len=4096, prompt_len_min=4096, n_q_heads=8,
+                                                n_kv_heads=2, level_keep_ppm=(100_000, 250_000, 500_000)), 20,
+     dict(fuse=-1)),
     ("fp32_two_launch_path", synth.C1.replace(n_layers=2, prompt_len=300, prompt_len_min=300), 18, {}),
     ("fixed_point_two_launch_path", synth.C3.replace(n_layers=3, prompt_len=1024, prompt_len_min=1024,
                                                      n_q_heads=8, n_kv_heads=2), 17,
@@ -113,11 +118,13 @@ def test_fused_step_equals_two_calls(name, w, E, kw):
     _twin(w, E, **dict(kw))
 
 
-def test_fused_step_is_one_launch_in_a_graph():
-    """The fused step replays inside a CUDA graph (one kernel per step, the
-    published selections and counters of the workspace carried from replay to
-    replay) and gives the eager run's outputs bit for bit (the static split
-    and the canonical merge order make them deterministic)."""
+@pytest.mark.parametrize("fuse", [1, -1])
+def test_decode_step_replays_in_a_graph(fuse):
+    """The decode step replays inside a CUDA graph (fused: one kernel per
+    step, the published selections and counters of the workspace carried
+    from replay to replay; automatic: the selection and attention launches)
+    and gives the eager run's outputs bit for bit (static splits and fixed
+    merge orders make them deterministic)."""
     w = synth.C3.replace(n_layers=6, prompt_len=2048, prompt_len_min=2048, n_q_heads=8, n_kv_heads=2)
     E = 20
     x = H.to_cuda(synth.generate(w, H.window_rows_for(w), device="cpu", decode_steps=E))
@@ -128,13 +135,13 @@ def test_fused_step_is_one_launch_in_a_graph():
     for eng in (eager, graphed):
         eng.prefill(x.k, x.v, x.q_win, lens)
     for e in range(E):
-        eager.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=outs_e[e])
-    graphed.decode_step(x.q[0], x.k_new[0], x.v_new[0], out=outs_g[0])  # allocates the workspace
+        eager.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=outs_e[e], fuse=fuse)
+    graphed.decode_step(x.q[0], x.k_new[0], x.v_new[0], out=outs_g[0], fuse=fuse)  # allocates the workspace
     torch.cuda.synchronize()
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g):
         for e in range(1, E):
-            graphed.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=outs_g[e])
+            graphed.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=outs_g[e], fuse=fuse)
     g.replay()
     torch.cuda.synchronize()
     diff = (outs_g - outs_e).abs().amax(dim=(2, 3, 4))  # [step][layer]
