@@ -65,6 +65,10 @@ def parse_args():
     p.add_argument("--level-keep-ppm", help="comma-separated kept ppm per level, finest first")
     p.add_argument("--share-every", type=int)
     p.add_argument("--layer-rho-ppm", type=int)
+    # the decode step's form: speculative first selection round (-1 auto),
+    # and one fused kernel (1) or the selection + attention launches (-1 / 0)
+    p.add_argument("--speculate", type=int, choices=[-1, 0, 1], default=-1)
+    p.add_argument("--fuse", type=int, choices=[-1, 0, 1], default=-1)
     # measured side reports instead of the bench line (one JSON line each):
     # adaptive-sharing: commonality of unshared selections, the group size the
     # adaptive rule picks, and the decode step with it; tokenwise: selection
@@ -269,9 +273,11 @@ def run_ours(args, rank, world, dist):
     def prefill():
         eng.prefill(x.k, x.v, x.q_win, lens, pt, w.page_size)
 
+    step_kw = dict(speculate=args.speculate, fuse=args.fuse)
+
     def decode_all():
         for e in range(E):
-            eng.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=out_all[e])
+            eng.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=out_all[e], **step_kw)
 
     # eager pass: counts the attended rows of every step, checks the status
     prefill()
@@ -280,7 +286,7 @@ def run_ours(args, rank, world, dist):
     s = w.cluster_size
     rep_rows = 0
     for e in range(E):
-        eng.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=out_all[e])
+        eng.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=out_all[e], **step_kw)
         n_sel = eng.n_sel.cpu().tolist()
         for b in range(w.batch):
             n_tok = n_keep[b] + e
@@ -339,12 +345,12 @@ def run_ours(args, rank, world, dist):
         gf = torch.cuda.CUDAGraph()
         prefill()
         for e in range(E):  # eager once: the fused call's workspace
-            eng.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=out_all[e], fuse=1)
+            eng.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=out_all[e], speculate=args.speculate, fuse=1)
         prefill()
         torch.cuda.synchronize()
         with torch.cuda.graph(gf):
             for e in range(E):
-                eng.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=out_all[e], fuse=1)
+                eng.decode_step(x.q[e], x.k_new[e], x.v_new[e], out=out_all[e], speculate=args.speculate, fuse=1)
         per = []
         for i in range(5):
             prefill()
@@ -510,12 +516,13 @@ def run_ours(args, rank, world, dist):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": w.dtype, "data": "synthetic (seeded generator shaped like the paper's models; no datasets or weights)",
-        "config": workload_config(w, E, f"replicas{world}"),
+        "config": dict(workload_config(w, E, f"replicas{world}"), speculate=args.speculate, fuse=args.fuse),
         # per step: static eviction (two score passes + budget, plus the gather
         # of paged bf16 keys), gathering (+ coarse levels), and per decode step
         # a selection and an attention kernel
         "gpu_launches": args.steps * (3 + (1 if w.paged and w.dtype == "bf16" else 0) + 1 +
-                                      (1 if len(w.fanouts) else 0) + 2 * E),
+                                      (1 if len(w.fanouts) else 0) +
+                                      (1 if args.fuse == 1 and w.dtype == "bf16" else 2) * E),
         "static_scoring_path": "tcgen05" if tensor_path else "simt",
         "phases_ms": {"static_evict": static_ms, "build_clusters": build_ms, "decode_all_steps": decode_ms},
         "decode_step_us": decode_ms / E * 1e3,

@@ -173,6 +173,28 @@ inline cudaError_t launch_pdl(void (*kernel)(P...), dim3 grid, dim3 block, size_
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<A>(args)...);
 }
 
+// launch_pdl for a kernel whose CTAs wait on one another: a cooperative
+// launch, which starts the grid only when every CTA can be resident at once
+// (and fails, with nothing launched, for a grid that could never be), so
+// every such wait ends.
+template <typename... P, typename... A>
+inline cudaError_t launch_pdl_coop(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                                   A&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[2];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  at[1].id = cudaLaunchAttributeCooperative;
+  at[1].val.cooperative = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 2;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<A>(args)...);
+}
+
 // Raises a kernel's dynamic shared-memory limit once per (kernel, device), so
 // later launches (including ones recorded into a CUDA graph) skip the call.
 inline cudaError_t ensure_dyn_smem(const void* kernel, int bytes) {

@@ -993,6 +993,15 @@ static cudaError_t launch_k(K kernel, dim3 grid, int smem, cudaStream_t st, cons
   return launch_pdl(kernel, grid, dim3(threads), smem, st, p);
 }
 
+// The persistent kernel's owners wait for pieces held by other CTAs, so its
+// grid is launched cooperatively: all CTAs resident together.
+template <typename K>
+static cudaError_t launch_persist(K kernel, dim3 grid, int smem, cudaStream_t st, const AttnParams& p, int threads) {
+  cudaError_t e = ensure_dyn_smem((const void*)kernel, smem);
+  if (e != cudaSuccess) return e;
+  return launch_pdl_coop(kernel, grid, dim3(threads), smem, st, p);
+}
+
 // CTAs of the persistent grid: one per SM, at most kMaxPersistCtas.
 static int persist_ctas() {
   static std::mutex mu;
@@ -1019,7 +1028,7 @@ cudaError_t launch_attn(const AttnParams& p0, int dtype, int D, int n_units, cud
     const int th = 32 * c.wpc;
 #define MPC_PERSIST(DD, HH, NN, WW)                                                                 \
   if (D == DD && (p.G <= 8 ? 1 : 2) == HH && c.nst == NN && c.wpc == WW)                           \
-    return launch_k(attn_bf16_persist_kernel<DD, HH, NN, WW>, grid, smem, st, p, th);
+    return launch_persist(attn_bf16_persist_kernel<DD, HH, NN, WW>, grid, smem, st, p, th);
     MPC_PERSIST(64, 1, 8, 4)
     MPC_PERSIST(128, 1, 3, 8)
     MPC_PERSIST(128, 1, 4, 6)
