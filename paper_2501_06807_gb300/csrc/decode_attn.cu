@@ -265,6 +265,8 @@ __device__ __forceinline__ void finish_grid(const AttnParams& p) {
 // sum, o) record (one slot per warp) and signals the owner with a release
 // reduction on the unit's counter, without waiting.  The owner waits (bounded)
 // for the count, then folds the records into its registers by log-sum-exp.
+// The grid is launched cooperatively (launch_persist), so every CTA whose
+// piece an owner waits for is resident.
 
 constexpr int kMaxPersistCtas = 152;
 
@@ -565,19 +567,27 @@ __global__ void __launch_bounds__(WPC * 32, 1) attn_bf16_persist_kernel(const __
         // this warp holds the unit's first piece, which ends last in time:
         // wait for the later pieces' records and merge them into registers
         const int nother = warp_of(uend - 1) - gw;
+        int arrived = 1;
         if (lane == 0) {
           if (ld_acquire(&p.unit_counter[unit_id]) < nother) {
             const uint64_t t0 = global_timer_ns();
             while (ld_acquire(&p.unit_counter[unit_id]) < nother) {
               if (global_timer_ns() - t0 > 1000000000ull) {
                 atomicOr(&g_mpc_status, kStatusWaitTimeout);
+                arrived = 0;
                 break;
               }
               __nanosleep(64);
             }
           }
-          p.unit_counter[unit_id] = 0;
+          // a wait that gave up leaves the counter to the late pieces (the
+          // caller zero-fills the workspace again after flag 1)
+          if (arrived) p.unit_counter[unit_id] = 0;
         }
+        arrived = __shfl_sync(0xffffffffu, arrived, 0);
+        // no partial output: a unit whose records did not all arrive keeps
+        // its previous o and is reported by flag 1 only
+        if (!arrived) goto unit_done;
         __syncwarp();
         // the records of warps gw + 1 .. gw + nother are contiguous: copy
         // them into this warp's ring (idle: the owner piece ends the warp's
@@ -634,6 +644,7 @@ __global__ void __launch_bounds__(WPC * 32, 1) attn_bf16_persist_kernel(const __
           }
         }
     }
+  unit_done:
     // the piece that holds the appended row seals a full tail
     if (uend <= x1) seal_tail<bf16, D>(p, u, reinterpret_cast<const bf16*>(kv_base(u, 0)));
   };

@@ -324,8 +324,7 @@ __global__ void __launch_bounds__(WPC * 32, 1) decode_step_kernel(const __grid_c
               }
               tsync();
               float4 qv[V4];
-#pragma unroll
-              for (int jj = 0; jj < V4; ++jj) qv[jj] = reinterpret_cast<const float4*>(qsum)[ql + 4 * jj];
+              qv_load_order<D>(qv, qsum, ql, rot);
               for (int r0 = twarp * 8; r0 < nb; r0 += TW * 8) {
                 const int r = r0 + rs;
                 float a = 0.f;

@@ -177,8 +177,7 @@ __global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_ker
       constexpr int V4 = D / 16;  // float4 chunks per lane
       const int ql = lane & 3, rs = lane >> 2, rot = rs & 1;
       float4 qv[V4];
-#pragma unroll
-      for (int jj = 0; jj < V4; ++jj) qv[jj] = reinterpret_cast<const float4*>(qsum)[ql + 4 * jj];
+      qv_load_order<D>(qv, qsum, ql, rot);
       for (int r0 = warp * 8; r0 < nrows; r0 += NW * 8) {
         const int r = r0 + rs;
         float a = 0.f;
