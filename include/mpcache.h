@@ -25,7 +25,9 @@
  *   space is the caller's too: `*_workspace_size` reports how many bytes a
  *   call needs and the call receives them as `workspace`.  A workspace must
  *   be 16-byte aligned and zero-filled once before its first use; the calls
- *   that keep counters in it leave them zero, so it can be reused as is.
+ *   that keep counters in it leave them zero, so it can be reused as is,
+ *   except after a call whose bounded wait gave up (flag 1 of
+ *   mpc_device_status): zero-fill the workspace again before reusing it.
  * - Every call is asynchronous on `stream` (a cudaStream_t; NULL = legacy
  *   default stream) and returns once its kernels are queued.  Arguments are
  *   validated on the host before anything is launched.
@@ -447,10 +449,16 @@ MPC_API int64_t mpc_summary_rows(int32_t cap_tokens, int32_t cluster_size,
 /* Thread-local description of the last error of this thread ("" if none). */
 MPC_API const char* mpc_last_error(void);
 
-/* Device status word of the current device: nonzero once a kernel of this
- * library gave up a bounded wait (for a bulk copy that did not complete);
- * such a kernel skips the rest of its work and returns.  Blocks on the
- * device (cudaDeviceSynchronize), returns the flags and clears them. */
+/* Device status word of the current device: flag 1 once a kernel of this
+ * library gave up a bounded wait (for a bulk copy, or for a split unit's
+ * pieces, that did not arrive); such a kernel skips the work that needed
+ * the wait (an attention unit whose pieces did not all arrive keeps its
+ * previous output, no partial o is written) and returns; the call's outputs
+ * are then undefined and its workspace must be zero-filled again.  Flag 2:
+ * a decode step found no cache row left (the sequence is skipped, its token
+ * count kept); flag 4: an index out of range was reported and skipped.
+ * Blocks on the device (cudaDeviceSynchronize), returns the flags and
+ * clears them. */
 MPC_API int mpc_device_status(int* flags);
 
 /* Failure-path self-test: launches one kernel whose wait is never
