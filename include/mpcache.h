@@ -324,15 +324,18 @@ MPC_API int mpc_sparse_decode_attn(const mpc_attn_args* args, void* workspace,
  *   the rest into slices of slice_tiles tiles that warps claim once their
  *   range is done (a balance for SMs that stream slower); 1e6 keeps every
  *   tile static; 0 picks either.  (Fused kernel only.)
- * - fuse: 0 or -1 (automatic): two launches, mpc_select's kernel followed by
+ * - fuse: 0: two launches, mpc_select's kernel followed by
  *   mpc_sparse_decode_attn's (with programmatic stream serialization, so the
  *   attention kernel becomes resident while the selection runs); 1: one
  *   persistent kernel for the whole step where it applies (bf16 caches, the
  *   EQ3 / BOUND / MEAN metrics, at most 1024 candidates at a level), else
- *   the two launches.  Measured on GB300, the two launches are the faster
- *   form on the 8k and 32k GQA workloads (22.8 and 32.0 us per step against
- *   25.2 and 35.6) and within 1.5% of the fused kernel on the 2k MHA one,
- *   so automatic takes them.
+ *   the two launches; -1 (automatic): the fused kernel for 305 to 1216
+ *   selection units (leader refs x batch x kv heads), the two launches
+ *   otherwise.  Measured on GB300 (us per step, two launches / fused): 8k
+ *   GQA, 80 units, 23.2 / 25.3; 32k GQA, 80 units, 31.7 / 35.2; 2k MHA, 544
+ *   units, 32.1 / 31.2; paged batch 1, 544 units, 42.4 / 39.5; batch 4,
+ *   2176 units, 90.5 / 96.2; batch 32, 17408 units, 693 / 700.
+ *   mpc_decode_step_plan reports which form a call takes.
  * In the fused kernel, selection teams publish each unit's ids in the
  * workspace (each word tagged with the call) and the attention warps wait
  * for them (bounded, 1 s; a wait that gives up sets flag 1 of
@@ -349,10 +352,13 @@ typedef struct {
   int32_t speculate;           /* -1 = automatic */
   int32_t static_ppm;          /* share of the attention tiles in static warp ranges; 0 = automatic */
   int32_t slice_tiles;         /* tiles per dynamically claimed slice of the rest; 0 = automatic */
-  int32_t fuse;                /* 1 = one fused kernel; 0 / -1 (automatic) = selection + attention launches */
+  int32_t fuse;                /* 1 = one fused kernel, 0 = selection + attention launches, -1 = automatic */
 } mpc_decode_args;
 
 MPC_API int mpc_decode_step_workspace_size(const mpc_decode_args* args, size_t* bytes);
+/* Validates like mpc_decode_step and writes the kernel launches the call
+ * makes (1: the fused kernel, 2: selection then attention); host only. */
+MPC_API int mpc_decode_step_plan(const mpc_decode_args* args, int32_t* launches);
 MPC_API int mpc_decode_step(const mpc_decode_args* args, void* workspace, size_t workspace_bytes,
                             void* stream);
 

@@ -510,9 +510,14 @@ int validate_step(const mpc_decode_args* a, StepParams* sp, SelectParams* sel, S
   const int n_src = select_n_src(a->metric);
   int wpc = 0, nst = 0;
   step_shape(D, G, B, &wpc, &nst);
-  // published ids and counts are 16-bit values; two launches unless the
-  // fused kernel is asked for (they measured faster, see the header)
-  plan->fused = a->fuse == 1 && t.dtype == MPC_BF16 && a->metric != MPC_SIM_FXP && sel->max_cand <= 1024 &&
+  // published ids and counts are 16-bit values.  Automatic: the fused kernel
+  // for 305-1216 selection units (2-8 per SM, where the standalone
+  // selection runs its 4-warp form and its latency shows: measured faster on
+  // the 2k MHA and batch-1 paged workloads), two launches otherwise
+  // (measured faster on the 8k and 32k GQA workloads and at batch 4-32)
+  const bool want = a->fuse == 1 || (a->fuse == -1 && plan->sel_units > 2 * kStepCtasMax &&
+                                     plan->sel_units <= 8 * kStepCtasMax);
+  plan->fused = want && t.dtype == MPC_BF16 && a->metric != MPC_SIM_FXP && sel->max_cand <= 1024 &&
                 step_smem_bytes(D, G, B) <= kSmemOptin && t.cap_tokens / s < 65535 && t.sel_cap < 65535;
   int tw = 1, rb = 0;
   if (plan->fused) {
@@ -789,6 +794,16 @@ MPC_API int mpc_decode_step_workspace_size(const mpc_decode_args* args, size_t* 
   StepPlan plan;
   MPC_TRY(validate_step(args, &sp, &sel, &plan));
   *bytes = plan.bytes;
+  return ok();
+}
+
+MPC_API int mpc_decode_step_plan(const mpc_decode_args* args, int32_t* launches) {
+  if (launches == nullptr) return fail(MPC_ERR_INVALID_ARG, "launches is NULL");
+  StepParams sp;
+  SelectParams sel;
+  StepPlan plan;
+  MPC_TRY(validate_step(args, &sp, &sel, &plan));
+  *launches = plan.fused ? 1 : 2;
   return ok();
 }
 

@@ -121,7 +121,8 @@ ENTRY_POINTS = ("mpc_static_evict_workspace_size", "mpc_build_clusters_workspace
                 "mpc_static_evict", "mpc_build_clusters", "mpc_select", "mpc_sparse_decode_attn",
                 "mpc_summary_rows", "mpc_last_error", "mpc_device_status", "mpc_abi_version",
                 "mpc_sparse_decode_attn_static_scratch", "mpc_commonality", "mpc_selftest_wait",
-                "mpc_decode_step_workspace_size", "mpc_decode_step", "mpc_layer_refs", "mpc_choose_share_every")
+                "mpc_decode_step_workspace_size", "mpc_decode_step", "mpc_decode_step_plan", "mpc_layer_refs",
+                "mpc_choose_share_every")
 
 _LIB = None
 
@@ -165,6 +166,8 @@ def load(path: Optional[str] = None) -> C.CDLL:
     lib.mpc_layer_refs.argtypes = [C.c_int32, C.c_int32, C.c_void_p]
     lib.mpc_choose_share_every.restype = C.c_int
     lib.mpc_choose_share_every.argtypes = [C.c_int32, C.POINTER(C.c_float), C.c_float]
+    lib.mpc_decode_step_plan.restype = C.c_int
+    lib.mpc_decode_step_plan.argtypes = [C.c_void_p, C.POINTER(C.c_int32)]
     if lib.mpc_abi_version() != ABI_VERSION:
         raise MPCError(MPC_ERR_INVALID_ARG,
                        f"libmpcache ABI {lib.mpc_abi_version()} does not match the binding's {ABI_VERSION}")
@@ -614,8 +617,8 @@ class Engine:
         """One decode step of every layer in one call (mpc_decode_step):
         q [L][B][Hq][d], k_new / v_new [L][B][Hkv][d] (layer index = position
         along dim 0).  Same selections and outputs as ``select`` followed by
-        ``attend``; ``fuse`` = 1 runs the step as one fused kernel, -1 / 0 as
-        the selection and attention launches."""
+        ``attend``; ``fuse`` = 1 runs the step as one fused kernel, 0 as the
+        selection and attention launches, -1 lets the library choose."""
         lib = load()
         a = self.step_args(q, k_new, v_new, True, out, metric, speculate=speculate, static_ppm=static_ppm,
                            slice_tiles=slice_tiles, fuse=fuse)
@@ -642,6 +645,14 @@ class Engine:
             raise ValueError("commonality needs a selection of at least one cluster per sequence")
         return commonality(self.sel, k, m, bound, kept=self.kept, cluster_size=self.s,
                            n_keep=self.n_keep, prompt_len=self.prompt_lens)
+
+    def decode_step_launches(self, q, k_new, v_new, out=None, metric: int = MPC_SIM_EQ3, fuse: int = -1) -> int:
+        """Kernel launches ``decode_step`` makes with these arguments
+        (mpc_decode_step_plan: 1 for the fused kernel, 2 otherwise)."""
+        a = self.step_args(q, k_new, v_new, True, out, metric, fuse=fuse)
+        n = C.c_int32(0)
+        _check(load().mpc_decode_step_plan(C.byref(a), C.byref(n)))
+        return n.value
 
     def decode_step_two_calls(self, q, k_new, v_new, out=None):
         """The same decode step as two calls: ``select`` (leaders), then

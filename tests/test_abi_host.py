@@ -323,6 +323,13 @@ def test_decode_step_validation(lib):
         a.attn.refs = C.cast(refs, C.POINTER(mpcache.LayerRef))
         assert _ws(lib, "mpc_decode_step_workspace_size", a)[0] == mpcache.MPC_ERR_INVALID_ARG
         assert b"leader" in lib.mpc_last_error()
+    # the form a call takes: two launches unless the fused kernel is asked for
+    # or chosen (305-1216 selection units); the fixture has 2 units
+    for fuse, want in ((0, 2), (-1, 2), (1, 1)):
+        n = C.c_int32(0)
+        assert lib.mpc_decode_step_plan(C.byref(_step_args(fuse=fuse)), C.byref(n)) == 0, lib.mpc_last_error()
+        assert n.value == want, (fuse, n.value)
+    assert lib.mpc_decode_step_plan(C.byref(_step_args(fuse=2)), C.byref(C.c_int32(0))) == mpcache.MPC_ERR_BAD_SHAPE
     # the call rejects a missing workspace before launching anything
     a = _step_args()
     a.attn.n_tok = a.attn.out = a.attn.sel = a.attn.n_sel = 8192

@@ -3,12 +3,14 @@
 mpc_sparse_decode_attn_static_scratch serves callers that cannot allocate
 device memory: it keeps its split-K scratch in a fixed array inside the
 library instead of a caller workspace.  These tests call it through the C ABI
-and check it against the regular entry point (same tolerance as the other
-attention tests), twice in a row so that state left in the shared array by
-the first call cannot leak into the second.  The file sorts last so that a
-run stopping at the first failure has already run every other test.
+and check it against the regular entry point and against the oracle's
+sparse attention over the same cache rows and selection (same tolerance as
+the other attention tests), twice in a row so that state left in the shared
+array by the first call cannot leak into the second.  The file sorts last so
+that a run stopping at the first failure has already run every other test.
 """
 import ctypes as C
+import math
 
 import numpy as np
 import pytest
@@ -34,6 +36,27 @@ def _static_call(lib, eng, q, kn, vn, advance):
     assert rc == 0, lib.mpc_last_error()
 
 
+def _oracle_worst(eng, x, e, w, got):
+    """The largest relative error of ``got`` ([layer][b][Hq][d]) against the
+    oracle's sparse attention (Alg. 1) over the engine's cache rows (the
+    appended row included) and its selection, for sequence 0."""
+    G, d, s = w.group, w.head_dim, w.cluster_size
+    n = int(eng.n_tok[0])  # rows before this step's append
+    n_sel = int(eng.n_sel[0])
+    sel = eng.sel.cpu().numpy()
+    worst = 0.0
+    for l in range(w.n_layers):
+        for h in range(w.n_kv_heads):
+            K = H.unswizzle(eng.kc[l, 0, h, :n + 1].cpu()).double().numpy()
+            V = H.unswizzle(eng.vc[l, 0, h, :n + 1].cpu()).double().numpy()
+            toks = O.attended_tokens(n, s, sel[eng.group_of[l], 0, h, :n_sel])
+            for g in range(G):
+                q = x.q[e, l, 0, h * G + g].double().cpu().numpy()
+                ref = O.sparse_attention(q, K[toks], V[toks], 1 / math.sqrt(d))
+                worst = max(worst, H.rel_err(got[l, 0, h * G + g].double().cpu().numpy(), ref))
+    return worst
+
+
 @pytest.mark.parametrize("Hq,Hkv,n_layers", [(8, 2, 3), (4, 4, 1)])
 def test_static_scratch_matches_workspace_path(lib, Hq, Hkv, n_layers):
     from paper_2501_06807_gb300 import mpcache
@@ -54,6 +77,7 @@ def test_static_scratch_matches_workspace_path(lib, Hq, Hkv, n_layers):
             got = eng.out.clone()
             err = (got - ref).abs().amax(dim=-1) / ref.abs().amax(dim=-1)
             assert float(err.max()) <= tol
+            assert _oracle_worst(eng, x, e, w, got) <= tol
         _static_call(lib, eng, x.q[e], x.k_new[e], x.v_new[e], advance=True)
     torch.cuda.synchronize()
     assert eng.n_tok.tolist() == [int(eng.n_keep[0]) + E]
