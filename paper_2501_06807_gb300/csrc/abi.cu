@@ -321,7 +321,15 @@ int validate_select(const mpc_select_args* a, SelectParams* p) {
   const long long budget = (kSmemOptin - 256 - (long long)select_smem_bytes(a->head_dim, P, 0, n_src)) /
                            ((long long)a->head_dim * 4 * n_src + 4);
   if (budget < 1) return fail(MPC_ERR_BAD_SHAPE, "%d candidates leave no shared memory to stage representatives", P);
-  p->row_buf = (int)(need < budget ? need : budget);
+  long long rb = need < budget ? need : budget;
+  // the 4-warp form (many units) runs six CTAs per SM: their shared memory
+  // (each plus the 1 KB the SM reserves per CTA) within the SM's 228 KB
+  if (select_threads_of(a->n_refs * a->batch * a->n_kv_heads) == 128) {
+    const long long b6 = ((233472 / 6 - 1024) - 256 - (long long)select_smem_bytes(a->head_dim, P, 0, n_src)) /
+                         ((long long)a->head_dim * 4 * n_src + 4);
+    if (b6 >= 16 && rb > b6) rb = b6;
+  }
+  p->row_buf = (int)rb;
   return MPC_OK;
 }
 

@@ -194,6 +194,7 @@ int take_status_step();
 cudaError_t launch_select(const SelectParams& p, int dtype, int D, int units, cudaStream_t st);
 int select_smem_bytes(int D, int max_cand, int row_buf, int n_src);
 int select_spec_first(int units);
+int select_threads_of(int units);
 cudaError_t launch_clusters(const ClusterParams& p, int dtype, int D, int n_units, int groups_x,
                             bool any_leader, bool host_src, cudaStream_t st);
 cudaError_t launch_static(const StaticParams& p, int dtype, int D, int n_layer_span, cudaStream_t st);

@@ -36,10 +36,12 @@ constexpr int kRankMax = 1024;  // candidates ranked by counting
 constexpr int kSelChunk = 8192; // bytes per bulk copy
 
 // Resident CTAs per SM asked of the 4-warp instantiation (many small units:
-// latency-bound, so residency sets the throughput).  Measured on the batch-32
-// paged workload: 4 (120 registers) 178 us per step, 5 (96) 153 us, 6 and 8
-// (80 and 64, with spills) 159 and 167 us.
-constexpr int kSelMinCtas128 = 5;
+// latency-bound, so residency sets the throughput); the call caps the staged
+// rows so that six CTAs' shared memory fits the SM.  Measured on the
+// batch-32 paged workload: 5 CTAs (96 registers) 163 us per selection, 6
+// (80 registers, no spills since the scoring keeps one float per chunk live)
+// 151 us; 7 and 8 spill.
+constexpr int kSelMinCtas128 = 6;
 
 // Fixed-point Eq. 3 (ring Z_{2^64}, f fractional bits) of four channels:
 // sum_j q_j rep_j with rep_j = tr(a enc(r_max_j)) + tr(b enc(r_min_j)), the
@@ -582,6 +584,7 @@ __global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_ker
 // Threads per CTA: 16 warps while the units fit one wave of SMs, 8 while
 // they fit two CTAs per SM, else 4 (up to five CTAs per SM).
 static int select_threads(int units) { return units <= 152 ? 512 : (units <= 304 ? 256 : 128); }
+int select_threads_of(int units) { return select_threads(units); }
 
 int select_smem_bytes(int D, int max_cand, int row_buf, int n_src) {
   return (int)SelLayout(D, max_cand, row_buf, n_src).total;
