@@ -582,7 +582,7 @@ __global__ void __launch_bounds__(NT, NT == 128 ? kSelMinCtas128 : 1) select_ker
 }
 
 // Threads per CTA: 16 warps while the units fit one wave of SMs, 8 while
-// they fit two CTAs per SM, else 4 (up to five CTAs per SM).
+// they fit two CTAs per SM, else 4 (six CTAs per SM).
 static int select_threads(int units) { return units <= 152 ? 512 : (units <= 304 ? 256 : 128); }
 int select_threads_of(int units) { return select_threads(units); }
 
