@@ -73,7 +73,9 @@ def parse_args():
     # adaptive-sharing: commonality of unshared selections, the group size the
     # adaptive rule picks, and the decode step with it; tokenwise: selection
     # and decode step of the clustered path and of the token-wise comparator
-    p.add_argument("--report", choices=["adaptive-sharing", "tokenwise"])
+    # read-floor: the time to read one decode step's attention tiles and
+    # nothing else (bench_floor.cu), at the step's size and multiples of it
+    p.add_argument("--report", choices=["adaptive-sharing", "tokenwise", "read-floor"])
     p.add_argument("--share-threshold", type=float, default=0.25)
     # internal: print the oracle sample of --workload as JSON (the bench runs
     # it in a child process with one BLAS thread for the single-core figure)
@@ -612,6 +614,23 @@ def run_report(args):
     build.build()
     mpcache.load()
     torch.cuda.set_device(0)
+    if args.report == "read-floor":
+        import tempfile
+        exe = os.path.join(tempfile.mkdtemp(prefix="mpc_floor_"), "bench_floor")
+        subprocess.run(["nvcc", "-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-std=c++17", "-o", exe,
+                        os.path.join(ROOT, "bench_floor.cu")], check=True)
+        for w in (synth.C3, synth.C5):
+            E = args.decode_steps or w.decode_steps
+            keep = mpcache.ppm_count(w.prompt_len, w.keep_ppm)
+            s = w.cluster_size
+            cap_rows = ((keep + E + s - 1) // s) * s + s  # the engine's cache rows per (layer, kv head)
+            clusters = keep // s
+            k1 = mpcache.ppm_count(clusters, w.level_keep_ppm[0])
+            units = w.n_layers * w.batch * w.n_kv_heads
+            r = subprocess.run([exe, str(units), str(clusters), str(k1), str(cap_rows), "6", "4", str(w.seed)],
+                               check=True, capture_output=True, text=True)
+            print(json.dumps({"report": "read-floor", "workload": w.name, **json.loads(r.stdout)}), flush=True)
+        return
     if args.report == "tokenwise":
         # the clustered method and the token-wise comparator (every prompt
         # token kept, one token per cluster) on the same shapes and inputs
