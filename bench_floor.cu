@@ -11,7 +11,9 @@
 // into one word so no load is dead.  It reports the time per launch (CUDA
 // events, after warm-up, L2 flushed by a 512 MB write before every launch)
 // at the step's size and at 2, 4, 8 and 16 times its tiles, so the fixed
-// cost of a launch of this size shows against the copy rate.
+// cost of a launch of this size shows against the copy rate; and at the
+// step's size once more with the same tiles read again right before (no
+// flush: the step's bytes then come from L2).
 //
 // usage: bench_floor <units> <clusters per unit> <selected per unit>
 //                    <cache rows per unit> <warps per CTA> <stages> <seed>
@@ -105,7 +107,7 @@ int main(int argc, char** argv) {
   const int wpc = std::atoi(argv[5]), nst = std::atoi(argv[6]);
   const unsigned seed = (unsigned)std::atoi(argv[7]);
   if (units < 1 || clusters < 1 || selected < 1 || selected > clusters || cache_rows < 16LL * (clusters + 1) ||
-      wpc < 1 || wpc > 16 || (nst != 3 && nst != 4 && nst != 5)) {
+      wpc < 1 || wpc > 16 || !(nst == 2 || nst == 3 || nst == 4 || nst == 5 || nst == 6 || nst == 8 || nst == 12)) {
     std::fprintf(stderr, "bad arguments\n");
     return 2;
   }
@@ -148,7 +150,13 @@ int main(int argc, char** argv) {
     std::fprintf(stderr, "%d warps x %d stages need %d bytes of shared memory (227 KB at most)\n", wpc, nst, smem);
     return 2;
   }
-  auto kern = nst == 3 ? floor_kernel<3> : (nst == 4 ? floor_kernel<4> : floor_kernel<5>);
+  auto kern = nst == 2 ? floor_kernel<2>
+              : nst == 3 ? floor_kernel<3>
+              : nst == 4 ? floor_kernel<4>
+              : nst == 5 ? floor_kernel<5>
+              : nst == 6 ? floor_kernel<6>
+              : nst == 8 ? floor_kernel<8>
+                         : floor_kernel<12>;
   CK(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
   const long long step_tiles = (long long)units * (selected + 1);
   cudaEvent_t a, b;
@@ -177,7 +185,20 @@ int main(int argc, char** argv) {
     std::printf("%s{\"tiles\": %lld, \"mbytes\": %.1f, \"us\": %.2f, \"gbs\": %.0f}", mi ? ", " : "", nt,
                 bytes / 1e6, us, bytes / us / 1e3);
   }
-  std::printf("]}\n");
+  // warm: the step's tiles twice in a row, the second launch timed
+  std::vector<float> wms;
+  for (int it = 0; it < 8; ++it) {
+    kern<<<sms, wpc * 32, smem>>>(kc, vc, d_tiles, step_tiles, sink);
+    CK(cudaEventRecord(a));
+    kern<<<sms, wpc * 32, smem>>>(kc, vc, d_tiles, step_tiles, sink);
+    CK(cudaEventRecord(b));
+    CK(cudaEventSynchronize(b));
+    float t = 0.f;
+    CK(cudaEventElapsedTime(&t, a, b));
+    if (it >= 3) wms.push_back(t);
+  }
+  std::sort(wms.begin(), wms.end());
+  std::printf("], \"warm_step_us\": %.2f}\n", wms[wms.size() / 2] * 1e3);
   CK(cudaDeviceSynchronize());
   return 0;
 }
