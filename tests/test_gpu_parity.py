@@ -762,6 +762,34 @@ def test_adaptive_sharing_loop():
     _pipeline(w.replace(share_every=chosen), E, list(range(L)))
 
 
+def test_commonality_positions_cover_sealed_clusters():
+    """mpc_commonality's token positions for clusters sealed while decoding
+    (R25: row r >= n_keep holds position T + r - n_keep): every cluster is
+    selected (ratio 1 at both levels), 20 steps seal one cluster of appended
+    rows, and the GPU's totals equal the oracle's commonality of the same
+    selections mapped by selected_positions."""
+    w = synth.C3.replace(n_layers=4, prompt_len=512, prompt_len_min=512, n_q_heads=4, n_kv_heads=2,
+                         keep_ppm=500_000, share_every=1, level_keep_ppm=(1_000_000, 1_000_000))
+    E, L, s = 20, w.n_layers, w.cluster_size
+    x = H.to_cuda(synth.generate(w, H.window_rows_for(w), device="cpu", decode_steps=E))
+    eng = H.make_engine(w, E)
+    eng.prefill(x.k, x.v, x.q_win, x.prompt_lens.cuda())
+    for e in range(E):
+        eng.decode_step(x.q[e], x.k_new[e], x.v_new[e])
+    eng.select(x.q[E - 1])  # selections over the cache after the last append
+    torch.cuda.synchronize()
+    T, nk, n_sel = int(x.prompt_lens[0]), int(eng.n_keep[0]), int(eng.n_sel[0])
+    assert n_sel == (nk + E) // s and n_sel * s > nk   # a sealed cluster of appended rows is selected
+    sel, kept = eng.sel.cpu().numpy(), eng.kept.cpu().numpy()
+    for m in (1, 2, 3):
+        total, _ = eng.commonality(m)
+        for h in range(w.n_kv_heads):
+            pos = [O.selected_positions(kept[l, 0, h, :nk], T, sel[l, 0, h, :n_sel], s) for l in range(L)]
+            assert max(max(p) for p in pos) >= T                   # appended positions take part
+            ref = O.commonality(pos, n_sel * s, m)
+            assert int(total[0, h]) == round(ref * n_sel * s * (L - m)), (m, h)
+
+
 # ------------------------------------------ full size, sampled outputs ----
 
 def _full_size_sampled(w, E, pick):
