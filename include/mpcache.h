@@ -18,6 +18,12 @@
  *                           softmax(q K'^T / sqrt(d)) V' over the selected
  *                           clusters and the tail (Alg. 1)
  *
+ * mpc_decode_step runs the last two for every layer of one decode step in
+ * one call (two launches, or one fused kernel; mpc_decode_step_plan says
+ * which).  mpc_layer_refs lays out the cross-layer sharing groups (Sec. 3.4),
+ * mpc_commonality measures the commonality of per-layer selections (Sec. 2,
+ * Observation 3) and mpc_choose_share_every turns it into a group size.
+ *
  * Conventions shared by every call
  * --------------------------------
  * - Pointers named "device" are CUDA device pointers owned by the caller; the
