@@ -330,6 +330,21 @@ def test_decode_step_validation(lib):
         assert lib.mpc_decode_step_plan(C.byref(_step_args(fuse=fuse)), C.byref(n)) == 0, lib.mpc_last_error()
         assert n.value == want, (fuse, n.value)
     assert lib.mpc_decode_step_plan(C.byref(_step_args(fuse=2)), C.byref(C.c_int32(0))) == mpcache.MPC_ERR_BAD_SHAPE
+    # automatic: the fused kernel from 305 to 1216 selection units (leader
+    # refs x batch x kv heads; the fixture has 1 leader ref and 2 kv heads)
+    for batch, want in ((152, 2), (153, 1), (512, 1)):
+        a = _step_args(fuse=-1)
+        a.attn.batch = batch
+        n = C.c_int32(0)
+        assert lib.mpc_decode_step_plan(C.byref(a), C.byref(n)) == 0, lib.mpc_last_error()
+        assert n.value == want, (batch, n.value)
+    a = _step_args(fuse=-1)
+    a.attn.refs[1].leader = 1
+    a.attn.refs[1].group = 1      # two leader refs: 4 units per sequence
+    a.attn.batch = 400            # 1600 units: two launches again
+    n = C.c_int32(0)
+    assert lib.mpc_decode_step_plan(C.byref(a), C.byref(n)) == 0, lib.mpc_last_error()
+    assert n.value == 2
     # the call rejects a missing workspace before launching anything
     a = _step_args()
     a.attn.n_tok = a.attn.out = a.attn.sel = a.attn.n_sel = 8192
