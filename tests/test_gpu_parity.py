@@ -526,7 +526,7 @@ def test_static_eviction(dtype, d, Hq, Hkv, lens, keep, page):
 
 # ------------------------------------------------------- full pipeline ----
 
-def _pipeline(w: synth.Workload, E: int, layers, max_skip=0.05, device="cpu"):
+def _pipeline(w: synth.Workload, E: int, layers, max_skip=0.02, device="cpu"):
     R = H.window_rows_for(w)
     x = synth.generate(w, R, device=device, decode_steps=E)
     xc = H.to_cuda(x)
