@@ -298,6 +298,10 @@ SELECT_CASES = [
     (torch.bfloat16, 128, 2, 1, 4, (), (150_000,), 2003, 2),     # 500 candidates: counting-rank path
     (torch.bfloat16, 128, 40, 20, 16, (4,), (125_000, 500_000), 700, 8),  # 160 units: 8-warp CTAs
     (torch.bfloat16, 64, 40, 40, 16, (4,), (125_000, 500_000), 600, 8),   # 320 units: 4-warp CTAs
+    # 320 units (4-warp CTAs, six per SM): 94 coarse rows and 188 children
+    # exceed the capped row buffer, so both rounds stage in several batches
+    (torch.bfloat16, 128, 40, 40, 16, (4,), (125_000, 500_000), 6000, 8),
+    (torch.bfloat16, 128, 8, 2, 16, (4, 4, 2), (60_000, 250_000, 500_000, 500_000), 4096 + 9, 2),  # four levels
 ]
 
 
