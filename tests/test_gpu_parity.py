@@ -616,8 +616,12 @@ def _pipeline(w: synth.Workload, E: int, layers, max_skip=0.02, device="cpu"):
 
 def test_pipeline_c1_full():
     """The GPT-2-small workload exactly as configured: 12 heads, 512 tokens,
-    fp32, 8 decode steps."""
-    _pipeline(synth.C1, synth.C1.decode_steps, [0], max_skip=0.0)
+    fp32, 8 decode steps; the sink token (key 0) is kept in every head."""
+    eng, _, _ = _pipeline(synth.C1, synth.C1.decode_steps, [0], max_skip=0.0)
+    kept = eng.kept.cpu().numpy()
+    n = int(eng.n_keep[0])
+    for h in range(synth.C1.n_kv_heads):
+        assert 0 in kept[0, 0, h, :n], h
 
 
 def test_pipeline_llama2_shape_reduced():

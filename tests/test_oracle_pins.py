@@ -569,6 +569,22 @@ def test_p9_sharing():
 # ---------------------------------------------------------------- P10 ------
 
 @pytest.mark.slow
+def test_p10_sink_token_kept_c1():
+    """The GPT-2-small workload's sink (key 0 scaled by 4 under the iid rule)
+    draws enough window attention that static eviction keeps it in every
+    head (a sanity check of the recipe and of the scoring, not a parity pin)."""
+    from paper_2501_06807_gb300 import synth
+    from tests import helpers as H
+    w = synth.C1
+    x = synth.generate(w, H.window_rows_for(w), decode_steps=0)
+    res = H.oracle_run(x, 0, [0])
+    for h in range(w.n_kv_heads):
+        kept = res.kept[(0, 0, h)]
+        assert 0 in kept, h
+        sc = res.scores[(0, 0, h)]
+        assert sc[0] > np.sort(sc)[len(sc) // 2] * 4   # far above the median token
+
+
 def test_p10_needles_survive_c5_shape():
     """The 32k-token needle workload at full size (layer 0, two kv heads,
     8 decode steps): every planted needle token is kept by static eviction and
