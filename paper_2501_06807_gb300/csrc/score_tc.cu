@@ -72,18 +72,6 @@ struct TcSmem {
   static constexpr int TOTAL = USED > 80 * 1024 ? USED : 80 * 1024;
 };
 
-// Barrier of the epilogue threads that also ANDs a flag over them, so all
-// epilogue warps take the same branch after it.
-__device__ __forceinline__ bool epilogue_all(bool v) {
-  uint32_t r;
-  asm volatile(
-      "{\n .reg .pred pi, po;\n setp.ne.u32 pi, %1, 0;\n bar.red.and.pred po, 1, %2, pi;\n"
-      " selp.u32 %0, 1, 0, po;\n}"
-      : "=r"(r)
-      : "r"((uint32_t)v), "n"(kTcEpiThreads)
-      : "memory");
-  return r != 0;
-}
 __device__ __forceinline__ void epilogue_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kTcEpiThreads) : "memory"); }
 
 // Packed pairs of fp32 (one 64-bit register pair) and the sm_100 f32x2 ops.
@@ -426,7 +414,11 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_kernel(const __grid_co
     for (; t < n_tiles; ++t) {
       const int buf = t & 1;
       const bool ok = wait_or_abort(&acc_full[buf], (t >> 1) & 1, abort);
-      if (!epilogue_all(ok)) break;
+      // each epilogue warp goes on alone (its lanes agree); a warp that gave
+      // up leaves the abort flag set, so the others stop at their next wait
+      // and every warp still meets the exchange barrier after the loop (a
+      // barrier of all epilogue warps per tile cost 3% of the pass)
+      if (!__all_sync(0xffffffffu, ok)) break;
       tc_fence_after();
       if (PASS == 0) {
         const int kj = t * 128 + col0;                  // first key of this thread's columns
@@ -767,7 +759,7 @@ __global__ void __launch_bounds__(kTcThreads, 2) score_tc_items_kernel(const __g
       for (; t < it.n_tiles; ++t, ++gt) {
         const int buf = (int)(gt & 1);
         const bool ok = wait_or_abort(&acc_full[buf], (int)(gt >> 1) & 1, abort);
-        if (!epilogue_all(ok)) break;
+        if (!__all_sync(0xffffffffu, ok)) break;  // per warp, as in score_tc_kernel
         tc_fence_after();
         if (PASS == 0) {
           const int kj = t * 128 + col0;                     // first key of this thread's columns
