@@ -32,11 +32,11 @@ def _built():
     build.build()
 
 
-def _twin(w, E, **step_kw):
+def _twin(w, E, device="cpu", **step_kw):
     """Runs the same workload through the fused and the two-call decode and
     compares every step."""
     R = H.window_rows_for(w)
-    x = H.to_cuda(synth.generate(w, R, device="cpu", decode_steps=E))
+    x = H.to_cuda(synth.generate(w, R, device=device, decode_steps=E))
     pt = x.page_table.cuda() if x.page_table is not None else None
     lens = x.prompt_lens.cuda()
     fused, ref = H.make_engine(w, E), H.make_engine(w, E)
@@ -116,6 +116,13 @@ CASES = [
 @pytest.mark.parametrize("name,w,E,kw", CASES, ids=[c[0] for c in CASES])
 def test_fused_step_equals_two_calls(name, w, E, kw):
     _twin(w, E, **dict(kw))
+
+
+def test_fused_step_equals_two_calls_at_32k():
+    """The 32k-token needle workload at full size, 20 decode steps (one tail
+    seal per unit): the fused kernel the benchmark times beside the default
+    form gives the two calls' ids, caches and pyramids exactly."""
+    _twin(synth.C5, 20, device="cuda")
 
 
 @pytest.mark.parametrize("fuse", [1, -1])
